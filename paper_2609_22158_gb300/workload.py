@@ -1,0 +1,332 @@
+"""Seeded synthetic agent-trajectory workloads.
+
+This module only draws random inputs: KV caches, window queries, the layout of
+reasoning steps over the token axis and the per-step trajectory signals.  It
+holds none of StepKV's arithmetic (no saliency, no utility, no selection), so
+both the CUDA path and the CPU oracle can be fed from it.
+
+Conventions (the paper's notation, Sec. 3 "Problem Formulation"):
+
+* a trajectory is the prompt followed by steps k = 0..t-1 (0-based here), each
+  step a contiguous span Thought || Action || Observation that shares one step
+  id (Sec. 3: "each completed step occupies a contiguous span");
+* the first ``n_prompt`` slots are the protected prompt/query tokens
+  (step id -1) and the last ``W`` slots are the observation window, also
+  protected, lying at the end of the last step;
+* K/V per layer are ``[Hkv, T, d]`` bf16, window queries ``[Hq, W, d]`` bf16,
+  both stored here as raw ``uint16`` bf16 bit patterns (round-to-nearest-even
+  from fp32 N(0, 1) draws).
+
+Random streams: one ``numpy.random.PCG64`` per array, spawned from one
+``SeedSequence(seed)`` by a fixed key, so every array is reproducible on its
+own and a trajectory can be regenerated lazily layer by layer.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence, Tuple
+
+import numpy as np
+
+FIELD_PROMPT, FIELD_THOUGHT, FIELD_ACTION, FIELD_OBSERVATION = 0, 1, 2, 3
+
+# Table H defaults are not needed here: this module draws inputs only.
+
+
+def _rng(seed: int, *key: int) -> np.random.Generator:
+    """Independent PCG64 stream for (seed, key...)."""
+    ss = np.random.SeedSequence([int(seed) & 0xFFFFFFFF] + [int(k) & 0xFFFFFFFF for k in key])
+    return np.random.Generator(np.random.PCG64(ss))
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """fp32 -> bf16 bit patterns, round to nearest even (inputs are finite)."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32)
+    rounded = u + (np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1)))
+    return (rounded >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
+
+
+# Stream keys (stable: changing one changes the workload).
+_K_LAYOUT, _K_SIGNALS, _K_KEYS, _K_VALUES, _K_QUERIES, _K_NEEDLE, _K_OUTLIER = 1, 2, 3, 4, 5, 6, 7
+
+
+@dataclass
+class Budget:
+    """KV budget: a keep ratio rho = num/den of the prunable count (Eq. 1), or a fixed count."""
+    mode: str = "ratio"  # "ratio" | "count"
+    num: int = 1
+    den: int = 10
+    count: int = 0
+
+    @staticmethod
+    def ratio(num: int, den: int) -> "Budget":
+        return Budget("ratio", int(num), int(den), 0)
+
+    @staticmethod
+    def fixed(count: int) -> "Budget":
+        return Budget("count", 0, 1, int(count))
+
+
+@dataclass
+class Shape:
+    L: int
+    Hq: int
+    Hkv: int
+    d: int
+    T: int
+    W: int
+    n_sal_layers: int = 3
+
+    @property
+    def G(self) -> int:
+        return self.Hq // self.Hkv
+
+    @property
+    def Ls(self) -> int:
+        return min(self.n_sal_layers, self.L)
+
+
+@dataclass
+class Trajectory:
+    """One agent trajectory at a pruning boundary (after step t = n_steps-1)."""
+    name: str
+    seed: int
+    shape: Shape
+    n_prompt: int
+    step_id: np.ndarray      # int32 [T], -1 for the prompt
+    field: np.ndarray        # int8  [T], FIELD_*
+    prot: np.ndarray         # uint8 [T], 1 = protected (prompt + window)
+    pos: np.ndarray          # int32 [T], original positions
+    valid: np.ndarray        # float32 [n_steps]  valid_k in {0,1}
+    gain: np.ndarray         # float32 [n_steps]  gain_k in [0,1]
+    red: np.ndarray          # float32 [n_steps]  red_k in [0,1]
+    obs_sim: np.ndarray      # float32 [n_steps]  sim(Obs_t, Obs_k)
+    reuse: np.ndarray        # float32 [n_steps]  c_k before this boundary
+    budget: Budget
+    needles: List[Tuple[int, int]] = field(default_factory=list)  # (start, length)
+    outlier_scale: float = 1.0
+    outlier_channels: int = 0
+    kv_std: float = 1.0
+
+    @property
+    def n_steps(self) -> int:
+        return int(self.valid.shape[0])
+
+    @property
+    def T(self) -> int:
+        return self.shape.T
+
+    # ---- lazily generated tensors (bf16 bits) ----
+    def sal_layer_ids(self) -> List[int]:
+        s = self.shape
+        return list(range(s.L - s.Ls, s.L))
+
+    def queries(self, layer: int) -> np.ndarray:
+        """Window queries of one layer, [Hq, W, d] bf16 bits."""
+        s = self.shape
+        g = _rng(self.seed, _K_QUERIES, layer)
+        q = g.standard_normal((s.Hq, s.W, s.d), dtype=np.float32)
+        return f32_to_bf16_bits(q)
+
+    def keys(self, layer: int) -> np.ndarray:
+        """K of one layer, [Hkv, T, d] bf16 bits (needles and outlier channels planted)."""
+        s = self.shape
+        g = _rng(self.seed, _K_KEYS, layer)
+        k = g.standard_normal((s.Hkv, s.T, s.d), dtype=np.float32)
+        if self.kv_std != 1.0:
+            k *= np.float32(self.kv_std)
+        if self.needles:
+            q = bf16_bits_to_f32(self.queries(layer)).reshape(s.Hkv, s.G * s.W, s.d)
+            gn = _rng(self.seed, _K_NEEDLE, layer)
+            for h in range(s.Hkv):
+                u = q[h].astype(np.float64).mean(axis=0)
+                u /= np.linalg.norm(u)
+                for (st, ln) in self.needles:
+                    z = gn.standard_normal((ln, s.d))
+                    z -= np.outer(z @ u, u)
+                    z /= np.linalg.norm(z, axis=1, keepdims=True)
+                    k[h, st:st + ln] = (np.sqrt(s.d) * (0.3 * u[None, :] + np.sqrt(0.91) * z)).astype(np.float32)
+        if self.outlier_channels > 0:
+            go = _rng(self.seed, _K_OUTLIER, layer)
+            for h in range(s.Hkv):
+                ch = go.choice(s.d, size=self.outlier_channels, replace=False)
+                k[h][:, ch] *= np.float32(self.outlier_scale)
+        return f32_to_bf16_bits(k)
+
+    def values(self, layer: int) -> np.ndarray:
+        s = self.shape
+        g = _rng(self.seed, _K_VALUES, layer)
+        return f32_to_bf16_bits(g.standard_normal((s.Hkv, s.T, s.d), dtype=np.float32))
+
+
+def _rescale_lengths(lens: np.ndarray, total: int) -> np.ndarray:
+    """Scale positive integer lengths to sum exactly to `total`, each >= 1 (largest remainder)."""
+    lens = np.asarray(lens, dtype=np.float64).ravel()
+    n = lens.size
+    if total < n:
+        raise ValueError("total smaller than the number of fields")
+    scaled = lens * (total / lens.sum())
+    base = np.maximum(np.floor(scaled).astype(np.int64), 1)
+    rem = total - int(base.sum())
+    frac = scaled - np.floor(scaled)
+    if rem > 0:
+        order = np.argsort(-frac, kind="stable")
+        for i in range(rem):
+            base[order[i % n]] += 1
+    elif rem < 0:
+        order = np.argsort(-base, kind="stable")
+        i = 0
+        while rem < 0:
+            j = order[i % n]
+            if base[j] > 1:
+                base[j] -= 1
+                rem += 1
+            i += 1
+    assert int(base.sum()) == total and base.min() >= 1
+    return base
+
+
+def _assemble(name, seed, shape, n_prompt, field_lens, budget, g_sig, needles_steps=0, **kw) -> Trajectory:
+    """field_lens: int [n_steps, 3] (Th, Act, Obs) lengths summing to T - n_prompt."""
+    T = shape.T
+    n_steps = field_lens.shape[0]
+    step_id = np.full(T, -1, dtype=np.int32)
+    fld = np.zeros(T, dtype=np.int8)
+    pos = n_prompt
+    obs_spans = []
+    for k in range(n_steps):
+        for f in range(3):
+            ln = int(field_lens[k, f])
+            step_id[pos:pos + ln] = k
+            fld[pos:pos + ln] = f + 1
+            if f == 2:
+                obs_spans.append((pos, ln))
+            pos += ln
+    assert pos == T
+    prot = np.zeros(T, dtype=np.uint8)
+    prot[:n_prompt] = 1
+    prot[T - shape.W:] = 1
+    valid = (g_sig.random(n_steps) >= 0.2).astype(np.float32)
+    gain = g_sig.random(n_steps).astype(np.float32)
+    red = g_sig.random(n_steps).astype(np.float32)
+    obs_sim = g_sig.random(n_steps).astype(np.float32)
+    # prior reuse accumulators: any value in [0, number of earlier boundaries that could have credited step k]
+    t = n_steps - 1
+    reuse = (g_sig.random(n_steps) * np.maximum(t - 1 - np.arange(n_steps), 0)).astype(np.float32)
+    reuse[t] = np.float32(0.5)  # stale value: the current step's accumulator must be reset to zero
+    needles = []
+    if needles_steps:
+        g_n = _rng(seed, _K_NEEDLE, 10_000)
+        cand = [s for s in obs_spans[1:1 + needles_steps] if s[1] >= 16]
+        for (st, ln) in cand[:3]:
+            off = int(g_n.integers(0, ln - 16 + 1))
+            needles.append((st + off, 16))
+    traj = Trajectory(name=name, seed=seed, shape=shape, n_prompt=n_prompt, step_id=step_id, field=fld, prot=prot,
+                      pos=np.arange(T, dtype=np.int32), valid=valid, gain=gain, red=red, obs_sim=obs_sim,
+                      reuse=reuse, budget=budget, needles=needles, **kw)
+    return traj
+
+
+def _cycle_steps(g, n_steps, th, act, obs, total, W, obs_log=False) -> np.ndarray:
+    for _ in range(1000):
+        lens = np.empty((n_steps, 3), dtype=np.int64)
+        lens[:, 0] = g.integers(th[0], th[1] + 1, n_steps)
+        lens[:, 1] = g.integers(act[0], act[1] + 1, n_steps)
+        if obs_log:
+            lens[:, 2] = np.round(np.exp(g.uniform(np.log(obs[0]), np.log(obs[1]), n_steps))).astype(np.int64)
+        else:
+            lens[:, 2] = g.integers(obs[0], obs[1] + 1, n_steps)
+        out = _rescale_lengths(lens, total).reshape(n_steps, 3)
+        if out[-1].sum() >= W + 1:
+            return out
+    raise RuntimeError("could not draw a step layout with a last step longer than the window")
+
+
+def tiny(seed: int = 0, budget: Optional[Budget] = None) -> Trajectory:
+    """1 layer, Hq=8/Hkv=2 (GQA 4), d=64, T=2048, W=32, 8 steps of U{100..400} tokens
+    (last step absorbs the remainder), prompt 16, budget 25% of the prunable tokens."""
+    shape = Shape(L=1, Hq=8, Hkv=2, d=64, T=2048, W=32)
+    g = _rng(seed, _K_LAYOUT)
+    n_prompt, total = 16, 2048 - 16
+    for _ in range(1000):
+        lens = g.integers(100, 401, 7)
+        last = total - int(lens.sum())
+        if last >= shape.W + 1 + 3:
+            break
+    step_lens = np.append(lens, last)
+    fl = np.empty((8, 3), dtype=np.int64)
+    for k, sl in enumerate(step_lens):
+        parts = np.array([g.integers(50, 301), g.integers(10, 51), g.integers(200, 2001)])
+        fl[k] = _rescale_lengths(parts, int(sl))
+    return _assemble("tiny", seed, shape, n_prompt, fl, budget or Budget.ratio(1, 4), _rng(seed, _K_SIGNALS))
+
+
+def llama8b_32k(seed: int = 1, budget: Optional[Budget] = None, T: int = 32768, L: int = 32,
+                n_steps: int = 40, needles: bool = True, W: int = 64) -> Trajectory:
+    """Llama-3-8B-shaped single trajectory: L=32, Hq=32/Hkv=8, d=128, T=32768, 40 steps cycling
+    Thought (50-300) / Action (10-50) / Observation (200-2000), rescaled to fill the context;
+    3 needle spans of 16 keys in early Observations aligned with the window queries (cos ~0.3);
+    window 64; budget 10%."""
+    shape = Shape(L=L, Hq=32, Hkv=8, d=128, T=T, W=W)
+    g = _rng(seed, _K_LAYOUT)
+    fl = _cycle_steps(g, n_steps, (50, 300), (10, 50), (200, 2000), T - 16, W)
+    return _assemble("llama8b_32k", seed, shape, 16, fl, budget or Budget.ratio(1, 10), _rng(seed, _K_SIGNALS),
+                     needles_steps=5 if needles else 0)
+
+
+def ragged_batch(seed: int = 2, n_traj: int = 16, budget: Optional[Budget] = None, L: int = 32,
+                 t_lo: int = 8192, t_hi: int = 32768) -> List[Trajectory]:
+    """16 trajectories, T ~ U(8K, 32K), Llama-3-8B head shapes, 24-60 steps each, 4 key channels
+    per (layer, KV head) scaled x8 before bf16 rounding, window 64."""
+    g = _rng(seed, _K_LAYOUT, 999)
+    out = []
+    for b in range(n_traj):
+        T = int(g.integers(t_lo, t_hi + 1))
+        n_steps = int(g.integers(24, 61))
+        shape = Shape(L=L, Hq=32, Hkv=8, d=128, T=T, W=64)
+        sub = seed * 1000 + 17 + b
+        gl = _rng(sub, _K_LAYOUT)
+        fl = _cycle_steps(gl, n_steps, (50, 300), (10, 50), (200, 2000), T - 16, 64)
+        out.append(_assemble(f"ragged{b}", sub, shape, 16, fl, budget or Budget.ratio(1, 10), _rng(sub, _K_SIGNALS),
+                             outlier_scale=8.0, outlier_channels=4))
+    return out
+
+
+def qwen32b_64k(seed: int = 3, budget: Optional[Budget] = None, T: int = 65536, L: int = 64) -> Trajectory:
+    """Qwen2.5-32B-shaped long horizon: L=64, Hq=40/Hkv=8, d=128, T=65536, 120 steps,
+    Observations log-uniform in [16, 4096] tokens before rescaling, window 128, fixed budget 4096."""
+    shape = Shape(L=L, Hq=40, Hkv=8, d=128, T=T, W=128)
+    g = _rng(seed, _K_LAYOUT)
+    fl = _cycle_steps(g, 120, (50, 300), (10, 50), (16, 4096), T - 16, 128, obs_log=True)
+    return _assemble("qwen32b_64k", seed, shape, 16, fl, budget or Budget.fixed(4096), _rng(seed, _K_SIGNALS))
+
+
+def custom(seed: int, L: int, Hq: int, Hkv: int, d: int, T: int, W: int, n_steps: int, n_prompt: int = 16,
+           budget: Optional[Budget] = None, n_sal_layers: int = 3, outlier_channels: int = 0,
+           kv_std: float = 1.0) -> Trajectory:
+    """Arbitrary small shape for parity and edge-case tests (steps cycle the Llama field ranges)."""
+    shape = Shape(L=L, Hq=Hq, Hkv=Hkv, d=d, T=T, W=W, n_sal_layers=n_sal_layers)
+    g = _rng(seed, _K_LAYOUT)
+    total = T - n_prompt
+    if n_steps * 3 > total:
+        raise ValueError("too many steps for T")
+    for _ in range(1000):
+        lens = np.empty((n_steps, 3), dtype=np.int64)
+        lens[:, 0] = g.integers(50, 301, n_steps)
+        lens[:, 1] = g.integers(10, 51, n_steps)
+        lens[:, 2] = g.integers(200, 2001, n_steps)
+        fl = _rescale_lengths(lens, total).reshape(n_steps, 3)
+        if fl[-1].sum() >= min(W, total - 3 * (n_steps - 1)):
+            break
+    return _assemble(f"custom{T}", seed, shape, n_prompt, fl, budget or Budget.ratio(1, 5), _rng(seed, _K_SIGNALS),
+                     outlier_scale=8.0, outlier_channels=outlier_channels, kv_std=kv_std)
+
+
+def decode_queries(seed: int, n_layers: int, Hq: int, d: int, n: int) -> np.ndarray:
+    """Single-token decode queries [n, n_layers, Hq, d] bf16 bits."""
+    g = _rng(seed, _K_QUERIES, 77_777)
+    return f32_to_bf16_bits(g.standard_normal((n, n_layers, Hq, d), dtype=np.float32))

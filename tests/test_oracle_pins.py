@@ -1,0 +1,433 @@
+"""Pins for the CPU oracle: each check ties an oracle function to something other than itself
+(hand-computed tables, closed forms, textbook/library special cases, brute force, invariants).
+
+Every check is written as ``check_*(O)`` taking an oracle-like namespace, so the planted-mistake
+tests at the bottom can run the same check against a deliberately broken copy of the oracle and
+confirm that the check fails.  CPU only.
+"""
+import itertools
+import math
+import os
+import types
+
+import numpy as np
+import pytest
+from scipy.special import expit, softmax
+
+from oracle import stepkv_oracle as REAL
+from paper_2609_22158_gb300 import workload as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _load_table(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+def _bits(x):
+    return wl.f32_to_bf16_bits(np.asarray(x, dtype=np.float32))
+
+
+# ------------------------------------------------------------------ Eqs. 2-4 (hand tables)
+def check_step_utility_table(O):
+    p = O.Params()
+    for case, valid, gain, red, logc, er, es in _load_table("eq2_4_table_h.txt"):
+        valid, gain, red, logc, er, es = map(float, (valid, gain, red, logc, er, es))
+        r = O.completion_score([valid], [gain], [red], p.lam)[0]
+        assert abs(r - er) < 1e-12, (case, r, er)
+        S = O.step_utility([r], [math.expm1(logc)], p)[0]
+        assert abs(S - es) < 1e-12, (case, S, es)
+
+
+def check_s_max_clip(O):
+    p = O.Params(w_c=10.0)
+    S = O.step_utility([2.0], [math.expm1(2.0)], p)[0]      # 0.85*2 + 10*2 = 21.7 -> 8
+    assert S == 8.0
+
+
+def check_reuse_table(O):
+    rows = _load_table("eq3_reuse.txt")
+    c_prev = [float(r[1]) for r in rows]
+    sim = [float(r[2]) for r in rows]
+    exp = [float(r[3]) for r in rows]
+    c = O.reuse_update(c_prev, sim, O.Params().eta)
+    assert np.allclose(c, exp, rtol=0, atol=1e-12), (c, exp)
+    # no similarity vector: only the Phase-1 reset of the new step
+    c2 = O.reuse_update(c_prev, None, 1.5)
+    assert np.allclose(c2, [0.5, 0.0, 2.0, 0.0])
+
+
+def test_step_utility_table():
+    check_step_utility_table(REAL)
+
+
+def test_s_max_clip():
+    check_s_max_clip(REAL)
+
+
+def test_reuse_table():
+    check_reuse_table(REAL)
+
+
+def test_step_utility_invariants():
+    # Eq. 4 range [0, S_max] and c_k >= 0 with increments <= 1 (appendix "Step Score")
+    rng = np.random.default_rng(5)
+    p = REAL.Params()
+    for _ in range(20):
+        n = 50
+        valid = (rng.random(n) > 0.3).astype(float)
+        gain, red, sim = rng.random(n), rng.random(n) * 3, rng.random(n) * 2
+        c0 = rng.random(n) * 5
+        c = REAL.reuse_update(c0, sim, p.eta)
+        assert (c >= 0).all()
+        assert (c[:-1] - c0[:-1] <= 1 + 1e-15).all() and (c[:-1] >= c0[:-1]).all()
+        S = REAL.step_utility(REAL.completion_score(valid, gain, red, p.lam), c, p)
+        assert (S >= 0).all() and (S <= p.s_max).all()
+
+
+# ------------------------------------------------------------------ saliency closed forms
+def _rand_qk(rng, Hkv, G, T, W, d):
+    K = _bits(rng.standard_normal((Hkv, T, d)))
+    Q = _bits(rng.standard_normal((Hkv * G, W, d)))
+    return K, Q
+
+
+def check_zero_keys_closed_form(O):
+    """K == 0: every visible logit is 0, so query w (slot p_w = T-W+w) spreads 1/(p_w+1) uniformly
+    over keys j <= p_w; A[h, j] = sum_w [j <= p_w] / (p_w + 1), for every head and any queries."""
+    rng = np.random.default_rng(1)
+    for (Hkv, G, T, W, d) in [(2, 3, 50, 7, 16), (1, 1, 9, 9, 8), (3, 2, 40, 1, 32)]:
+        K = np.zeros((Hkv, T, d), np.uint16)
+        Q = _bits(rng.standard_normal((Hkv * G, W, d)))
+        A = O.window_attention_saliency(K, Q)
+        exp = np.zeros(T)
+        for w in range(W):
+            pw = T - W + w
+            exp[:pw + 1] += 1.0 / (pw + 1)
+        for h in range(Hkv):
+            assert np.allclose(A[h], exp, rtol=1e-12, atol=1e-15), (Hkv, G, T, W)
+
+
+def check_mass_conservation(O):
+    """Each window query's softmax sums to 1, so sum_j A[h, j] = W (mean over the group)."""
+    rng = np.random.default_rng(2)
+    K, Q = _rand_qk(rng, 2, 4, 300, 13, 32)
+    A = O.window_attention_saliency(K, Q)
+    assert np.allclose(A.sum(axis=1), 13.0, rtol=1e-12)
+
+
+def check_single_query_softmax(O):
+    """W = 1, G = 1: the one query sits at slot T-1 and sees every key, so A[h] is the textbook
+    softmax of q.K^T / sqrt(d) (scipy)."""
+    rng = np.random.default_rng(3)
+    for d in (16, 64, 128):
+        K, Q = _rand_qk(rng, 3, 1, 257, 1, d)
+        A = O.window_attention_saliency(K, Q)
+        Kf, Qf = REAL.bf16_to_f64(K), REAL.bf16_to_f64(Q)
+        for h in range(3):
+            ref = softmax(Kf[h] @ Qf[h, 0] / math.sqrt(d))
+            assert np.allclose(A[h], ref, rtol=1e-12, atol=1e-300)
+
+
+def check_two_key_analytic(O):
+    """T=2, W=1: q=(1,0,0,0), k0=(2,0,0,0), k1=0, d=4: logits 2/sqrt(4)=1 and 0, so
+    A = (sigmoid(1), sigmoid(-1))."""
+    K = _bits([[[2, 0, 0, 0], [0, 0, 0, 0]]])
+    Q = _bits([[[1, 0, 0, 0]]])
+    A = O.window_attention_saliency(K, Q)
+    assert np.allclose(A[0], [expit(1.0), expit(-1.0)], rtol=1e-14)
+
+
+def check_gqa_grouping(O):
+    """q heads h*G..h*G+G-1 read KV head h.  KV head 1 is all zeros, so A[1] must be the uniform
+    closed form whatever its group's queries are; A[0] must be the mean over q heads 0..G-1 of
+    their own softmaxes against K[0] (last query sees everything; W=1)."""
+    rng = np.random.default_rng(4)
+    G, T, d = 2, 64, 16
+    K = np.zeros((2, T, d), np.uint16)
+    K[0] = _bits(rng.standard_normal((T, d)) * 2)
+    Q = _bits(rng.standard_normal((4, 1, d)) * 2)
+    A = O.window_attention_saliency(K, Q)
+    Kf, Qf = REAL.bf16_to_f64(K), REAL.bf16_to_f64(Q)
+    ref0 = np.mean([softmax(Kf[0] @ Qf[g, 0] / math.sqrt(d)) for g in (0, 1)], axis=0)
+    assert np.allclose(A[0], ref0, rtol=1e-12)
+    assert np.allclose(A[1], np.full(T, 1.0 / T), rtol=1e-12)
+
+
+def check_causal_last_key(O):
+    """Key at slot T-1 is visible only to the last window query: A[h, T-1] equals the mean over
+    the group of that query's softmax weight on it."""
+    rng = np.random.default_rng(6)
+    G, T, W, d = 3, 40, 5, 16
+    K, Q = _rand_qk(rng, 1, G, T, W, d)
+    A = O.window_attention_saliency(K, Q)
+    Kf, Qf = REAL.bf16_to_f64(K), REAL.bf16_to_f64(Q)
+    ref = np.mean([softmax(Kf[0] @ Qf[g, W - 1] / math.sqrt(d))[T - 1] for g in range(G)])
+    assert abs(A[0, T - 1] - ref) <= 1e-12 * ref
+
+
+@pytest.mark.parametrize("chk", [check_zero_keys_closed_form, check_mass_conservation, check_single_query_softmax,
+                                 check_two_key_analytic, check_gqa_grouping, check_causal_last_key])
+def test_saliency_pins(chk):
+    chk(REAL)
+
+
+def test_token_saliency_mean_and_normalisation():
+    A = [np.array([[1.0, 2.0, 3.0, 9.0]]), np.array([[3.0, 2.0, 1.0, 9.0]])]
+    T = REAL.token_saliency(A)
+    assert np.allclose(T, [2.0, 2.0, 2.0, 9.0])
+    prunable = np.array([True, True, True, False])       # protected token holds the largest value
+    That = REAL.normalise_saliency(T, prunable, "max")
+    assert np.allclose(That, [1.0, 1.0, 1.0, 4.5])      # max over prunable tokens only
+    assert np.allclose(REAL.normalise_saliency(T, prunable, "none"), T)
+    assert np.allclose(REAL.normalise_saliency(T, np.zeros(4, bool), "max"), T)
+
+
+# ------------------------------------------------------------------ budget (Eq. 1)
+def check_budget(O):
+    assert O.budget_tokens(2000, "ratio", 1, 4) == 500
+    assert O.budget_tokens(32688, "ratio", 1, 10) == 3268
+    assert O.budget_tokens(3, "ratio", 1, 10) == 1          # max(1, floor(0.3))
+    assert O.budget_tokens(0, "ratio", 1, 2) == 0            # nothing prunable: K is empty
+    assert O.budget_tokens(100, "count", count=4096) == 100  # |K| <= N
+    assert O.budget_tokens(10, "ratio", 7, 7) == 10
+    assert O.budget_tokens(9, "ratio", 1, 3) == 3
+
+
+def test_budget():
+    check_budget(REAL)
+
+
+# ------------------------------------------------------------------ global top-B selection
+def _dominance_ok(P, prunable, K):
+    Ks = set(K.tolist())
+    for i in Ks:
+        for j in np.nonzero(prunable)[0]:
+            if j in Ks:
+                continue
+            if not (P[i] > P[j] or (P[i] == P[j] and i < j)):
+                return False
+    return True
+
+
+def check_select_bruteforce(O):
+    """Enumerate every subset of size B of the prunable tokens; exactly one keeps each retained
+    token ahead of each evicted one under (P desc, index asc), and it is the oracle's set."""
+    rng = np.random.default_rng(7)
+    for trial in range(25):
+        N = int(rng.integers(1, 10))
+        P = rng.choice([0.0, 0.25, 0.5, 0.75, 1.0], size=N)   # many ties
+        prunable = rng.random(N) > 0.25
+        idx = np.nonzero(prunable)[0]
+        for B in range(0, len(idx) + 1):
+            valid = [np.array(c, dtype=np.int64) for c in itertools.combinations(idx, B)
+                     if _dominance_ok(P, prunable, np.array(c, dtype=np.int64))]
+            assert len(valid) == 1
+            got = O.select_top(P, prunable, B)
+            assert np.array_equal(got, valid[0]), (P, prunable, B, got, valid[0])
+
+
+def check_select_rank_count(O):
+    """O(N^2) rank counting: token i is kept iff fewer than B prunable tokens beat it
+    (larger P, or equal P and smaller index)."""
+    rng = np.random.default_rng(8)
+    for N in (50, 400, 1500):
+        P = np.round(rng.random(N) * 40) / 40                   # ties
+        prunable = rng.random(N) > 0.1
+        idx = np.nonzero(prunable)[0]
+        Pi = P[idx]
+        beats = (Pi[None, :] > Pi[:, None]) | ((Pi[None, :] == Pi[:, None]) & (idx[None, :] < idx[:, None]))
+        rank = beats.sum(axis=1)
+        for B in (0, 1, len(idx) // 3, len(idx)):
+            exp = np.sort(idx[rank < B])
+            assert np.array_equal(O.select_top(P, prunable, B), exp)
+
+
+def test_select_pins():
+    check_select_bruteforce(REAL)
+    check_select_rank_count(REAL)
+
+
+def test_ablation_special_cases():
+    """Table 3 ablations: alpha=0 ranks by step utility alone (ties inside a step fall to the older
+    tokens); beta=0 is plain saliency top-k."""
+    rng = np.random.default_rng(9)
+    T, n_steps = 300, 6
+    step_id = np.repeat(np.arange(n_steps), T // n_steps).astype(np.int32)
+    prunable = np.ones(T, bool)
+    prunable[:5] = False
+    T_hat = rng.random(T)
+    S = np.array([0.3, 1.5, 0.1, 1.1, 0.9, 0.2])
+    B = 77
+    p0 = REAL.Params(alpha=0.0, beta=1.0)
+    got = REAL.select_top(REAL.priority(T_hat, S, step_id, prunable, p0), prunable, B)
+    # expected: walk steps by descending S, taking tokens in index order
+    exp = []
+    for k in np.argsort(-S, kind="stable"):
+        for i in np.nonzero((step_id == k) & prunable)[0]:
+            if len(exp) < B:
+                exp.append(i)
+    assert np.array_equal(got, np.sort(exp))
+    p1 = REAL.Params(alpha=1.0, beta=0.0)
+    got = REAL.select_top(REAL.priority(T_hat, S, step_id, prunable, p1), prunable, B)
+    idx = np.nonzero(prunable)[0]
+    assert np.array_equal(got, np.sort(idx[np.argsort(-T_hat[idx], kind="stable")[:B]]))
+
+
+def test_priority_range_and_sharing():
+    """Eq. 5 / appendix score range: P in [0, alpha*1 + beta*S_max] with T_hat in [0,1];
+    tokens of one step share S_k, so P differences inside a step are alpha*(T_i - T_j)."""
+    rng = np.random.default_rng(10)
+    p = REAL.Params()
+    T = 200
+    step_id = np.repeat(np.arange(4), 50).astype(np.int32)
+    prunable = np.ones(T, bool)
+    T_hat = rng.random(T)
+    S = np.array([0.0, 8.0, 3.0, 1.0])
+    P = REAL.priority(T_hat, S, step_id, prunable, p)
+    assert (P >= 0).all() and (P <= p.alpha + p.beta * p.s_max).all()
+    i, j = 60, 70
+    assert abs((P[i] - P[j]) - p.alpha * (T_hat[i] - T_hat[j])) < 1e-12
+
+
+# ------------------------------------------------------------------ end-to-end invariants
+def test_boundary_invariants_tiny():
+    tr = wl.tiny(0)
+    s = tr.shape
+    p = REAL.Params()
+    Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+    Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+    out = REAL.compress(Ks, Qs, tr.step_id, tr.prot, tr.valid, tr.gain, tr.red, tr.obs_sim, tr.reuse, p,
+                        tr.budget.mode, tr.budget.num, tr.budget.den, tr.budget.count)
+    prot = tr.prot.astype(bool)
+    N = int((~prot).sum())
+    assert out["N"] == N == 2048 - 16 - 32
+    assert out["B"] == N // 4 == 500
+    kept = out["kept"]
+    assert len(kept) == int(prot.sum()) + out["B"]
+    assert np.all(np.diff(kept) > 0)
+    assert set(np.nonzero(prot)[0]).issubset(set(kept.tolist()))
+    assert out["step_kept"].sum() == out["B"] and out["step_count"].sum() == N
+    assert (out["S"] >= 0).all() and (out["S"] <= p.s_max).all()
+    assert out["reuse"][-1] == 0.0
+    assert abs(out["T_hat"][~prot].max() - 1.0) < 1e-15
+    assert np.allclose(out["A"].sum(axis=2), s.W)
+    V = tr.values(0)
+    C = REAL.compact_rows(V, kept)
+    for r in range(0, len(kept), 37):
+        assert np.array_equal(C[:, r, :], V[:, kept[r], :])
+
+
+# ------------------------------------------------------------------ planted mistakes
+def _mutant(**overrides):
+    ns = types.SimpleNamespace(**{k: getattr(REAL, k) for k in dir(REAL) if not k.startswith("__")})
+    for k, v in overrides.items():
+        setattr(ns, k, v)
+    return ns
+
+
+def _sal_interleaved_groups(K, Q, row_chunk=256):
+    # wrong GQA convention: q head g reads KV head g % Hkv
+    Hkv = K.shape[0]
+    Hq = Q.shape[0]
+    G = Hq // Hkv
+    perm = np.array([h + Hkv * g for h in range(Hkv) for g in range(G)])
+    return REAL.window_attention_saliency(K, Q[perm], row_chunk)
+
+
+def _sal_no_causal(K, Q, row_chunk=256):
+    Kf, Qf = REAL.bf16_to_f64(K), REAL.bf16_to_f64(Q)
+    Hkv, T, d = Kf.shape
+    G = Qf.shape[0] // Hkv
+    W = Qf.shape[1]
+    A = np.zeros((Hkv, T))
+    for h in range(Hkv):
+        s = Qf[h * G:(h + 1) * G].reshape(-1, d) @ Kf[h].T / math.sqrt(d)
+        A[h] = softmax(s, axis=1).sum(axis=0) / G
+    return A
+
+
+def _sal_no_scale(K, Q, row_chunk=256):
+    # logits without the 1/sqrt(d) scale
+    return _scaled(K, Q, 1.0)
+
+
+def _scaled(K, Q, scale):
+    Kf, Qf = REAL.bf16_to_f64(K), REAL.bf16_to_f64(Q)
+    Hkv, T, d = Kf.shape
+    G, W = Qf.shape[0] // Hkv, Qf.shape[1]
+    A = np.zeros((Hkv, T))
+    j = np.arange(T)
+    for h in range(Hkv):
+        rows = Qf[h * G:(h + 1) * G].reshape(G * W, d)
+        p = T - W + np.arange(G * W) % W
+        s = rows @ Kf[h].T * scale
+        s = np.where(j[None] <= p[:, None], s, -np.inf)
+        A[h] = softmax(s, axis=1).sum(axis=0) / G
+    return A
+
+
+def _reuse_uncapped(c_prev, obs_sim, eta):
+    c = np.asarray(c_prev, float).copy()
+    t = len(c) - 1
+    c[t] = 0.0
+    if obs_sim is not None:
+        c[:t] += eta * np.asarray(obs_sim, float)[:t]
+    return c
+
+
+def _reuse_no_reset(c_prev, obs_sim, eta):
+    c = np.asarray(c_prev, float).copy()
+    t = len(c) - 1
+    if obs_sim is not None:
+        for k in range(t):
+            c[k] += min(1.0, eta * obs_sim[k])
+    return c
+
+
+def _utility_no_inner_clip(r, c, p):
+    return REAL.clip(p.w_r * np.asarray(r, float) + p.w_c * np.log1p(np.asarray(c, float)), 0.0, p.s_max)
+
+
+def _utility_log10(r, c, p):
+    return REAL.clip(p.w_r * REAL.clip(np.asarray(r, float), p.r_min, p.r_max)
+                     + p.w_c * np.log10(1 + np.asarray(c, float)), 0.0, p.s_max)
+
+
+def _completion_wrong_sign(valid, gain, red, lam):
+    return np.asarray(valid, float) + np.asarray(gain, float) + lam * np.asarray(red, float)
+
+
+def _select_newer_wins(P, prunable, B):
+    idx = np.nonzero(prunable)[0]
+    order = np.lexsort((-idx, -P[idx]))
+    return np.sort(idx[order[:B]])
+
+
+def _budget_no_floor_one(N, mode, num=1, den=1, count=0):
+    if N <= 0:
+        return 0
+    return min((num * N) // den if mode == "ratio" else count, N)
+
+
+@pytest.mark.parametrize("check, mutant", [
+    (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
+    (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
+    (check_two_key_analytic, _mutant(window_attention_saliency=_sal_no_scale)),
+    (check_reuse_table, _mutant(reuse_update=_reuse_uncapped)),
+    (check_reuse_table, _mutant(reuse_update=_reuse_no_reset)),
+    (check_step_utility_table, _mutant(step_utility=_utility_no_inner_clip)),
+    (check_step_utility_table, _mutant(step_utility=_utility_log10)),
+    (check_step_utility_table, _mutant(completion_score=_completion_wrong_sign)),
+    (check_select_bruteforce, _mutant(select_top=_select_newer_wins)),
+    (check_budget, _mutant(budget_tokens=_budget_no_floor_one)),
+])
+def test_planted_mistake_is_caught(check, mutant):
+    with pytest.raises(AssertionError):
+        check(mutant)

@@ -1,0 +1,474 @@
+"""Benchmark of the fused StepKV compression pass (score -> reduce/fuse -> select -> compact).
+
+Workload (default): one Llama-3-8B-shaped trajectory per GPU -- 32 layers, 32 query / 8 KV heads,
+head dim 128, bf16, T = 32768 cached tokens, 40 reasoning steps, 64-token observation window,
+budget 10% of the prunable tokens -- drawn by the seeded generator (saliency layers, step layout,
+signals) and by torch's seeded device RNG (K/V of the other layers).  Inputs are resident in HBM when
+the timed region starts; an L2 flush (a 512 MB write) runs between timed steps, outside their events.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank compresses its own trajectory
+(independent problems: weak scaling, no collective on the data path); timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "compressed tokens/sec (score+select+compact) at 32K ctx; % HBM roofline"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+# ---------------------------------------------------------------------------------- workload
+def make_traj(args):
+    from paper_2609_22158_gb300 import workload as wl
+    return wl.llama8b_32k(seed=args.seed, T=args.T, L=args.layers)
+
+
+def workload_config(tr, args, n):
+    s = tr.shape
+    b = tr.budget
+    return {
+        "workload": (f"llama3-8b-shaped agent trajectory: L={s.L}, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, T={s.T}, "
+                     f"W={s.W}, {tr.n_steps} steps, saliency from last {s.Ls} layers, budget "
+                     + (f"{b.num}/{b.den} of prunable" if b.mode == "ratio" else f"{b.count} tokens")),
+        "global_batch": n, "seq_len": s.T, "parallelism": f"dp{n} (independent trajectories)",
+        "l2": "flushed between timed steps (512 MB write outside the step events); inputs 4 GB > L2",
+    }
+
+
+class DeviceTraj:
+    """Device-resident inputs/outputs of one trajectory and the C-ABI problem descriptor."""
+
+    def __init__(self, tr, device, seed=1234):
+        import numpy as np
+        import torch
+        from paper_2609_22158_gb300 import binding as B
+        self.tr = tr
+        s = tr.shape
+        gen = torch.Generator(device=device).manual_seed(seed)
+        sal_ids = set(tr.sal_layer_ids())
+
+        def bf16(bits):
+            return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(device)
+
+        self.K = [bf16(tr.keys(l)) if l in sal_ids else
+                  torch.randn((s.Hkv, s.T, s.d), generator=gen, device=device, dtype=torch.bfloat16)
+                  for l in range(s.L)]
+        self.V = [torch.randn((s.Hkv, s.T, s.d), generator=gen, device=device, dtype=torch.bfloat16)
+                  for _ in range(s.L)]
+        self.Q = [bf16(tr.queries(l)) for l in tr.sal_layer_ids()]
+        t = lambda a: torch.from_numpy(a).to(device)
+        self.step_id, self.prot, self.pos = t(tr.step_id), t(tr.prot), t(tr.pos)
+        self.steps = B.StepSignals(t(tr.valid), t(tr.gain), t(tr.red), t(tr.reuse), t(tr.obs_sim),
+                                   torch.empty(tr.n_steps, dtype=torch.float32, device=device))
+        n_prot = int(tr.prot.sum())
+        N = s.T - n_prot
+        B_t = (max(1, tr.budget.num * N // tr.budget.den) if tr.budget.mode == "ratio" else tr.budget.count)
+        self.n_kept_expected = n_prot + min(B_t, N)
+        self.cap = self.n_kept_expected
+        self.K_out = [torch.empty((s.Hkv, self.cap, s.d), dtype=torch.bfloat16, device=device) for _ in range(s.L)]
+        self.V_out = [torch.empty((s.Hkv, self.cap, s.d), dtype=torch.bfloat16, device=device) for _ in range(s.L)]
+        self.out = B.SelectOutputs.allocate(s.T, tr.n_steps, self.cap, device, full=False)
+        self.step_id_out = torch.empty(self.cap, dtype=torch.int32, device=device)
+        self.pos_out = torch.empty(self.cap, dtype=torch.int32, device=device)
+        b = tr.budget
+        self.budget = B.budget_ratio(b.num, b.den) if b.mode == "ratio" else B.budget_count(b.count)
+        self.problem = B.Problem(self.K, self.V, self.Q, s.T, self.step_id, self.prot, self.steps, self.budget,
+                                 self.K_out, self.V_out, self.out, pos_in=self.pos, step_id_out=self.step_id_out,
+                                 pos_out=self.pos_out)
+        self.ws = torch.empty(B.stepkv_workspace_size([self.problem]) + 512, dtype=torch.uint8, device=device)
+        self.status = B.new_status(device)
+
+    def compress(self, params, stream=None):
+        from paper_2609_22158_gb300 import binding as B
+        B.stepkv_compress([self.problem], params, ws=self.ws, status=self.status, stream=stream)
+
+
+def launches_per_pass(tr) -> int:
+    """Kernel launches of one stepkv_compress call (mirrors the library's launch plan)."""
+    s = tr.shape
+    n_pairs = s.Ls * s.Hkv
+    ppg = min(n_pairs, max(1, int(80e6 // (s.T * s.d * 2))))
+    groups = math.ceil(n_pairs / ppg)
+    return 2 * groups + 1 + math.ceil(s.L / 96)
+
+
+def algorithmic_bytes(tr, n_kept):
+    """Bytes the pass must move at minimum (stage by stage)."""
+    s = tr.shape
+    G = s.Hq // s.Hkv
+    score = s.Ls * s.Hkv * s.T * s.d * 2 + s.Ls * s.Hq * s.W * s.d * 2 + s.Ls * s.Hkv * s.T * 4
+    select = s.Ls * s.Hkv * s.T * 4 + s.T * (4 + 1) + n_kept * 4
+    compact = 2 * s.L * s.Hkv * n_kept * s.d * 2 * 2 + n_kept * 4 * 3
+    return {"score": score, "select": select, "compact": compact, "total": score + select + compact}
+
+
+# ---------------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100", "-i", str(gpu_index)], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        self.marks = []
+
+    def mark(self, name):
+        self.marks.append((name, time.time()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    try:
+                        rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+                    except ValueError:
+                        pass
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        loaded = [r for r in rows if r[0] > 0.5 * r[1]] or rows
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[2]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": max(r[1] for r in rows),
+                "samples": len(rows), "reasons": reasons}
+
+
+# ---------------------------------------------------------------------------------- oracle timing
+ORACLE_SNIPPET = r"""
+import json, sys, time
+sys.path.insert(0, {root!r})
+import numpy as np
+from oracle import stepkv_oracle as O
+from paper_2609_22158_gb300 import workload as wl
+tr = wl.llama8b_32k(seed={seed}, T={T}, L={L})
+s = tr.shape
+pairs = {pairs}
+Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+V0 = tr.values(tr.sal_layer_ids()[0])
+G = s.Hq // s.Hkv
+t0 = time.perf_counter()
+A = []
+done = 0
+for li in range(len(Ks)):
+    rows = []
+    for h in range(s.Hkv):
+        if done < pairs:
+            rows.append(O.window_attention_saliency(Ks[li][h:h + 1], Qs[li][h * G:(h + 1) * G])[0])
+            done += 1
+        else:
+            rows.append(np.zeros(s.T))
+    A.append(np.stack(rows))
+t1 = time.perf_counter()
+b = tr.budget
+out = O.stepkv_boundary(A, tr.step_id, tr.prot, tr.valid, tr.gain, tr.red, tr.obs_sim, tr.reuse, O.Params(),
+                        b.mode, b.num, b.den, b.count)
+t2 = time.perf_counter()
+for rep in range({compact_sets}):
+    C = O.compact_rows(V0[rep % s.Hkv:rep % s.Hkv + 1], out["kept"])
+t3 = time.perf_counter()
+print(json.dumps({{"score_s": t1 - t0, "select_s": t2 - t1, "compact_s": t3 - t2, "n_kept": int(len(out["kept"]))}}))
+"""
+
+
+def oracle_pass_seconds(args, pairs: int, compact_sets: int, threads: int = 1):
+    """Run the oracle (as it stands) on a bounded sample in a fresh single-threaded process and scale
+    each stage to the whole pass.  Returns (seconds per full pass, description, threads)."""
+    from paper_2609_22158_gb300 import workload as wl
+    tr = make_traj(args)
+    s = tr.shape
+    code = ORACLE_SNIPPET.format(root=ROOT, seed=args.seed, T=args.T, L=args.layers, pairs=pairs,
+                                 compact_sets=compact_sets)
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS"):
+        env[k] = str(threads)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, "-c", code], stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True,
+                       env=env, timeout=1800)
+    if r.returncode != 0:
+        raise RuntimeError("oracle run failed: " + r.stderr[-2000:])
+    m = json.loads(r.stdout.strip().splitlines()[-1])
+    n_pairs = s.Ls * s.Hkv
+    n_sets = 2 * s.L * s.Hkv
+    total = m["score_s"] * n_pairs / pairs + m["select_s"] + m["compact_s"] * n_sets / compact_sets
+    desc = (f"oracle (numpy fp64, {threads} thread) on the same workload: saliency of {pairs} of {n_pairs} "
+            f"(layer, KV head) pairs, full selection, compaction of {compact_sets} of {n_sets} (layer, tensor, head) "
+            f"row sets; each stage's time scaled to the whole pass")
+    return total, desc, m
+
+
+# ---------------------------------------------------------------------------------- ours
+def run_ours(args):
+    import numpy as np
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if world > 1 else 0)
+    torch.cuda.set_device(dev)
+    from paper_2609_22158_gb300 import build
+    build.build_library()
+    B.load_library()
+
+    tr = make_traj(args)
+    s = tr.shape
+    dt = DeviceTraj(tr, dev, seed=1234 + rank)
+    params = B.Params()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    hbm, _, peak_kind = _peaks()
+
+    sampler = ClockSampler(dev.index if world == 1 else local) if rank == 0 else None
+
+    # warm-up
+    for _ in range(args.warmup):
+        dt.compress(params, stream)
+        flush.fill_(1)
+    torch.cuda.synchronize()
+    st = int(dt.status.item())
+    if st != 0:
+        raise RuntimeError(f"device status {st} after warm-up")
+    n_kept = int(dt.out.n_kept.item())
+    assert n_kept == dt.n_kept_expected, (n_kept, dt.n_kept_expected)
+
+    # timed region: exactly K fused passes, each bracketed by CUDA events on the launching stream
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark("timed_start")
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        dt.compress(params, stream)
+        ev[i][1].record(stream)
+        flush.fill_(i & 0xFF)
+    torch.cuda.synchronize()
+    wall1 = time.perf_counter()
+    if dist:
+        dist.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    ms = sum(step_ms) / len(step_ms)
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    if int(dt.status.item()) != 0:
+        raise RuntimeError(f"device status {int(dt.status.item())} in the timed region")
+    value = world * s.T / (ms * 1e-3)
+
+    # per-stage timing (same shapes, separate entry points, same stream) for the roofline
+    stage = {}
+    if rank == 0 and not args.no_stages:
+        sal = torch.empty((s.Ls, s.Hkv, s.T), dtype=torch.float32, device=dev)
+        ws_s = torch.empty(B.load_library().stepkv_score_workspace_size(s.Ls, s.Hkv, s.Hq, s.T, s.W) + 512,
+                           dtype=torch.uint8, device=dev)
+        ws_sel = torch.empty(B.load_library().stepkv_select_workspace_size(s.Ls * s.Hkv, s.T, tr.n_steps) + 512,
+                             dtype=torch.uint8, device=dev)
+        sel_out = B.SelectOutputs.allocate(s.T, tr.n_steps, dt.cap, dev, full=False)
+        Ksal = [dt.K[l] for l in tr.sal_layer_ids()]
+        reps = max(3, min(args.steps, 20))
+        times = {"score": [], "select": [], "compact": []}
+        for r in range(reps + 2):
+            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            flush.fill_(r & 0xFF)
+            e[0].record(stream)
+            B.stepkv_score(Ksal, dt.Q, s.T, sal=sal, ws=ws_s, status=dt.status, stream=stream)
+            e[1].record(stream)
+            B.stepkv_select(sal, dt.step_id, dt.prot, dt.steps, params, dt.budget, sel_out, ws=ws_sel,
+                            status=dt.status, stream=stream)
+            e[2].record(stream)
+            flush.fill_((r + 1) & 0xFF)
+            e3 = torch.cuda.Event(enable_timing=True)
+            e3.record(stream)
+            B.stepkv_compact(dt.K, dt.V, s.T, sel_out.kept_idx, sel_out.n_kept, dt.cap, dt.K_out, dt.V_out,
+                             dt.step_id, dt.pos, dt.step_id_out, dt.pos_out, status=dt.status, stream=stream)
+            e[3].record(stream)
+            torch.cuda.synchronize()
+            if r >= 2:
+                times["score"].append(e[0].elapsed_time(e[1]))
+                times["select"].append(e[1].elapsed_time(e[2]))
+                times["compact"].append(e3.elapsed_time(e[3]))
+        stage = {k: statistics.median(v) * 1e3 for k, v in times.items()}  # us
+
+    # e2e: host buffers through the same public call; H2D of every input and D2H of the result per step
+    e2e = None
+    if not args.no_e2e:
+        host_in = [t.cpu().pin_memory() for t in dt.K + dt.V + dt.Q]
+        dev_in = dt.K + dt.V + dt.Q
+        host_small = [x.cpu().pin_memory() for x in (dt.step_id, dt.prot, dt.pos)]
+        dev_small = [dt.step_id, dt.prot, dt.pos]
+        host_out = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.K_out + dt.V_out]
+        host_idx = torch.empty(dt.cap + 1, dtype=torch.int32).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in host_in + host_small)
+        d2h = sum(t.numel() * t.element_size() for t in host_out) + host_idx.numel() * 4
+        k2 = max(1, min(args.steps, args.e2e_steps))
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(k2):
+            for h, d in zip(host_in + host_small, dev_in + dev_small):
+                d.copy_(h, non_blocking=True)
+            dt.compress(params, stream)
+            for h, d in zip(host_out, dt.K_out + dt.V_out):
+                h.copy_(d, non_blocking=True)
+            host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
+            host_idx[dt.cap:].copy_(dt.out.n_kept, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1) / k2
+        if dist:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        assert int(host_idx[dt.cap].item()) == dt.n_kept_expected
+        e2e = {"value": world * s.T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": k2}
+
+    clocks = sampler.stop() if sampler else None
+    if dist:
+        dist.barrier()
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+
+    ab = algorithmic_bytes(tr, n_kept)
+    roof = None
+    if stage:
+        comp_gbs = ab["compact"] / (stage["compact"] * 1e-6) / 1e9
+        roof = {"kernel": "compact_kernel (stage 5: retained K/V row gather, all 32 layers)", "bound": "hbm",
+                "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
+                "peak_source": f"{peak_kind} hbm_gbs (burst copy)", "traffic": args.compact_traffic,
+                "algorithmic_bytes_per_launch": ab["compact"], "launch_us": round(stage["compact"], 2)}
+    pass_gbs = ab["total"] / (ms * 1e-3) / 1e9
+    cpu = None
+    if not args.no_cpu_baseline:
+        secs, desc, _ = oracle_pass_seconds(args, pairs=args.oracle_pairs, compact_sets=args.oracle_compact_sets)
+        cpu = {"value": s.T / secs, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
+               "seconds_per_pass": round(secs, 3)}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded generator + torch device RNG; no datasets or model weights)",
+        "config": workload_config(tr, args, world),
+        "roofline": roof,
+        "pass_hbm": {"algorithmic_bytes": ab["total"], "achieved_gbs": round(pass_gbs, 1),
+                     "frac_of_measured": round(pass_gbs / hbm, 4), "frac_of_nominal_8tbs": round(pass_gbs / 8000, 4)},
+        "stages_us": {k: round(v, 2) for k, v in stage.items()} if stage else None,
+        "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": launches_per_pass(tr) * args.steps,
+        "clocks": clocks,
+        "wall_s_timed_region": round(wall1 - wall0, 4),
+        "step_ms_min_max": [round(min(step_ms), 4), round(max(step_ms), 4)],
+        "n_kept": n_kept,
+    }
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+# ---------------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    """The oracle as it stands on the host cores, same workload/metric; each step a bounded sample."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    tr = make_traj(args)
+    s = tr.shape
+    times = []
+    desc = ""
+    for i in range(args.warmup + args.steps):
+        secs, desc, _ = oracle_pass_seconds(args, pairs=args.ref_pairs, compact_sets=args.ref_compact_sets)
+        if i >= args.warmup:
+            times.append(secs)
+    sec = sum(times) / len(times)
+    value = s.T / sec
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
+        "config": workload_config(tr, args, 1),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--seed", type=int, default=1)
+    ap.add_argument("--T", type=int, default=32768)
+    ap.add_argument("--layers", type=int, default=32)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-stages", action="store_true")
+    ap.add_argument("--oracle-pairs", type=int, default=24)
+    ap.add_argument("--oracle-compact-sets", type=int, default=16)
+    ap.add_argument("--ref-pairs", type=int, default=2)
+    ap.add_argument("--ref-compact-sets", type=int, default=4)
+    ap.add_argument("--compact-traffic", type=float, default=None,
+                    help="dram bytes (read+write) per compaction launch from an ncu capture of this workload")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,236 @@
+/*
+ * stepkv.h -- C ABI of the StepKV compression pass on GB300 (sm_103a).
+ *
+ * StepKV (arXiv 2609.22158) compresses an agent's KV cache at each completed-step boundary
+ * (Sec. 3, Eq. 1): every prunable token i gets a retention priority P_i = alpha*T_i + beta*S_k
+ * (Eq. 5), where T_i is attention-based token saliency and S_k the utility of the step k that
+ * produced token i (Eqs. 2-4, Algorithm 1), and the B_t highest-priority tokens are kept.
+ *
+ * The pass has five stages, all computed by this library's CUDA kernels:
+ *   1. score   -- T_i from the observation-window queries against all cached keys (stepkv_score)
+ *   2. reduce  -- per-step aggregation of saliency, keyed by each token's step id
+ *   3. fuse    -- Eqs. 2-5 (stages 2-5 of this list are in stepkv_select)
+ *   4. select  -- exact global top-B over the prunable tokens under the budget
+ *   5. compact -- gather of the retained K/V rows into a dense cache (stepkv_compact)
+ * stepkv_compress runs all five for one or more trajectories.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Pointers are DEVICE pointers unless a comment says "host".  Arrays of per-layer tensors are
+ *    HOST arrays of device pointers.
+ *  - bf16 tensors are passed as void* holding IEEE bfloat16 values.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream).  Every call
+ *    only enqueues work on `stream` and returns; nothing synchronises the host.
+ *  - The library never allocates or frees memory and keeps no state between calls; scratch
+ *    memory is the caller's `ws` (size from the matching *_workspace_size function, 256-byte
+ *    aligned).  Calls on different streams with different workspaces may run concurrently.
+ *  - Errors: argument problems are detected on the host and returned (STEPKV_EINVAL,
+ *    STEPKV_EUNSUPPORTED, STEPKV_ENOSPACE) before anything is enqueued.  A failed launch returns
+ *    STEPKV_ECUDA.  Data-dependent problems found on the device (a step id out of range, kept_cap
+ *    too small, a bounded device-side wait that ran out) are written to *dev_status with
+ *    atomicCAS(0 -> code): the FIRST error wins and later calls never clear it.  dev_status is a
+ *    device int32 the caller zeroes once and reads after its own synchronisation.  Kernels that
+ *    hit such an error skip the affected work and return; they never trap.
+ *  - Token order: slots 0..T-1 of a layer's cache.  Retained slots are reported in ascending
+ *    original order, so with the protected prompt as a prefix the compacted cache is exactly
+ *    C_prot || C_traj[K] of Eq. 1.
+ *  - GQA: query head g reads KV head g / G, G = Hq / Hkv.
+ */
+#ifndef STEPKV_H
+#define STEPKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define STEPKV_API __attribute__((visibility("default")))
+#else
+#define STEPKV_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  STEPKV_OK = 0,
+  STEPKV_EINVAL = 1,        /* invalid argument (host check, nothing enqueued) */
+  STEPKV_ECUDA = 2,         /* a CUDA runtime call or launch failed */
+  STEPKV_ENOSPACE = 3,      /* workspace too small (host) / kept_cap < n_kept (device) */
+  STEPKV_EUNSUPPORTED = 4,  /* shape or alignment outside what the kernels handle */
+  STEPKV_EDATA = 5,         /* device: invalid data (step id out of [0, n_steps), bad kept index) */
+  STEPKV_ETIMEOUT = 6       /* device: a bounded wait inside a kernel expired */
+} stepkv_status_t;
+
+enum { STEPKV_NORM_MAX = 0, STEPKV_NORM_NONE = 1 };
+enum { STEPKV_BUDGET_RATIO = 0, STEPKV_BUDGET_COUNT = 1 };
+
+/* Hyper-parameters of Eqs. 2-5 (Table H defaults from stepkv_default_params). */
+typedef struct {
+  float lambda;   /* redundancy penalty in r_k (Eq. 2) */
+  float w_r;      /* completion weight (Eq. 4) */
+  float w_c;      /* reuse weight (Eq. 4) */
+  float r_min;    /* inner clip of r_k (Eq. 4) */
+  float r_max;
+  float s_max;    /* outer clip of S_k (Eq. 4) */
+  float eta;      /* reuse update scale (Eq. 3) */
+  float alpha;    /* token-saliency weight (Eq. 5) */
+  float beta;     /* step-utility weight (Eq. 5) */
+  int32_t sal_norm; /* STEPKV_NORM_MAX: T_i divided by its maximum over prunable tokens (appendix,
+                       "H_i normalised to [0, H_max]"); STEPKV_NORM_NONE: T_i used as is */
+} stepkv_params_t;
+
+/* KV budget (Eq. 1).  RATIO: B_t = max(1, floor(ratio_num * N_t / ratio_den)) of the N_t
+ * prunable tokens (exact integer arithmetic); COUNT: B_t = count.  In both cases |K| = min(B_t, N_t),
+ * and |K| = 0 when N_t = 0.  Protected tokens are kept on top of the budget. */
+typedef struct {
+  int32_t mode;
+  int32_t ratio_num;
+  int32_t ratio_den;
+  int32_t count;
+} stepkv_budget_t;
+
+/* Per-step trajectory signals at the boundary after step t = n_steps-1 (0-based step ids).
+ * All arrays are device float32 [n_steps].  valid/gain/red are the inputs of Eq. 2 for every step
+ * (they do not change once a step is final); obs_sim[k] = sim(Obs_t, Obs_k) drives Eq. 3 for k < t
+ * (obs_sim[t] is ignored; NULL = no Phase-2 update).  reuse_in holds c_k from the previous boundary
+ * (reuse_in[t] is ignored: Algorithm 1 Phase 1 sets c_t = 0); reuse_out receives the updated c_k
+ * (may alias reuse_in; NULL = not written). */
+typedef struct {
+  int32_t n_steps;
+  const float* valid;
+  const float* gain;
+  const float* red;
+  const float* obs_sim;
+  const float* reuse_in;
+  float* reuse_out;
+} stepkv_steps_t;
+
+/* Outputs of the selection stage.  kept_idx/n_kept are required, the rest may be NULL. */
+typedef struct {
+  int32_t* kept_idx;      /* [kept_cap]: retained slots (protected + selected), ascending */
+  int32_t kept_cap;       /* capacity of kept_idx (and of the compacted caches) */
+  int32_t* n_kept;        /* [1]: number of retained slots = n_protected + min(B_t, N_t) */
+  int32_t* n_budget;      /* [2] or NULL: (N_t, B_t) */
+  float* priority;        /* [T] or NULL: P_i (Eq. 5); -inf for protected tokens */
+  float* token_sal;       /* [T] or NULL: normalised saliency T_i used in Eq. 5 */
+  float* step_util;       /* [n_steps] or NULL: S_k (Eq. 4) after this boundary's update */
+  int32_t* step_count;    /* [n_steps] or NULL: prunable tokens per step */
+  float* step_sal_sum;    /* [n_steps] or NULL: sum of T_i over the step's prunable tokens */
+  float* step_sal_max;    /* [n_steps] or NULL: max of T_i over the step's prunable tokens */
+  int32_t* step_kept;     /* [n_steps] or NULL: retained prunable tokens per step */
+} stepkv_select_out_t;
+
+/* One trajectory for stepkv_compress. */
+typedef struct {
+  int32_t L, Hkv, Hq, d, T, W;
+  int32_t n_sal_layers;            /* saliency from layers L-n_sal_layers .. L-1 (Table H: last 3) */
+  const void* const* K;            /* host [L]: K of layer l, [Hkv][rows >= T][d] bf16 */
+  const void* const* V;            /* host [L]: V of layer l, same layout */
+  int64_t kv_head_stride;          /* elements between KV heads (>= T*d, multiple of 8) */
+  const void* const* Q;            /* host [n_sal_layers]: window queries of layer L-n_sal_layers+i,
+                                      [Hq][W][d] bf16; query w sits at slot T-W+w */
+  int64_t q_head_stride;           /* elements between query heads (>= W*d, multiple of 8) */
+  const int32_t* step_id;          /* [T]: step of each token; ignored for protected tokens */
+  const uint8_t* prot;             /* [T]: 1 = protected (never pruned, always kept) */
+  const int32_t* pos_in;           /* [T] or NULL: original position of each slot */
+  stepkv_steps_t steps;
+  stepkv_budget_t budget;
+  void* const* K_out;              /* host [L]: compacted K, [Hkv][rows >= kept_cap][d] */
+  void* const* V_out;              /* host [L] */
+  int64_t out_head_stride;         /* elements (>= kept_cap*d, multiple of 8) */
+  int32_t* step_id_out;            /* [kept_cap] or NULL: step_id of each retained slot */
+  int32_t* pos_out;                /* [kept_cap] or NULL: pos_in (or the slot index) of each retained slot */
+  stepkv_select_out_t sel;
+} stepkv_problem_t;
+
+/* Table H defaults (appendix "Implementation Details"): lambda=0.3, w_r=0.85, w_c=0.15, r_min=-1,
+ * r_max=2, S_max=8, eta=1.5, alpha=0.2, beta=0.8, max-normalised saliency. */
+STEPKV_API void stepkv_default_params(stepkv_params_t* p);
+
+/* Static text for a status code (never NULL). */
+STEPKV_API const char* stepkv_status_string(int32_t status);
+
+/* Library ABI version (major*1000 + minor). */
+STEPKV_API int32_t stepkv_version(void);
+
+/* Message of the last CUDA error seen by this thread inside the library ("" if none). */
+STEPKV_API const char* stepkv_last_cuda_error(void);
+
+/* ---------------------------------------------------------------------------------------------
+ * Stage 1: token saliency (Sec. 4.2 "Token Saliency"; the attention-based T_i collected from the
+ * observation-window queries of the last layers, Table H).
+ *
+ * For each of n_layers layers, KV head h and key slot j:
+ *   sal[l][h][j] = (1/G) * sum_{g = hG}^{hG+G-1} sum_{w < W} softmax_{j' <= T-W+w}( q_{l,g,w} . k_{l,h,j'} / sqrt(d) )[j]
+ * i.e. a causal scaled softmax of each window query over the whole visible context (protected
+ * tokens included), summed over the window queries and averaged over the GQA group.
+ *
+ *  K[l]   host array of device pointers, [Hkv][rows][d] bf16 with head stride k_head_stride
+ *         elements; rows >= T.  Base 16-byte aligned, k_head_stride % 8 == 0.
+ *  Q[l]   host array, [Hq][W][d] bf16 with head stride q_head_stride (% 8 == 0).
+ *  sal    [n_layers][Hkv][T] float32 output.
+ *  Supported: d in {64, 128}; Hq % Hkv == 0; 1 <= W <= T; W <= 4096; 1 <= n_layers <= 8.
+ *  Work: two tensor-core passes over K (row statistics, then saliency).
+ */
+STEPKV_API size_t stepkv_score_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t T, int32_t W);
+STEPKV_API stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_head_stride,
+                             const void* const* Q, int64_t q_head_stride,
+                             int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
+                             float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Stages 2-4: step reduction, fusion and selection (Eqs. 1-5, Algorithm 1 Phases 1-3).
+ *
+ *  sal       [n_sal][T] float32: saliency rows (e.g. stepkv_score's n_layers*Hkv rows);
+ *            T_i = mean over the n_sal rows, then normalised per params->sal_norm.
+ *  step_id   [T] int32: step of each token (must lie in [0, n_steps) for prunable tokens; a
+ *            violation sets STEPKV_EDATA and no selection is written).
+ *  prot      [T] uint8: 1 = protected.
+ *  steps, params, budget: host structs (device arrays inside steps).
+ *  out       host struct of device output pointers (see stepkv_select_out_t).
+ *  Ranking: (P_i descending, slot index ascending) -- on equal priority the older token wins.
+ *  Supported: 1 <= T <= 262144, 1 <= n_steps <= 65536, n_sal >= 1.
+ */
+STEPKV_API size_t stepkv_select_workspace_size(int32_t n_sal, int32_t T, int32_t n_steps);
+STEPKV_API stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T,
+                              const int32_t* step_id, const uint8_t* prot,
+                              const stepkv_steps_t* steps, const stepkv_params_t* params,
+                              const stepkv_budget_t* budget, const stepkv_select_out_t* out,
+                              void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Stage 5: compaction (Eq. 1, C_hat = C_prot || C_traj[K]).
+ *
+ * For every layer l < n_layers, KV head h and r < *n_kept:
+ *   K_out[l][h][r][:] = K_in[l][h][kept_idx[r]][:]   (same for V; bit-exact copies)
+ *   step_id_out[r] = step_id_in[kept_idx[r]],  pos_out[r] = pos_in ? pos_in[kept_idx[r]] : kept_idx[r]
+ *  n_kept is read on the device (no host synchronisation); *n_kept > kept_cap or a kept index
+ *  outside [0, T) sets STEPKV_ENOSPACE / STEPKV_EDATA and skips the bad rows.
+ *  V_in/V_out may be NULL (keys only); step/pos pointers may be NULL.
+ *  Rows are d bf16 values; d*2 bytes must be a multiple of 16; bases 16-byte aligned; in/out head
+ *  strides % 8 == 0.  In-place compaction (K_out == K_in) is not supported.
+ */
+STEPKV_API stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
+                               int64_t in_head_stride, int32_t Hkv, int32_t d, int32_t T,
+                               const int32_t* kept_idx, const int32_t* n_kept, int32_t kept_cap,
+                               void* const* K_out, void* const* V_out, int64_t out_head_stride,
+                               const int32_t* step_id_in, const int32_t* pos_in,
+                               int32_t* step_id_out, int32_t* pos_out,
+                               int32_t* dev_status, void* stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * The fused pass (score -> reduce/fuse -> select -> compact) for n_traj independent trajectories
+ * (one pruning boundary each, Algorithm 1).  probs is a host array; all trajectories run on
+ * `stream` in order, sharing `ws` (size from stepkv_compress_workspace_size over the same array).
+ */
+STEPKV_API size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj);
+STEPKV_API stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj,
+                                const stepkv_params_t* params, void* ws, size_t ws_bytes,
+                                int32_t* dev_status, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STEPKV_H */

@@ -1,0 +1,430 @@
+"""ctypes binding of libstepkv.so (C ABI in include/stepkv.h).
+
+Argument marshalling only: shapes and dtypes are checked, torch tensors are turned into device
+pointers, and every step of the pass runs in the library's CUDA kernels.  PyTorch provides device
+memory and streams.  There is no fallback: if the library is missing or a call fails, an exception
+is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass, field
+from typing import List, Optional, Sequence
+
+_PKG_DIR = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG_DIR, "libstepkv.so")
+
+STEPKV_OK, STEPKV_EINVAL, STEPKV_ECUDA, STEPKV_ENOSPACE, STEPKV_EUNSUPPORTED, STEPKV_EDATA, STEPKV_ETIMEOUT = range(7)
+NORM_MAX, NORM_NONE = 0, 1
+BUDGET_RATIO, BUDGET_COUNT = 0, 1
+
+
+class StepKVError(RuntimeError):
+    def __init__(self, code: int, where: str, detail: str = ""):
+        self.code = code
+        super().__init__(f"{where}: status {code} ({status_string(code)}){' ' + detail if detail else ''}")
+
+
+# ----------------------------------------------------------------------------- C structs
+class CParams(ctypes.Structure):
+    _fields_ = [("lambda_", ctypes.c_float), ("w_r", ctypes.c_float), ("w_c", ctypes.c_float),
+                ("r_min", ctypes.c_float), ("r_max", ctypes.c_float), ("s_max", ctypes.c_float),
+                ("eta", ctypes.c_float), ("alpha", ctypes.c_float), ("beta", ctypes.c_float),
+                ("sal_norm", ctypes.c_int32)]
+
+
+class CBudget(ctypes.Structure):
+    _fields_ = [("mode", ctypes.c_int32), ("ratio_num", ctypes.c_int32), ("ratio_den", ctypes.c_int32),
+                ("count", ctypes.c_int32)]
+
+
+class CSteps(ctypes.Structure):
+    _fields_ = [("n_steps", ctypes.c_int32), ("valid", ctypes.c_void_p), ("gain", ctypes.c_void_p),
+                ("red", ctypes.c_void_p), ("obs_sim", ctypes.c_void_p), ("reuse_in", ctypes.c_void_p),
+                ("reuse_out", ctypes.c_void_p)]
+
+
+class CSelOut(ctypes.Structure):
+    _fields_ = [("kept_idx", ctypes.c_void_p), ("kept_cap", ctypes.c_int32), ("n_kept", ctypes.c_void_p),
+                ("n_budget", ctypes.c_void_p), ("priority", ctypes.c_void_p), ("token_sal", ctypes.c_void_p),
+                ("step_util", ctypes.c_void_p), ("step_count", ctypes.c_void_p), ("step_sal_sum", ctypes.c_void_p),
+                ("step_sal_max", ctypes.c_void_p), ("step_kept", ctypes.c_void_p)]
+
+
+class CProblem(ctypes.Structure):
+    _fields_ = [("L", ctypes.c_int32), ("Hkv", ctypes.c_int32), ("Hq", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("T", ctypes.c_int32), ("W", ctypes.c_int32), ("n_sal_layers", ctypes.c_int32),
+                ("K", ctypes.c_void_p), ("V", ctypes.c_void_p), ("kv_head_stride", ctypes.c_int64),
+                ("Q", ctypes.c_void_p), ("q_head_stride", ctypes.c_int64),
+                ("step_id", ctypes.c_void_p), ("prot", ctypes.c_void_p), ("pos_in", ctypes.c_void_p),
+                ("steps", CSteps), ("budget", CBudget),
+                ("K_out", ctypes.c_void_p), ("V_out", ctypes.c_void_p), ("out_head_stride", ctypes.c_int64),
+                ("step_id_out", ctypes.c_void_p), ("pos_out", ctypes.c_void_p), ("sel", CSelOut)]
+
+
+_lib = None
+
+# (name, restype, argtypes) for every function declared in include/stepkv.h
+_VP, _I32, _I64, _SZ = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+SIGNATURES = {
+    "stepkv_default_params": (None, [ctypes.POINTER(CParams)]),
+    "stepkv_status_string": (ctypes.c_char_p, [_I32]),
+    "stepkv_version": (_I32, []),
+    "stepkv_last_cuda_error": (ctypes.c_char_p, []),
+    "stepkv_score_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
+    "stepkv_score": (_I32, [_I32, _VP, _I64, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ, _VP, _VP]),
+    "stepkv_select_workspace_size": (_SZ, [_I32, _I32, _I32]),
+    "stepkv_select": (_I32, [_VP, _I32, _I32, _VP, _VP, ctypes.POINTER(CSteps), ctypes.POINTER(CParams),
+                             ctypes.POINTER(CBudget), ctypes.POINTER(CSelOut), _VP, _SZ, _VP, _VP]),
+    "stepkv_compact": (_I32, [_I32, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _VP, _I32, _VP, _VP, _I64, _VP, _VP,
+                              _VP, _VP, _VP, _VP]),
+    "stepkv_compress_workspace_size": (_SZ, [ctypes.POINTER(CProblem), _I32]),
+    "stepkv_compress": (_I32, [ctypes.POINTER(CProblem), _I32, ctypes.POINTER(CParams), _VP, _SZ, _VP, _VP]),
+}
+
+
+def load_library(path: Optional[str] = None):
+    """Load libstepkv.so (built in-tree by paper_2609_22158_gb300.build); raises if it is missing."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise StepKVError(STEPKV_ECUDA, "load_library",
+                          f"{p} not found: build it with `python -m paper_2609_22158_gb300.build`")
+    lib = ctypes.CDLL(p)
+    for name, (res, args) in SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def status_string(code: int) -> str:
+    try:
+        return load_library().stepkv_status_string(int(code)).decode()
+    except Exception:  # library not built yet
+        return "status %d" % code
+
+
+@dataclass
+class Params:
+    """Table H defaults (appendix "Implementation Details")."""
+    lam: float = 0.3
+    w_r: float = 0.85
+    w_c: float = 0.15
+    r_min: float = -1.0
+    r_max: float = 2.0
+    s_max: float = 8.0
+    eta: float = 1.5
+    alpha: float = 0.2
+    beta: float = 0.8
+    sal_norm: int = NORM_MAX
+
+    def c(self) -> CParams:
+        return CParams(self.lam, self.w_r, self.w_c, self.r_min, self.r_max, self.s_max, self.eta, self.alpha,
+                       self.beta, self.sal_norm)
+
+
+def default_params() -> Params:
+    cp = CParams()
+    load_library().stepkv_default_params(ctypes.byref(cp))
+    return Params(cp.lambda_, cp.w_r, cp.w_c, cp.r_min, cp.r_max, cp.s_max, cp.eta, cp.alpha, cp.beta, cp.sal_norm)
+
+
+# ----------------------------------------------------------------------------- helpers
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream_handle(stream) -> int:
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _check(code: int, where: str):
+    if code != STEPKV_OK:
+        detail = ""
+        if code == STEPKV_ECUDA:
+            detail = load_library().stepkv_last_cuda_error().decode()
+        raise StepKVError(code, where, detail)
+
+
+def _need(t, dtype, name, ndim=None):
+    torch = _torch()
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if ndim is not None and t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims")
+    return t
+
+
+def _rows_layout(ts: Sequence, name: str):
+    """[H, rows, d] bf16 tensors with unit stride in d and dense rows; returns (head_stride, rows)."""
+    torch = _torch()
+    hs = None
+    for i, t in enumerate(ts):
+        _need(t, torch.bfloat16, f"{name}[{i}]", 3)
+        H, R, d = t.shape
+        if t.stride(2) != 1 or (R > 1 and t.stride(1) != d):
+            raise ValueError(f"{name}[{i}] rows must be dense (stride(1) == d, stride(2) == 1)")
+        s = t.stride(0) if H > 1 else R * d
+        if hs is None:
+            hs = s
+        elif hs != s:
+            raise ValueError(f"all {name} tensors must share one head stride")
+    return hs
+
+
+def _ptr_array(ts) -> ctypes.Array:
+    arr = (ctypes.c_void_p * max(1, len(ts)))()
+    for i, t in enumerate(ts):
+        arr[i] = t.data_ptr()
+    return arr
+
+
+def new_status(device=None):
+    torch = _torch()
+    return torch.zeros(1, dtype=torch.int32, device=device or "cuda")
+
+
+def _workspace(nbytes: int, ws, device):
+    torch = _torch()
+    if ws is None:
+        ws = torch.empty(max(nbytes, 256) + 256, dtype=torch.uint8, device=device)
+    if ws.numel() < nbytes:
+        raise ValueError(f"workspace too small: {ws.numel()} < {nbytes}")
+    return ws
+
+
+def _aligned_ws(ws):
+    off = (-ws.data_ptr()) % 256
+    return ws.data_ptr() + off, ws.numel() - off
+
+
+# ----------------------------------------------------------------------------- stage 1
+def stepkv_score(K: Sequence, Q: Sequence, T: int, W: Optional[int] = None, sal=None, ws=None, status=None,
+                 stream=None):
+    """Window-attention saliency of len(K) layers: returns sal [n_layers, Hkv, T] float32.
+    K[l]: [Hkv, rows >= T, d] bf16; Q[l]: [Hq, W, d] bf16 (query w at slot T-W+w)."""
+    torch = _torch()
+    lib = load_library()
+    n = len(K)
+    if n != len(Q) or n == 0:
+        raise ValueError("K and Q need the same non-zero number of layers")
+    ks = _rows_layout(K, "K")
+    qs = _rows_layout(Q, "Q")
+    Hkv, _, d = K[0].shape
+    Hq, Wq, dq = Q[0].shape
+    W = Wq if W is None else W
+    if dq != d:
+        raise ValueError("K and Q head dims differ")
+    dev = K[0].device
+    if sal is None:
+        sal = torch.empty((n, Hkv, T), dtype=torch.float32, device=dev)
+    _need(sal, torch.float32, "sal")
+    need = lib.stepkv_score_workspace_size(n, Hkv, Hq, T, W)
+    ws = _workspace(need + 256, ws, dev)
+    wp, wn = _aligned_ws(ws)
+    status = status if status is not None else new_status(dev)
+    kp, qp = _ptr_array(K), _ptr_array(Q)
+    code = lib.stepkv_score(n, ctypes.cast(kp, ctypes.c_void_p), ks, ctypes.cast(qp, ctypes.c_void_p), qs, Hkv, Hq, d,
+                            T, W, sal.data_ptr(), wp, wn, status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_score")
+    return sal
+
+
+# ----------------------------------------------------------------------------- stages 2-4
+@dataclass
+class StepSignals:
+    """Per-step trajectory signals (device float32 [n_steps]); see stepkv_steps_t."""
+    valid: object
+    gain: object
+    red: object
+    reuse_in: object
+    obs_sim: object = None
+    reuse_out: object = None
+
+    @property
+    def n_steps(self) -> int:
+        return int(self.valid.numel())
+
+    def c(self) -> CSteps:
+        torch = _torch()
+        for nm in ("valid", "gain", "red", "reuse_in"):
+            _need(getattr(self, nm), torch.float32, nm, 1)
+        return CSteps(self.n_steps, _ptr(self.valid), _ptr(self.gain), _ptr(self.red), _ptr(self.obs_sim),
+                      _ptr(self.reuse_in), _ptr(self.reuse_out))
+
+
+def budget_ratio(num: int, den: int) -> CBudget:
+    return CBudget(BUDGET_RATIO, int(num), int(den), 0)
+
+
+def budget_count(n: int) -> CBudget:
+    return CBudget(BUDGET_COUNT, 0, 1, int(n))
+
+
+@dataclass
+class SelectOutputs:
+    kept_idx: object
+    n_kept: object
+    n_budget: object = None
+    priority: object = None
+    token_sal: object = None
+    step_util: object = None
+    step_count: object = None
+    step_sal_sum: object = None
+    step_sal_max: object = None
+    step_kept: object = None
+
+    @staticmethod
+    def allocate(T: int, n_steps: int, kept_cap: int, device, full: bool = True) -> "SelectOutputs":
+        torch = _torch()
+        i32, f32 = torch.int32, torch.float32
+        o = SelectOutputs(torch.full((max(kept_cap, 1),), -1, dtype=i32, device=device),
+                          torch.zeros(1, dtype=i32, device=device))
+        if full:
+            o.n_budget = torch.zeros(2, dtype=i32, device=device)
+            o.priority = torch.empty(T, dtype=f32, device=device)
+            o.token_sal = torch.empty(T, dtype=f32, device=device)
+            o.step_util = torch.empty(n_steps, dtype=f32, device=device)
+            o.step_count = torch.empty(n_steps, dtype=i32, device=device)
+            o.step_sal_sum = torch.empty(n_steps, dtype=f32, device=device)
+            o.step_sal_max = torch.empty(n_steps, dtype=f32, device=device)
+            o.step_kept = torch.empty(n_steps, dtype=i32, device=device)
+        o._cap = kept_cap
+        return o
+
+    def c(self) -> CSelOut:
+        cap = getattr(self, "_cap", self.kept_idx.numel())
+        return CSelOut(_ptr(self.kept_idx), cap, _ptr(self.n_kept), _ptr(self.n_budget), _ptr(self.priority),
+                       _ptr(self.token_sal), _ptr(self.step_util), _ptr(self.step_count), _ptr(self.step_sal_sum),
+                       _ptr(self.step_sal_max), _ptr(self.step_kept))
+
+
+def stepkv_select(sal, step_id, prot, steps: StepSignals, params: Params, budget: CBudget, out: SelectOutputs,
+                  ws=None, status=None, stream=None) -> SelectOutputs:
+    """Eqs. 1-5 + top-B over the prunable tokens.  sal: [n_sal, T] (or [..., T]) float32 rows."""
+    torch = _torch()
+    lib = load_library()
+    _need(sal, torch.float32, "sal")
+    T = sal.shape[-1]
+    n_sal = sal.numel() // T
+    if not sal.is_contiguous():
+        raise ValueError("sal must be contiguous")
+    _need(step_id, torch.int32, "step_id", 1)
+    _need(prot, torch.uint8, "prot", 1)
+    if step_id.numel() < T or prot.numel() < T:
+        raise ValueError("step_id/prot shorter than T")
+    dev = sal.device
+    need = lib.stepkv_select_workspace_size(n_sal, T, steps.n_steps)
+    ws = _workspace(need + 256, ws, dev)
+    wp, wn = _aligned_ws(ws)
+    status = status if status is not None else new_status(dev)
+    cs, cp, co = steps.c(), params.c(), out.c()
+    code = lib.stepkv_select(sal.data_ptr(), n_sal, T, step_id.data_ptr(), prot.data_ptr(), ctypes.byref(cs),
+                             ctypes.byref(cp), ctypes.byref(budget), ctypes.byref(co), wp, wn, status.data_ptr(),
+                             _stream_handle(stream))
+    _check(code, "stepkv_select")
+    return out
+
+
+# ----------------------------------------------------------------------------- stage 5
+def stepkv_compact(K_in: Sequence, V_in: Optional[Sequence], T: int, kept_idx, n_kept, kept_cap: int,
+                   K_out: Sequence, V_out: Optional[Sequence], step_id_in=None, pos_in=None, step_id_out=None,
+                   pos_out=None, status=None, stream=None):
+    """Gather retained rows of every layer: K_out[l][h, r] = K_in[l][h, kept_idx[r]] (same for V)."""
+    torch = _torch()
+    lib = load_library()
+    n = len(K_in)
+    ins = _rows_layout(K_in + (list(V_in) if V_in else []), "K_in/V_in") if n else 0
+    outs = _rows_layout(K_out + (list(V_out) if V_out else []), "K_out/V_out") if n else 0
+    Hkv, _, d = K_in[0].shape if n else (1, 0, 8)
+    _need(kept_idx, torch.int32, "kept_idx", 1)
+    _need(n_kept, torch.int32, "n_kept")
+    dev = kept_idx.device
+    status = status if status is not None else new_status(dev)
+    kin, vin, kout, vout = _ptr_array(K_in), _ptr_array(V_in or []), _ptr_array(K_out), _ptr_array(V_out or [])
+    code = lib.stepkv_compact(n, ctypes.cast(kin, ctypes.c_void_p) if n else None,
+                              ctypes.cast(vin, ctypes.c_void_p) if V_in else None, ins, Hkv, d, T,
+                              kept_idx.data_ptr(), n_kept.data_ptr(), kept_cap,
+                              ctypes.cast(kout, ctypes.c_void_p) if n else None,
+                              ctypes.cast(vout, ctypes.c_void_p) if V_out else None, outs,
+                              _ptr(step_id_in), _ptr(pos_in), _ptr(step_id_out), _ptr(pos_out), status.data_ptr(),
+                              _stream_handle(stream))
+    _check(code, "stepkv_compact")
+
+
+# ----------------------------------------------------------------------------- fused pass
+@dataclass
+class Problem:
+    """One trajectory for stepkv_compress (tensors on the device)."""
+    K: List            # L x [Hkv, rows >= T, d] bf16
+    V: List
+    Q: List            # n_sal_layers x [Hq, W, d] bf16 (layers L-n_sal_layers .. L-1)
+    T: int
+    step_id: object    # [T] int32
+    prot: object       # [T] uint8
+    steps: StepSignals
+    budget: CBudget
+    K_out: List
+    V_out: List
+    out: SelectOutputs
+    pos_in: object = None
+    step_id_out: object = None
+    pos_out: object = None
+    _keep: list = field(default_factory=list, repr=False)
+
+    def c(self) -> CProblem:
+        torch = _torch()
+        L = len(self.K)
+        Ls = len(self.Q)
+        ks = _rows_layout(list(self.K) + list(self.V), "K/V")
+        qs = _rows_layout(self.Q, "Q")
+        outs = _rows_layout(list(self.K_out) + list(self.V_out), "K_out/V_out")
+        Hkv, _, d = self.K[0].shape
+        Hq, W, _ = self.Q[0].shape
+        _need(self.step_id, torch.int32, "step_id", 1)
+        _need(self.prot, torch.uint8, "prot", 1)
+        arrs = [_ptr_array(self.K), _ptr_array(self.V), _ptr_array(self.Q), _ptr_array(self.K_out),
+                _ptr_array(self.V_out)]
+        self._keep = arrs
+        cv = lambda a: ctypes.cast(a, ctypes.c_void_p)
+        return CProblem(L, Hkv, Hq, d, self.T, W, Ls, cv(arrs[0]), cv(arrs[1]), ks, cv(arrs[2]), qs,
+                        _ptr(self.step_id), _ptr(self.prot), _ptr(self.pos_in), self.steps.c(), self.budget,
+                        cv(arrs[3]), cv(arrs[4]), outs, _ptr(self.step_id_out), _ptr(self.pos_out), self.out.c())
+
+
+def stepkv_workspace_size(problems: Sequence[Problem]) -> int:
+    arr = (CProblem * len(problems))(*[p.c() for p in problems])
+    return int(load_library().stepkv_compress_workspace_size(arr, len(problems)))
+
+
+def stepkv_compress(problems: Sequence[Problem], params: Params, ws=None, status=None, stream=None):
+    """score -> reduce/fuse -> select -> compact for every trajectory, in order on one stream."""
+    lib = load_library()
+    probs = list(problems)
+    arr = (CProblem * len(probs))(*[p.c() for p in probs])
+    need = int(lib.stepkv_compress_workspace_size(arr, len(probs)))
+    dev = probs[0].step_id.device
+    ws = _workspace(need + 256, ws, dev)
+    wp, wn = _aligned_ws(ws)
+    status = status if status is not None else new_status(dev)
+    cp = params.c()
+    code = lib.stepkv_compress(arr, len(probs), ctypes.byref(cp), wp, wn, status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_compress")
+    return status

@@ -1,0 +1,279 @@
+// C ABI of the StepKV compression pass: argument validation, workspace layout, and the order of
+// kernel launches.  Every function only enqueues work on the caller's stream.
+#include <stdio.h>
+
+#include <algorithm>
+#include <mutex>
+#include <map>
+#include <utility>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace stepkv {
+
+static thread_local char g_last_error[256] = {0};
+
+void set_last_cuda_error(cudaError_t e) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+cudaError_t device_sm_count(int* n) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  return cudaDeviceGetAttribute(n, cudaDevAttrMultiProcessorCount, dev);
+}
+
+// Raise a kernel's dynamic shared-memory limit on the current device.  The limit only ever grows, so a
+// launch that needs less than an earlier one keeps working.
+cudaError_t ensure_smem_attr(const void* func, int bytes) {
+  static std::mutex mu;
+  static std::map<std::pair<const void*, int>, int> limit;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  auto key = std::make_pair(func, dev);
+  auto it = limit.find(key);
+  if (it != limit.end() && it->second >= bytes) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) limit[key] = bytes;
+  return e;
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+static stepkv_status_t check_score_args(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                                        int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W) {
+  if (n_layers < 1 || n_layers > kMaxSalLayers) return STEPKV_EUNSUPPORTED;
+  if (!K || !Q) return STEPKV_EINVAL;
+  if (Hkv < 1 || Hq < 1 || Hq % Hkv != 0 || T < 1 || W < 1 || W > T) return STEPKV_EINVAL;
+  if (d != 64 && d != 128) return STEPKV_EUNSUPPORTED;
+  if (W > 4096) return STEPKV_EUNSUPPORTED;
+  if (k_head_stride < (int64_t)T * d || q_head_stride < (int64_t)W * d) return STEPKV_EINVAL;
+  if (k_head_stride % 8 || q_head_stride % 8) return STEPKV_EUNSUPPORTED;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!K[l] || !Q[l]) return STEPKV_EINVAL;
+    if (!aligned16(K[l]) || !aligned16(Q[l])) return STEPKV_EUNSUPPORTED;
+  }
+  return STEPKV_OK;
+}
+
+static stepkv_status_t check_select_args(int n_sal, int T, const int32_t* step_id, const uint8_t* prot,
+                                         const stepkv_steps_t* steps, const stepkv_params_t* params,
+                                         const stepkv_budget_t* budget, const stepkv_select_out_t* out) {
+  if (!steps || !params || !budget || !out || !step_id || !prot) return STEPKV_EINVAL;
+  if (n_sal < 1 || T < 1) return STEPKV_EINVAL;
+  if (T > 262144) return STEPKV_EUNSUPPORTED;
+  if (steps->n_steps < 1 || steps->n_steps > 65536) return STEPKV_EINVAL;
+  if (!steps->valid || !steps->gain || !steps->red || !steps->reuse_in) return STEPKV_EINVAL;
+  if (!out->kept_idx || !out->n_kept || out->kept_cap < 0) return STEPKV_EINVAL;
+  if (params->sal_norm != STEPKV_NORM_MAX && params->sal_norm != STEPKV_NORM_NONE) return STEPKV_EINVAL;
+  if (budget->mode == STEPKV_BUDGET_RATIO) {
+    if (budget->ratio_num < 0 || budget->ratio_den < 1) return STEPKV_EINVAL;
+  } else if (budget->mode == STEPKV_BUDGET_COUNT) {
+    if (budget->count < 0) return STEPKV_EINVAL;
+  } else {
+    return STEPKV_EINVAL;
+  }
+  return STEPKV_OK;
+}
+
+static stepkv_status_t check_compact_args(int n_layers, const void* const* K_in, const void* const* V_in,
+                                          int64_t in_head_stride, int Hkv, int d, int T, const int32_t* kept_idx,
+                                          const int32_t* n_kept, int kept_cap, void* const* K_out,
+                                          void* const* V_out, int64_t out_head_stride) {
+  if (n_layers < 0 || Hkv < 1 || d < 8 || T < 1 || kept_cap < 0) return STEPKV_EINVAL;
+  if (!kept_idx || !n_kept) return STEPKV_EINVAL;
+  if ((d * 2) % 16) return STEPKV_EUNSUPPORTED;
+  if (n_layers > 0) {
+    if (!K_in || !K_out) return STEPKV_EINVAL;
+    if ((V_in == nullptr) != (V_out == nullptr)) return STEPKV_EINVAL;
+    if (in_head_stride < (int64_t)T * d || out_head_stride < (int64_t)kept_cap * d) return STEPKV_EINVAL;
+    if (in_head_stride % 8 || out_head_stride % 8) return STEPKV_EUNSUPPORTED;
+    for (int l = 0; l < n_layers; ++l) {
+      if (!K_in[l] || !K_out[l]) return STEPKV_EINVAL;
+      if (!aligned16(K_in[l]) || !aligned16(K_out[l])) return STEPKV_EUNSUPPORTED;
+      if (K_in[l] == K_out[l]) return STEPKV_EUNSUPPORTED;
+      if (V_in) {
+        if (!V_in[l] || !V_out[l]) return STEPKV_EINVAL;
+        if (!aligned16(V_in[l]) || !aligned16(V_out[l])) return STEPKV_EUNSUPPORTED;
+        if (V_in[l] == V_out[l]) return STEPKV_EUNSUPPORTED;
+      }
+    }
+  }
+  return STEPKV_OK;
+}
+
+static size_t score_ws(int n_layers, int Hkv, int Hq, int T, int W, bool need_rows) {
+  const int n_rg = score_row_groups(Hkv, Hq, W);
+  size_t b = align256(score_partial_bytes(n_layers, Hkv, Hq, W));
+  if (need_rows) b += align256((size_t)n_layers * Hkv * n_rg * T * sizeof(float));
+  return b;
+}
+
+}  // namespace stepkv
+
+using namespace stepkv;
+
+extern "C" {
+
+void stepkv_default_params(stepkv_params_t* p) {
+  if (!p) return;
+  p->lambda = 0.3f;
+  p->w_r = 0.85f;
+  p->w_c = 0.15f;
+  p->r_min = -1.0f;
+  p->r_max = 2.0f;
+  p->s_max = 8.0f;
+  p->eta = 1.5f;
+  p->alpha = 0.2f;
+  p->beta = 0.8f;
+  p->sal_norm = STEPKV_NORM_MAX;
+}
+
+const char* stepkv_status_string(int32_t status) {
+  switch (status) {
+    case STEPKV_OK: return "ok";
+    case STEPKV_EINVAL: return "invalid argument";
+    case STEPKV_ECUDA: return "CUDA error";
+    case STEPKV_ENOSPACE: return "insufficient space (workspace or kept_cap)";
+    case STEPKV_EUNSUPPORTED: return "unsupported shape or alignment";
+    case STEPKV_EDATA: return "invalid data (step id or kept index out of range)";
+    case STEPKV_ETIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+  }
+}
+
+int32_t stepkv_version(void) { return 1000; }
+
+const char* stepkv_last_cuda_error(void) { return g_last_error; }
+
+size_t stepkv_score_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t T, int32_t W) {
+  if (n_layers < 1 || Hkv < 1 || Hq < Hkv || T < 1 || W < 1) return 0;
+  return score_ws(n_layers, Hkv, Hq, T, W, score_row_groups(Hkv, Hq, W) > 1);
+}
+
+stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                             int64_t q_head_stride, int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
+                             float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
+  stepkv_status_t st = check_score_args(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W);
+  if (st != STEPKV_OK) return st;
+  if (!sal || !ws) return STEPKV_EINVAL;
+  const int n_rg = score_row_groups(Hkv, Hq, W);
+  const size_t need = score_ws(n_layers, Hkv, Hq, T, W, n_rg > 1);
+  if (ws_bytes < need) return STEPKV_ENOSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float2* part = static_cast<float2*>(ws);
+  float* rows = sal;
+  if (n_rg > 1)
+    rows = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + align256(score_partial_bytes(n_layers, Hkv, Hq, W)));
+  st = score_run(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W, rows, T, part, dev_status, s);
+  if (st != STEPKV_OK) return st;
+  if (n_rg > 1) st = score_sum_row_groups(rows, n_layers * Hkv, n_rg, T, sal, s);
+  return st;
+}
+
+size_t stepkv_select_workspace_size(int32_t n_sal, int32_t T, int32_t n_steps) {
+  (void)n_sal;
+  if (T < 1 || n_steps < 1) return 0;
+  return select_ws_bytes(T, n_steps);
+}
+
+stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T, const int32_t* step_id,
+                              const uint8_t* prot, const stepkv_steps_t* steps, const stepkv_params_t* params,
+                              const stepkv_budget_t* budget, const stepkv_select_out_t* out, void* ws,
+                              size_t ws_bytes, int32_t* dev_status, void* stream) {
+  stepkv_status_t st = check_select_args(n_sal, T, step_id, prot, steps, params, budget, out);
+  if (st != STEPKV_OK) return st;
+  if (!sal || !ws) return STEPKV_EINVAL;
+  if (ws_bytes < select_ws_bytes(T, steps->n_steps)) return STEPKV_ENOSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
+  return select_run(sal, n_sal, T, 1.0f / (float)n_sal, T, step_id, prot, *steps, *params, *budget, *out, ws,
+                    dev_status, static_cast<cudaStream_t>(stream));
+}
+
+stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
+                               int64_t in_head_stride, int32_t Hkv, int32_t d, int32_t T, const int32_t* kept_idx,
+                               const int32_t* n_kept, int32_t kept_cap, void* const* K_out, void* const* V_out,
+                               int64_t out_head_stride, const int32_t* step_id_in, const int32_t* pos_in,
+                               int32_t* step_id_out, int32_t* pos_out, int32_t* dev_status, void* stream) {
+  stepkv_status_t st = check_compact_args(n_layers, K_in, V_in, in_head_stride, Hkv, d, T, kept_idx, n_kept, kept_cap,
+                                          K_out, V_out, out_head_stride);
+  if (st != STEPKV_OK) return st;
+  return compact_run(n_layers, K_in, V_in, in_head_stride, Hkv, d, T, kept_idx, n_kept, kept_cap, K_out, V_out,
+                     out_head_stride, step_id_in, pos_in, step_id_out, pos_out, dev_status,
+                     static_cast<cudaStream_t>(stream));
+}
+
+static size_t compress_ws_one(const stepkv_problem_t& p) {
+  const int Ls = std::min(p.n_sal_layers, p.L);
+  const int n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
+  size_t b = align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
+  b += align256((size_t)Ls * p.Hkv * n_rg * p.T * sizeof(float));
+  b += align256(select_ws_bytes(p.T, p.steps.n_steps));
+  return b;
+}
+
+size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj) {
+  if (!probs || n_traj < 1) return 0;
+  size_t m = 0;
+  for (int i = 0; i < n_traj; ++i) {
+    const stepkv_problem_t& p = probs[i];
+    if (p.L < 1 || p.Hkv < 1 || p.Hq < p.Hkv || p.T < 1 || p.W < 1 || p.n_sal_layers < 1 || p.steps.n_steps < 1)
+      return 0;
+    m = std::max(m, compress_ws_one(p));
+  }
+  return m;
+}
+
+stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, const stepkv_params_t* params,
+                                void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
+  if (!probs || n_traj < 1 || !params || !ws) return STEPKV_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
+  // validate everything before enqueueing anything
+  for (int i = 0; i < n_traj; ++i) {
+    const stepkv_problem_t& p = probs[i];
+    if (p.L < 1 || p.n_sal_layers < 1) return STEPKV_EINVAL;
+    const int Ls = std::min(p.n_sal_layers, p.L);
+    if (Ls > kMaxSalLayers) return STEPKV_EUNSUPPORTED;
+    if (!p.K || !p.Q) return STEPKV_EINVAL;
+    stepkv_status_t st = check_score_args(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq,
+                                          p.d, p.T, p.W);
+    if (st != STEPKV_OK) return st;
+    st = check_select_args(Ls * p.Hkv, p.T, p.step_id, p.prot, &p.steps, params, &p.budget, &p.sel);
+    if (st != STEPKV_OK) return st;
+    st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
+                            p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride);
+    if (st != STEPKV_OK) return st;
+    if (ws_bytes < compress_ws_one(p)) return STEPKV_ENOSPACE;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  for (int i = 0; i < n_traj; ++i) {
+    const stepkv_problem_t& p = probs[i];
+    const int Ls = std::min(p.n_sal_layers, p.L);
+    const int n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
+    uint8_t* w = static_cast<uint8_t*>(ws);
+    float2* part = reinterpret_cast<float2*>(w);
+    w += align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
+    float* rows = reinterpret_cast<float*>(w);
+    w += align256((size_t)Ls * p.Hkv * n_rg * p.T * sizeof(float));
+    void* sel_ws = w;
+    stepkv_status_t st = score_run(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
+                                   p.T, p.W, rows, p.T, part, dev_status, s);
+    if (st != STEPKV_OK) return st;
+    st = select_run(rows, Ls * p.Hkv * n_rg, p.T, 1.0f / (float)(Ls * p.Hkv), p.T, p.step_id, p.prot, p.steps,
+                    *params, p.budget, p.sel, sel_ws, dev_status, s);
+    if (st != STEPKV_OK) return st;
+    st = compact_run(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap,
+                     p.K_out, p.V_out, p.out_head_stride, p.step_id, p.pos_in, p.step_id_out, p.pos_out, dev_status,
+                     s);
+    if (st != STEPKV_OK) return st;
+  }
+  return STEPKV_OK;
+}
+
+}  // extern "C"

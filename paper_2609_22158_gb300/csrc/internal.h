@@ -1,0 +1,88 @@
+// Host-side internals shared by the StepKV translation units (not part of the C ABI).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <utility>
+
+#include "../../include/stepkv.h"
+
+namespace stepkv {
+
+constexpr int kMaxSalLayers = 8;        // saliency layers per score launch (tensor maps in kernel params)
+constexpr int kMaxGrid = 1024;          // upper bound on the persistent score grid (partial-slot sizing)
+constexpr double kL2GroupBytes = 80e6;  // K bytes per score launch group (re-read from L2 by pass 2)
+constexpr int kMaxCompactLayers = 256;  // layers per compaction launch (pointer tables in kernel params)
+
+void set_last_cuda_error(cudaError_t e);
+cudaError_t device_sm_count(int* n);
+cudaError_t ensure_smem_attr(const void* func, int bytes);
+
+// Launch with programmatic stream serialization (PDL): the kernel may start while its predecessor
+// drains and must call griddepcontrol.wait before touching memory the predecessor produced.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cluster_x, size_t smem,
+                               cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = cluster_x;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
+// ---- score (score.cu)
+int score_row_groups(int Hkv, int Hq, int W);
+size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W);
+// Writes pass-2 rows: row (pair*n_rg + rg) of rows_out (stride out_stride) for pair = layer*Hkv + h.
+stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                          int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
+                          int64_t out_stride, float2* part, int32_t* status, cudaStream_t stream);
+stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal, cudaStream_t stream);
+
+// ---- select (select.cu)
+size_t select_ws_bytes(int T, int n_steps);
+// rows: n_rows saliency rows of length T (stride row_stride); T_i = inv_div * sum of the rows.
+stepkv_status_t select_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T,
+                           const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
+                           const stepkv_params_t& params, const stepkv_budget_t& budget,
+                           const stepkv_select_out_t& out, void* ws, int32_t* status, cudaStream_t stream);
+
+// ---- compact (compact.cu)
+stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* const* V_in, int64_t in_head_stride,
+                            int Hkv, int d, int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
+                            void* const* K_out, void* const* V_out, int64_t out_head_stride,
+                            const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
+                            int32_t* pos_out, int32_t* status, cudaStream_t stream);
+
+}  // namespace stepkv

@@ -1,0 +1,607 @@
+// Stage 1 -- token saliency from the observation-window queries (Sec. 4.2 "Token Saliency";
+// Table H: last 3 layers).  For layer l, KV head h, key j:
+//   A[l,h,j] = (1/G) sum_{g in group(h)} sum_w softmax_{j' <= T-W+w}(q_{g,w} . k_{j'} / sqrt(d))[j]
+//
+// GB300 design.  The softmax normalises over keys while A sums over query rows, so the two
+// reductions run in two tensor-core passes over K, each in the orientation that makes its
+// reduction a per-thread loop over TMEM columns:
+//   pass 1  S   = Q . K^T  (M = 128 query rows, N = 128 keys): per-row running max m and
+//                 Z = sum 2^((s - m) c), c = log2(e)/sqrt(d); one partial (m, Z) per CTA segment;
+//   pass 2  S^T = K . Q^T  (M = 128 keys, N = up to 256 query rows): per-key
+//                 sum_r 2^(s c - off_r), off_r = m_r c + log2 Z_r combined from the pass-1 partials.
+// K tiles are TMA-staged (128-byte swizzle) through an mbarrier ring; one thread issues tcgen05.mma
+// into a double-buffered TMEM accumulator (2 x 256 columns); 8 epilogue warps read TMEM with
+// tcgen05.ld and spend one MUFU ex2 per logit.  Each CTA (one per SM) owns a contiguous range of key
+// tiles, so a (pair, row-group) unit has a few pass-1 partials that pass 2 combines in a fixed order
+// (deterministic).  Pairs are launched in groups whose K fits in L2, so pass 2 re-reads K from L2.
+#include <math.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace stepkv {
+
+constexpr int kThreads = 320;   // warp 0: TMA producer, warp 1: MMA issuer + TMEM owner, warps 2..9: epilogue
+constexpr int kEpiWarps = 8;
+constexpr int kKeyTile = 128;
+constexpr int kMaxRows = 256;   // query rows per row group
+constexpr int kTmemCols = 512;  // two accumulator buffers of 256 columns
+constexpr int kQChunkBytes = kMaxRows * 128;   // one 64-wide d chunk of the Q staging area
+constexpr int kKChunkBytes = kKeyTile * 128;   // one 64-wide d chunk of a K tile
+
+struct ScoreGeom {
+  int Hkv, Hq, G, d, T, W;
+  int W_pad;         // W rounded up to 8 (each head's block starts on a 1024-byte swizzle atom)
+  int split;         // 0: several whole heads per row group; 1: a head's window split over row groups
+  int hpr;           // heads per row group (split == 0)
+  int rph;           // row groups per head (split == 1)
+  int n_rg;          // row groups per (layer, KV head) pair
+  int n_tiles;       // ceil(T / 128)
+  float c;           // log2(e) / sqrt(d)
+  float inv_G;
+};
+
+struct ScoreLaunch {
+  CUtensorMap tmK[kMaxSalLayers];
+  CUtensorMap tmQ[kMaxSalLayers];
+  ScoreGeom g;
+  int n_layers;
+  int pair0;          // first (layer*Hkv + head) pair of this launch
+  int n_units;        // units = pairs of this launch x n_rg
+  int tpc;            // tiles per CTA (contiguous range)
+  float2* part;       // pass-1 partials: slot (unit + cta) x 256 rows
+  float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride
+  int64_t out_stride;
+  int32_t* status;
+};
+
+struct RowGroup {
+  int g_first;   // first local query head (0..G-1) of this group
+  int n_blk;     // head blocks
+  int blk_rows;  // rows per block
+  int w0;        // window offset of the block's first row
+  int rows;      // n_blk * blk_rows (<= 256)
+};
+
+__host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
+  RowGroup r;
+  if (!g.split) {
+    r.g_first = rg * g.hpr;
+    r.n_blk = min(g.hpr, g.G - r.g_first);
+    r.blk_rows = g.W_pad;
+    r.w0 = 0;
+  } else {
+    r.g_first = rg / g.rph;
+    r.n_blk = 1;
+    r.w0 = (rg % g.rph) * kMaxRows;
+    r.blk_rows = min(kMaxRows, g.W_pad - r.w0);
+  }
+  r.rows = r.n_blk * r.blk_rows;
+  return r;
+}
+
+template <int NCH>
+struct ScoreCfg {
+  static constexpr int kStages = NCH == 2 ? 4 : 8;
+  static constexpr int kQBytes = NCH * kQChunkBytes;
+  static constexpr int kStageBytes = NCH * kKChunkBytes;
+  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;  // float sOff[256]
+  static constexpr int kPwOff = kOffOff + kMaxRows * 4;            // int   sPw[256]
+  static constexpr int kCombOff = kPwOff + kMaxRows * 4;           // 2 KB: float2[256] (pass 1) / float[2][128] (pass 2)
+  static constexpr int kBarOff = kCombOff + kMaxRows * 8;
+  static constexpr int kNumBars = 2 * kStages + 2 + 4 + 1;
+  static constexpr int kMiscOff = kBarOff + kNumBars * 8;          // tmem base, abort flag
+  static constexpr int kBytes = kMiscOff + 16;
+  static constexpr int kDynSmem = kBytes + 1024;                   // + alignment slack
+};
+
+// Bounded barrier among the 8 epilogue warps (an mbarrier with one arrival per warp).  Returns false
+// if the CTA aborted or the wait limit passed.
+__device__ __forceinline__ bool epi_sync(uint64_t* bar, uint32_t& phase, volatile int* abort_flag) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+  const bool ok = mbar_wait(bar, phase, abort_flag);
+  phase ^= 1;
+  __syncwarp();
+  return ok;
+}
+
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) {
+  int zero = 0;
+  return mbar_wait(bar, parity, &zero);
+}
+
+template <int PASS, int NCH>
+__global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreLaunch p) {
+  using Cfg = ScoreCfg<NCH>;
+  constexpr int S = Cfg::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = sm;
+  uint8_t* sK = sm + Cfg::kQBytes;
+  float* sOff = reinterpret_cast<float*>(sm + Cfg::kOffOff);
+  int* sPw = reinterpret_cast<int*>(sm + Cfg::kPwOff);
+  float2* sComb = reinterpret_cast<float2*>(sm + Cfg::kCombOff);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kBarOff);
+  uint64_t* k_full = bars;
+  uint64_t* k_empty = bars + S;
+  uint64_t* q_full = bars + 2 * S;
+  uint64_t* q_empty = q_full + 1;
+  uint64_t* acc_full = q_empty + 1;    // [2]
+  uint64_t* acc_empty = acc_full + 2;  // [2]
+  uint64_t* epi_bar = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + Cfg::kMiscOff);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + Cfg::kMiscOff + 4);
+
+  const ScoreGeom& g = p.g;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int U = p.n_units * g.n_tiles;
+  const int t_lo = blockIdx.x * p.tpc;
+  const int t_hi = min(U, t_lo + p.tpc);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], kEpiWarps);
+    }
+    mbar_init(epi_bar, kEpiWarps);
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0 && lane == 0) {
+    for (int l = 0; l < p.n_layers; ++l) {
+      tma_prefetch_desc(&p.tmK[l]);
+      tma_prefetch_desc(&p.tmQ[l]);
+    }
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+  // Zero the Q staging area once: rows the TMA never writes (MMA padding) must hold finite values.
+  for (int i = threadIdx.x; i < Cfg::kQBytes / 16; i += kThreads) reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0, 0, 0, 0);
+  fence_proxy_async_smem();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  pdl_wait();  // K/Q (possibly written by an earlier compaction) and pass-1 partials are complete
+  pdl_launch_dependents();
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer (one thread)
+    if (lane == 0) {
+      int stage = 0, cur = -1;
+      uint32_t phase = 0, qe_phase = 0, q_issue_phase = 0;
+      uint32_t last_parity[S];
+      bool used[S];
+      for (int i = 0; i < S; ++i) used[i] = false;
+      bool q_used = false, ok = true;
+      for (int gt = t_lo; gt < t_hi; ++gt) {
+        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+        const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
+        const int layer = pair / g.Hkv, h = pair - layer * g.Hkv;
+        if (u != cur) {
+          if (cur >= 0) {
+            if (!mbar_wait(q_empty, qe_phase, abort_flag)) { ok = false; break; }
+            qe_phase ^= 1;
+          }
+          const RowGroup r = row_group(g, rg);
+          const int box_rows = min(g.W_pad, kMaxRows);
+          mbar_arrive_expect_tx(q_full, (uint32_t)(r.n_blk * NCH * box_rows * 128));
+          for (int b = 0; b < r.n_blk; ++b)
+            for (int c = 0; c < NCH; ++c)
+              tma_load_3d(sQ + c * kQChunkBytes + b * r.blk_rows * 128, &p.tmQ[layer], c * 64, r.w0,
+                          h * g.G + r.g_first + b, q_full);
+          q_used = true;
+          q_issue_phase ^= 1;
+          cur = u;
+        }
+        if (!mbar_wait(&k_empty[stage], phase ^ 1, abort_flag)) { ok = false; break; }
+        mbar_arrive_expect_tx(&k_full[stage], (uint32_t)(NCH * kKChunkBytes));
+        for (int c = 0; c < NCH; ++c)
+          tma_load_3d(sK + stage * Cfg::kStageBytes + c * kKChunkBytes, &p.tmK[layer], c * 64, tile * kKeyTile, h,
+                      &k_full[stage]);
+        used[stage] = true;
+        last_parity[stage] = phase;
+        if (++stage == S) { stage = 0; phase ^= 1; }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        record_status(p.status, STEPKV_ETIMEOUT);
+      }
+      // Drain: every copy this thread issued has landed before the CTA may exit.
+      for (int i = 0; i < S; ++i)
+        if (used[i]) mbar_wait_drain(&k_full[i], last_parity[i]);
+      if (q_used) mbar_wait_drain(q_full, q_issue_phase ^ 1);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (one thread)
+    if (lane == 0) {
+      int stage = 0, buf = 0, cur = -1;
+      uint32_t phase = 0, buf_phase = 0, q_phase = 0;
+      bool issued = false, ok = true;
+      int last_buf = 0;
+      uint32_t last_buf_parity = 0;
+      for (int gt = t_lo; gt < t_hi; ++gt) {
+        const int u = gt / g.n_tiles;
+        const RowGroup r = row_group(g, u % g.n_rg);
+        if (u != cur) {
+          if (cur >= 0) umma_commit(q_empty);  // Q may be overwritten once the previous unit's MMAs finish
+          if (!mbar_wait(q_full, q_phase, abort_flag)) { ok = false; break; }
+          q_phase ^= 1;
+          cur = u;
+        }
+        if (!mbar_wait(&acc_empty[buf], buf_phase ^ 1, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(&k_full[stage], phase, abort_flag)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t kst = smem_u32(sK + stage * Cfg::kStageBytes);
+        const uint32_t qst = smem_u32(sQ);
+        const uint32_t dcol = tmem_base + (uint32_t)(buf * 256);
+        if (PASS == 1) {
+          const int n_mt = r.rows > 128 ? 2 : 1;
+          constexpr uint32_t idesc = umma_idesc_bf16(128, kKeyTile);
+          for (int mt = 0; mt < n_mt; ++mt)
+#pragma unroll
+            for (int kk = 0; kk < NCH * 4; ++kk) {
+              const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + mt * 128 * 128 + (kk & 3) * 32);
+              const uint32_t koff = (uint32_t)((kk >> 2) * kKChunkBytes + (kk & 3) * 32);
+              umma_bf16(dcol + (uint32_t)(mt * 128), umma_desc_sw128(qst + qoff), umma_desc_sw128(kst + koff), idesc,
+                        kk > 0 ? 1u : 0u);
+            }
+        } else {
+          const int n_mma = (r.rows + 31) & ~31;  // every TMEM column the epilogue loads is written
+          const uint32_t idesc = umma_idesc_bf16(128, n_mma);
+#pragma unroll
+          for (int kk = 0; kk < NCH * 4; ++kk) {
+            const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + (kk & 3) * 32);
+            const uint32_t koff = (uint32_t)((kk >> 2) * kKChunkBytes + (kk & 3) * 32);
+            umma_bf16(dcol, umma_desc_sw128(kst + koff), umma_desc_sw128(qst + qoff), idesc, kk > 0 ? 1u : 0u);
+          }
+        }
+        umma_commit(&k_empty[stage]);
+        umma_commit(&acc_full[buf]);
+        issued = true;
+        last_buf = buf;
+        last_buf_parity = buf_phase;
+        if (++stage == S) { stage = 0; phase ^= 1; }
+        if (++buf == 2) { buf = 0; buf_phase ^= 1; }
+      }
+      if (!ok) {
+        *abort_flag = 1;
+        record_status(p.status, STEPKV_ETIMEOUT);
+      }
+      // Drain: the last MMA group has completed before TMEM is released.
+      if (issued) mbar_wait_drain(&acc_full[last_buf], last_buf_parity);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (8 warps)
+    const int ew = warp - 2;
+    const int q = warp & 3;    // TMEM lane quarter this warp may access
+    const int hsel = ew >> 2;  // which of the two warps sharing the quarter
+    const float c = g.c;
+    int buf = 0, cur = -1;
+    uint32_t buf_phase = 0, eb_phase = 0;
+    RowGroup r{};
+    float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row
+    int my_row = 0, my_pw = 0;
+    bool row_ok = false, ok = true;
+
+    for (int gt = t_lo; gt < t_hi && ok; ++gt) {
+      const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+      if (u != cur) {
+        if (PASS == 1) {
+          if (cur >= 0) {
+            // flush the partial of the previous unit
+            float mm = m, zz = Z;
+            const bool two = r.rows > 128;
+            if (!two) {
+              if (hsel == 1) sComb[q * 32 + lane] = make_float2(m, Z);
+              if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
+              if (hsel == 0) {
+                const float2 o = sComb[q * 32 + lane];
+                const float M = fmaxf(mm, o.x);
+                if (M != -INFINITY) zz = zz * ex2_approx((mm - M) * c) + o.y * ex2_approx((o.x - M) * c);
+                mm = M;
+              }
+              if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
+            }
+            if (two || hsel == 0) p.part[(size_t)(cur + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(mm, zz);
+          }
+          r = row_group(g, u % g.n_rg);
+          my_row = (r.rows > 128 ? hsel * 128 : 0) + q * 32 + lane;
+          const int w = r.w0 + my_row % r.blk_rows;
+          row_ok = my_row < r.rows && w < g.W;
+          my_pw = g.T - g.W + w;
+          m = -INFINITY;
+          Z = 0.f;
+        } else {
+          // Combine the pass-1 partials of unit u into per-row offsets, in contributing-CTA order.
+          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;  // previous unit's offsets no longer read
+          r = row_group(g, u % g.n_rg);
+          const int row = threadIdx.x - 64;
+          const int w = r.w0 + row % r.blk_rows;
+          const bool valid = row < r.rows && w < g.W;
+          float off = INFINITY;
+          if (valid) {
+            const int c0 = (u * g.n_tiles) / p.tpc;
+            const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+            float M = -INFINITY;
+            for (int ci = c0; ci <= c1; ++ci) M = fmaxf(M, __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]).x);
+            float Zs = 0.f;
+            for (int ci = c0; ci <= c1; ++ci) {
+              const float2 pz = __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]);
+              if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
+            }
+            off = M * c + __log2f(Zs);
+          }
+          sOff[row] = off;
+          sPw[row] = valid ? g.T - g.W + w : -1;
+          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
+        }
+        cur = u;
+      }
+      if (!(ok = mbar_wait(&acc_full[buf], buf_phase, abort_flag))) break;
+      tc_fence_after();
+      const int key0 = tile * kKeyTile;
+      const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
+      const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * 256);
+      if (PASS == 1) {
+        const bool two = r.rows > 128;
+        const int col_lo = two ? 0 : hsel * 64;
+        const int col_hi = two ? 128 : col_lo + 64;
+        const uint32_t mt_col = two ? (uint32_t)(hsel * 128) : 0u;
+        for (int cc = col_lo; cc < col_hi; cc += 32) {
+          float v[32];
+          tmem_ld32(lane_base + mt_col + (uint32_t)cc, v);
+          if (!row_ok) continue;
+          const int j0 = key0 + cc;
+          if (need_mask) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = (j0 + i <= my_pw) ? v[i] : -INFINITY;
+          }
+          float cm0 = fmaxf(v[0], v[1]), cm1 = fmaxf(v[2], v[3]);
+#pragma unroll
+          for (int i = 4; i < 32; i += 4) {
+            cm0 = fmaxf(cm0, fmaxf(v[i], v[i + 1]));
+            cm1 = fmaxf(cm1, fmaxf(v[i + 2], v[i + 3]));
+          }
+          const float mn = fmaxf(m, fmaxf(cm0, cm1));
+          if (mn == -INFINITY) continue;
+          const float mc = mn * c;
+          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+          for (int i = 0; i < 32; i += 4) {
+            s0 += ex2_approx(fmaf(v[i + 0], c, -mc));
+            s1 += ex2_approx(fmaf(v[i + 1], c, -mc));
+            s2 += ex2_approx(fmaf(v[i + 2], c, -mc));
+            s3 += ex2_approx(fmaf(v[i + 3], c, -mc));
+          }
+          Z = Z * ex2_approx((m - mn) * c) + ((s0 + s1) + (s2 + s3));
+          m = mn;
+        }
+      } else {
+        const int n_cols = (r.rows + 31) & ~31;
+        const int j = key0 + q * 32 + lane;
+        float acc = 0.f;
+        for (int cc = hsel * 32; cc < n_cols; cc += 64) {
+          float v[32];
+          tmem_ld32(lane_base + (uint32_t)cc, v);
+          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          if (!need_mask) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) {
+              const float4 o = *reinterpret_cast<const float4*>(&sOff[cc + i]);
+              s0 += ex2_approx(fmaf(v[i + 0], c, -o.x));
+              s1 += ex2_approx(fmaf(v[i + 1], c, -o.y));
+              s2 += ex2_approx(fmaf(v[i + 2], c, -o.z));
+              s3 += ex2_approx(fmaf(v[i + 3], c, -o.w));
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) {
+              const float4 o = *reinterpret_cast<const float4*>(&sOff[cc + i]);
+              const int4 pw = *reinterpret_cast<const int4*>(&sPw[cc + i]);
+              s0 += j <= pw.x ? ex2_approx(fmaf(v[i + 0], c, -o.x)) : 0.f;
+              s1 += j <= pw.y ? ex2_approx(fmaf(v[i + 1], c, -o.y)) : 0.f;
+              s2 += j <= pw.z ? ex2_approx(fmaf(v[i + 2], c, -o.z)) : 0.f;
+              s3 += j <= pw.w ? ex2_approx(fmaf(v[i + 3], c, -o.w)) : 0.f;
+            }
+          }
+          acc += (s0 + s1) + (s2 + s3);
+        }
+        float* comb = reinterpret_cast<float*>(sComb) + buf * 128;
+        if (hsel == 1) comb[q * 32 + lane] = acc;
+        // TMEM reads of this buffer are done: hand it back to the MMA issuer before the exchange
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
+        if (hsel == 0 && j < g.T) {
+          const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
+          p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = (acc + comb[q * 32 + lane]) * g.inv_G;
+        }
+        if (++buf == 2) { buf = 0; buf_phase ^= 1; }
+        continue;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      if (++buf == 2) { buf = 0; buf_phase ^= 1; }
+    }
+    if (PASS == 1 && ok && cur >= 0) {
+      float mm = m, zz = Z;
+      const bool two = r.rows > 128;
+      if (!two) {
+        if (hsel == 1) sComb[q * 32 + lane] = make_float2(m, Z);
+        ok = epi_sync(epi_bar, eb_phase, abort_flag);
+        if (ok && hsel == 0) {
+          const float2 o = sComb[q * 32 + lane];
+          const float M = fmaxf(mm, o.x);
+          if (M != -INFINITY) zz = zz * ex2_approx((mm - M) * c) + o.y * ex2_approx((o.x - M) * c);
+          mm = M;
+        }
+      }
+      if (ok && (two || hsel == 0)) p.part[(size_t)(cur + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(mm, zz);
+    }
+    if (!ok) {
+      *abort_flag = 1;
+      record_status(p.status, STEPKV_ETIMEOUT);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// -------------------------------------------------------------------------------------------------
+// Sum of row-group partial rows into the [n_pairs][T] saliency output (only needed when n_rg > 1).
+__global__ void sum_row_groups_kernel(const float* __restrict__ rows, int n_pairs, int n_rg, int T,
+                                      float* __restrict__ sal) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int64_t n = (int64_t)n_pairs * T;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t pair = i / T, j = i - pair * T;
+    float s = 0.f;
+    for (int rg = 0; rg < n_rg; ++rg) s += rows[(pair * n_rg + rg) * T + j];
+    sal[i] = s;
+  }
+}
+
+// -------------------------------------------------------------------------------------------------
+// Host side
+static ScoreGeom make_geom(int Hkv, int Hq, int d, int T, int W) {
+  ScoreGeom g;
+  memset(&g, 0, sizeof(g));
+  g.Hkv = Hkv;
+  g.Hq = Hq;
+  g.G = Hq / Hkv;
+  g.d = d;
+  g.T = T;
+  g.W = W;
+  g.W_pad = (W + 7) & ~7;
+  if (g.W_pad <= kMaxRows) {
+    g.split = 0;
+    g.hpr = kMaxRows / g.W_pad;
+    g.rph = 1;
+    g.n_rg = (g.G + g.hpr - 1) / g.hpr;
+  } else {
+    g.split = 1;
+    g.hpr = 1;
+    g.rph = (g.W_pad + kMaxRows - 1) / kMaxRows;
+    g.n_rg = g.G * g.rph;
+  }
+  g.n_tiles = (T + kKeyTile - 1) / kKeyTile;
+  g.c = (float)(1.4426950408889634 / sqrt((double)d));
+  g.inv_G = 1.0f / (float)g.G;
+  return g;
+}
+
+int score_row_groups(int Hkv, int Hq, int W) { return make_geom(Hkv, Hq, 64, W, W).n_rg; }
+
+size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
+  const int n_rg = score_row_groups(Hkv, Hq, W);
+  return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kMaxRows * sizeof(float2);
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn get_encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(f);
+  }
+  return fn;
+}
+
+// 3-D bf16 tensor map over [heads][rows][d] with a 64 x box_rows x 1 box and 128-byte swizzle.
+static bool encode_3d(CUtensorMap* map, const void* base, int d, int rows, int heads, int64_t head_stride,
+                      int box_rows) {
+  EncodeTiledFn enc = get_encode_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)heads};
+  cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)head_stride * 2};
+  cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int PASS, int NCH>
+static cudaError_t launch_pass(const ScoreLaunch& L, int grid, cudaStream_t stream) {
+  using Cfg = ScoreCfg<NCH>;
+  void (*kern)(ScoreLaunch) = score_kernel<PASS, NCH>;
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), Cfg::kDynSmem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(kern, dim3(grid), dim3(kThreads), Cfg::kDynSmem, stream, L);
+}
+
+stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                          int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
+                          int64_t out_stride, float2* part, int32_t* status, cudaStream_t stream) {
+  const ScoreGeom g = make_geom(Hkv, Hq, d, T, W);
+  ScoreLaunch L;
+  memset(&L, 0, sizeof(L));
+  L.g = g;
+  L.n_layers = n_layers;
+  L.part = part;
+  L.out = rows_out;
+  L.out_stride = out_stride;
+  L.status = status;
+  const int box_rows = std::min(g.W_pad, kMaxRows);
+  for (int l = 0; l < n_layers; ++l) {
+    if (!encode_3d(&L.tmK[l], K[l], d, T, Hkv, k_head_stride, kKeyTile)) return STEPKV_ECUDA;
+    if (!encode_3d(&L.tmQ[l], Q[l], d, W, Hq, q_head_stride, box_rows)) return STEPKV_ECUDA;
+  }
+  int n_sm = 0;
+  cudaError_t e = device_sm_count(&n_sm);
+  if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
+  const int grid_cap = std::max(1, std::min(n_sm, kMaxGrid));
+  // pairs per launch: one launch's K stays within L2, so pass 2 re-reads it from L2
+  const double pair_bytes = (double)T * d * 2.0;
+  const int n_pairs = n_layers * Hkv;
+  const int ppg = std::min(n_pairs, (int)std::max(1.0, floor(kL2GroupBytes / pair_bytes)));
+  for (int p0 = 0; p0 < n_pairs; p0 += ppg) {
+    const int np = std::min(ppg, n_pairs - p0);
+    L.pair0 = p0;
+    L.n_units = np * g.n_rg;
+    const int U = L.n_units * g.n_tiles;
+    const int grid0 = std::min(grid_cap, U);
+    L.tpc = (U + grid0 - 1) / grid0;
+    const int grid = (U + L.tpc - 1) / L.tpc;
+    e = d == 128 ? launch_pass<1, 2>(L, grid, stream) : launch_pass<1, 1>(L, grid, stream);
+    if (e == cudaSuccess) e = d == 128 ? launch_pass<2, 2>(L, grid, stream) : launch_pass<2, 1>(L, grid, stream);
+    if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
+  }
+  return STEPKV_OK;
+}
+
+stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal,
+                                     cudaStream_t stream) {
+  const int64_t n = (int64_t)n_pairs * T;
+  const int blocks = (int)std::min<int64_t>((n + 255) / 256, 4096);
+  cudaError_t e = launch_pdl(sum_row_groups_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_pairs, n_rg, T, sal);
+  if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
+  return STEPKV_OK;
+}
+
+}  // namespace stepkv

@@ -1,0 +1,116 @@
+"""CPU-only checks of the C ABI library: it builds for sm_103a, loads without a GPU, exports every
+function declared in include/stepkv.h, and rejects bad arguments on the host before touching CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "stepkv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_22158_gb300 import binding, build
+    build.build_library()
+    return binding.load_library()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"\b(stepkv_[a-z_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("stepkv_score", "stepkv_select", "stepkv_compact", "stepkv_compress"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    from paper_2609_22158_gb300 import binding
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert name in binding.SIGNATURES, f"binding lacks a signature for {name}"
+
+
+def test_default_params_are_table_h(lib):
+    from paper_2609_22158_gb300 import binding
+    p = binding.default_params()
+    assert abs(p.lam - 0.3) < 1e-7 and abs(p.w_r - 0.85) < 1e-7 and abs(p.w_c - 0.15) < 1e-7
+    assert p.r_min == -1.0 and p.r_max == 2.0 and p.s_max == 8.0
+    assert p.eta == 1.5 and abs(p.alpha - 0.2) < 1e-7 and abs(p.beta - 0.8) < 1e-7 and p.sal_norm == 0
+
+
+def test_status_strings(lib):
+    for code in range(7):
+        assert lib.stepkv_status_string(code)
+    assert lib.stepkv_status_string(99) == b"unknown status"
+    assert lib.stepkv_version() >= 1000
+
+
+def test_workspace_sizes(lib):
+    assert lib.stepkv_score_workspace_size(3, 8, 32, 32768, 64) > 0
+    assert lib.stepkv_score_workspace_size(0, 8, 32, 32768, 64) == 0
+    assert lib.stepkv_select_workspace_size(24, 32768, 40) > 0
+    assert lib.stepkv_select_workspace_size(24, 32768, 0) == 0
+
+
+def test_score_rejects_bad_arguments_on_host(lib):
+    from paper_2609_22158_gb300.binding import STEPKV_EINVAL, STEPKV_EUNSUPPORTED
+    arr = (ctypes.c_void_p * 1)(256)
+    p = ctypes.cast(arr, ctypes.c_void_p)
+    ws = ctypes.c_void_p(1 << 20)
+    # d not supported
+    assert lib.stepkv_score(1, p, 96 * 100, p, 96 * 10, 2, 8, 96, 100, 10, 4096, ws, 1 << 30, None, None) == STEPKV_EUNSUPPORTED
+    # Hq not a multiple of Hkv
+    assert lib.stepkv_score(1, p, 128 * 100, p, 128 * 10, 3, 8, 128, 100, 10, 4096, ws, 1 << 30, None, None) == STEPKV_EINVAL
+    # W > T
+    assert lib.stepkv_score(1, p, 128 * 100, p, 128 * 200, 2, 8, 128, 100, 200, 4096, ws, 1 << 30, None, None) == STEPKV_EINVAL
+    # too many layers for one call
+    assert lib.stepkv_score(9, p, 128 * 100, p, 128 * 10, 2, 8, 128, 100, 10, 4096, ws, 1 << 30, None, None) == STEPKV_EUNSUPPORTED
+    # head stride smaller than T*d
+    assert lib.stepkv_score(1, p, 128 * 99, p, 128 * 10, 2, 8, 128, 100, 10, 4096, ws, 1 << 30, None, None) == STEPKV_EINVAL
+
+
+def test_select_rejects_bad_arguments_on_host(lib):
+    from paper_2609_22158_gb300 import binding as B
+    steps = B.CSteps(0, 256, 256, 256, None, 256, None)
+    params = B.Params().c()
+    bud = B.budget_ratio(1, 10)
+    out = B.CSelOut(256, 10, 256, None, None, None, None, None, None, None, None)
+    args = lambda s, pr, b, o: lib.stepkv_select(256, 1, 100, 256, 256, ctypes.byref(s), ctypes.byref(pr),
+                                                 ctypes.byref(b), ctypes.byref(o), 256, 1 << 20, None, None)
+    assert args(steps, params, bud, out) == B.STEPKV_EINVAL          # n_steps = 0
+    steps.n_steps = 4
+    bad = B.budget_ratio(1, 0)
+    assert args(steps, params, bad, out) == B.STEPKV_EINVAL          # zero denominator
+    bad_norm = B.Params(sal_norm=7).c()
+    assert args(steps, bad_norm, bud, out) == B.STEPKV_EINVAL
+    out.kept_idx = None
+    assert args(steps, params, bud, out) == B.STEPKV_EINVAL
+
+
+def test_compact_rejects_bad_arguments_on_host(lib):
+    from paper_2609_22158_gb300 import binding as B
+    a = (ctypes.c_void_p * 1)(256)
+    same = ctypes.cast(a, ctypes.c_void_p)
+    other = ctypes.cast((ctypes.c_void_p * 1)(512), ctypes.c_void_p)
+    # in-place compaction is refused
+    assert lib.stepkv_compact(1, same, None, 128 * 100, 2, 128, 100, 256, 256, 50, same, None, 128 * 50,
+                              None, None, None, None, None, None) == B.STEPKV_EUNSUPPORTED
+    # misaligned row size (d*2 not a multiple of 16)
+    assert lib.stepkv_compact(1, same, None, 100 * 4, 2, 4, 100, 256, 256, 50, other, None, 4 * 50,
+                              None, None, None, None, None, None) == B.STEPKV_EINVAL
+    # output head stride too small for kept_cap
+    assert lib.stepkv_compact(1, same, None, 128 * 100, 2, 128, 100, 256, 256, 50, other, None, 128 * 49,
+                              None, None, None, None, None, None) == B.STEPKV_EINVAL
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    from paper_2609_22158_gb300 import binding
+    with pytest.raises(binding.StepKVError):
+        binding.load_library(str(tmp_path / "missing.so"))

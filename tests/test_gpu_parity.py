@@ -1,0 +1,374 @@
+"""GPU parity of every stage against the CPU oracle, through the C ABI (libstepkv.so).
+
+Sizes span several 128-key tiles with ragged tails, row groups above 256 query rows, windows split
+over row groups, d = 64 and 128, GQA groups 1/2/4/5, the paper's seeds (233, 42, 3407) and the
+full 32K-token, 32-layer workload the benchmark times.
+"""
+import numpy as np
+import pytest
+
+from oracle import stepkv_oracle as O
+from paper_2609_22158_gb300 import workload as wl
+import stepkv_testlib as TL
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def B():
+    import torch
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    from paper_2609_22158_gb300 import binding, build
+    build.build_library()
+    binding.load_library()
+    return binding
+
+
+def _rand_bits(rng, shape, scale=1.0):
+    return wl.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32) * np.float32(scale))
+
+
+# ------------------------------------------------------------------------------------ stage 1
+SCORE_CASES = [
+    # Hkv, G, d, T, W, n_layers
+    (2, 4, 64, 2048, 32, 1),     # tiny workload shape
+    (8, 4, 128, 4100, 64, 2),    # ragged T, one row group of 256
+    (2, 5, 128, 1000, 128, 1),   # 640 query rows -> 3 row groups
+    (1, 1, 128, 300, 1, 1),      # single query (textbook softmax case)
+    (2, 2, 64, 130, 7, 3),       # W not a multiple of 8
+    (1, 2, 128, 700, 300, 1),    # window split over two row groups
+    (4, 1, 64, 64, 64, 1),       # W = T, T below one tile
+    (2, 4, 128, 127, 5, 1),
+    (1, 8, 128, 513, 33, 1),     # 8 heads x 40 padded rows = 320 rows -> 2 row groups
+]
+
+
+@pytest.mark.parametrize("Hkv,G,d,T,W,nl", SCORE_CASES)
+def test_score_matches_oracle(B, Hkv, G, d, T, W, nl):
+    import torch
+    rng = np.random.default_rng(1000 + T + W)
+    Ks = [_rand_bits(rng, (Hkv, T, d)) for _ in range(nl)]
+    Qs = [_rand_bits(rng, (Hkv * G, W, d)) for _ in range(nl)]
+    st = B.new_status()
+    sal = B.stepkv_score([TL.bf16_dev(k) for k in Ks], [TL.bf16_dev(q) for q in Qs], T, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    g = sal.cpu().numpy()
+    for l in range(nl):
+        ref = O.window_attention_saliency(Ks[l], Qs[l])
+        TL.assert_close(g[l], ref, f"sal layer {l}")
+        assert np.allclose(g[l].sum(axis=1), W, rtol=1e-4)
+
+
+def test_score_capacity_head_stride(B):
+    """K rows live in a larger capacity buffer ([Hkv, cap, d] with cap > T)."""
+    import torch
+    rng = np.random.default_rng(7)
+    Hkv, G, d, T, W, cap = 2, 4, 128, 1500, 64, 2048
+    Kfull = _rand_bits(rng, (Hkv, cap, d))
+    Q = _rand_bits(rng, (Hkv * G, W, d))
+    Kd = TL.bf16_dev(Kfull)[:, :T]  # strided view: head stride cap*d
+    sal = B.stepkv_score([Kd], [TL.bf16_dev(Q)], T)
+    torch.cuda.synchronize()
+    ref = O.window_attention_saliency(np.ascontiguousarray(Kfull[:, :T]), Q)
+    TL.assert_close(sal[0].cpu().numpy(), ref, "sal (capacity layout)")
+
+
+def test_score_outlier_channels(B):
+    """Keys with 4 channels scaled x8 (the ragged-batch workload's outliers): wider logit range."""
+    import torch
+    tr = wl.custom(11, L=3, Hq=32, Hkv=8, d=128, T=3000, W=64, n_steps=6, outlier_channels=4)
+    Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+    Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+    sal = B.stepkv_score([TL.bf16_dev(k) for k in Ks], [TL.bf16_dev(q) for q in Qs], tr.T)
+    torch.cuda.synchronize()
+    for l in range(3):
+        TL.assert_close(sal[l].cpu().numpy(), O.window_attention_saliency(Ks[l], Qs[l]), "sal outliers")
+
+
+# ------------------------------------------------------------------------------------ stages 2-4
+def _select_case(B, tr, p, sal_fp32, kept_cap=None):
+    import torch
+    g = TL.GpuTraj.__new__(TL.GpuTraj)
+    g.tr = tr
+    g.step_id = torch.from_numpy(tr.step_id).cuda()
+    g.prot = torch.from_numpy(tr.prot).cuda()
+    g.valid = torch.from_numpy(tr.valid).cuda()
+    g.gain = torch.from_numpy(tr.gain).cuda()
+    g.red = torch.from_numpy(tr.red).cuda()
+    g.obs_sim = torch.from_numpy(tr.obs_sim).cuda()
+    g.reuse_in = torch.from_numpy(tr.reuse).cuda()
+    g.reuse_out = torch.empty_like(g.reuse_in)
+    cap = kept_cap if kept_cap is not None else tr.T
+    g.out = B.SelectOutputs.allocate(tr.T, tr.n_steps, cap, "cuda")
+    st = B.new_status()
+    b = tr.budget
+    bud = B.budget_ratio(b.num, b.den) if b.mode == "ratio" else B.budget_count(b.count)
+    B.stepkv_select(torch.from_numpy(sal_fp32).cuda(), g.step_id, g.prot, g.steps(), p, bud, g.out, status=st)
+    torch.cuda.synchronize()
+    A = [sal_fp32[i].astype(np.float64) for i in range(sal_fp32.shape[0])]
+    out = O.stepkv_boundary([a[None] for a in A], tr.step_id, tr.prot, tr.valid, tr.gain, tr.red, tr.obs_sim,
+                            tr.reuse, TL.oracle_params(p), b.mode, b.num, b.den, b.count)
+    return g, out, int(st.item())
+
+
+@pytest.mark.parametrize("seed", [0, 233, 42, 3407])
+def test_select_matches_oracle(B, seed):
+    tr = wl.tiny(seed)
+    Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+    Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+    sal = np.concatenate([O.window_attention_saliency(k, q) for k, q in zip(Ks, Qs)]).astype(np.float32)
+    g, out, st = _select_case(B, tr, B.Params(), sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
+@pytest.mark.parametrize("budget", [wl.Budget.ratio(1, 10), wl.Budget.ratio(1, 2), wl.Budget.fixed(1),
+                                    wl.Budget.fixed(5000), wl.Budget.ratio(1, 1), wl.Budget.fixed(0)])
+def test_select_budgets(B, budget):
+    tr = wl.custom(5, L=1, Hq=4, Hkv=1, d=64, T=4000, W=16, n_steps=9, budget=budget)
+    rng = np.random.default_rng(3)
+    sal = (rng.random((2, tr.T)) * 3).astype(np.float32)
+    g, out, st = _select_case(B, tr, B.Params(), sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
+@pytest.mark.parametrize("levels", [2, 7, 1000])
+def test_select_exact_on_shared_fp32_priorities(B, levels):
+    """alpha=1, beta=0, no normalisation, one saliency row: the kernel ranks exactly the fp32 values
+    it is given, so its retained set must equal the oracle's ranking of the same values bit for bit,
+    ties (few distinct levels) included."""
+    import torch
+    T = 20000
+    tr = wl.custom(9, L=1, Hq=1, Hkv=1, d=64, T=T, W=8, n_steps=12, budget=wl.Budget.ratio(3, 10))
+    rng = np.random.default_rng(levels)
+    sal = (rng.integers(0, levels, (1, T)) / levels).astype(np.float32)
+    p = B.Params(alpha=1.0, beta=0.0, sal_norm=B.NORM_NONE)
+    g, out, st = _select_case(B, tr, p, sal)
+    assert st == 0
+    n = int(g.out.n_kept.item())
+    gk = g.out.kept_idx[:n].cpu().numpy()
+    prunable = ~tr.prot.astype(bool)
+    Bt = O.budget_tokens(int(prunable.sum()), "ratio", 3, 10)
+    exp = O.kept_indices(tr.prot, O.select_top(sal[0].astype(np.float64), prunable, Bt))
+    assert np.array_equal(gk, exp)
+    assert np.array_equal(g.out.step_kept.cpu().numpy(), out["step_kept"])
+
+
+def test_select_large_T(B):
+    """T = 200000 (beyond 8 x 16K): every CTA of the cluster holds ~25K tokens."""
+    T = 200000
+    tr = wl.custom(21, L=1, Hq=8, Hkv=2, d=64, T=T, W=64, n_steps=150, budget=wl.Budget.fixed(8192))
+    rng = np.random.default_rng(21)
+    sal = rng.random((6, T)).astype(np.float32) ** 4
+    g, out, st = _select_case(B, tr, B.Params(), sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
+def test_select_bad_step_id_sets_edata(B):
+    tr = wl.custom(4, L=1, Hq=2, Hkv=1, d=64, T=600, W=8, n_steps=3)
+    tr.step_id = tr.step_id.copy()
+    assert tr.prot[300] == 0
+    tr.step_id[300] = 3  # == n_steps: out of range
+    g, _, st = _select_case_status(B, tr, np.ones((1, tr.T), np.float32))
+    assert st == B.STEPKV_EDATA
+    assert int(g.out.n_kept.item()) == 0
+
+
+def _select_case_status(B, tr, sal):
+    import torch
+    g = TL.GpuTraj.__new__(TL.GpuTraj)
+    g.tr = tr
+    step_id = torch.from_numpy(tr.step_id).cuda()
+    prot = torch.from_numpy(tr.prot).cuda()
+    steps = B.StepSignals(*(torch.from_numpy(a).cuda() for a in (tr.valid, tr.gain, tr.red, tr.reuse)))
+    g.out = B.SelectOutputs.allocate(tr.T, tr.n_steps, tr.T, "cuda")
+    st = B.new_status()
+    B.stepkv_select(torch.from_numpy(sal).cuda(), step_id, prot, steps, B.Params(), B.budget_ratio(1, 2), g.out,
+                    status=st)
+    torch.cuda.synchronize()
+    return g, None, int(st.item())
+
+
+# ------------------------------------------------------------------------------------ stage 5
+@pytest.mark.parametrize("d", [64, 128])
+def test_compact_bit_exact(B, d):
+    import torch
+    rng = np.random.default_rng(d)
+    L, Hkv, T, cap = 3, 4, 3001, 1200
+    Kin = [_rand_bits(rng, (Hkv, T, d)) for _ in range(L)]
+    Vin = [_rand_bits(rng, (Hkv, T, d)) for _ in range(L)]
+    kept = np.sort(rng.choice(T, 1111, replace=False)).astype(np.int32)
+    step_in = rng.integers(-1, 50, T).astype(np.int32)
+    pos_in = (np.arange(T) * 3 + 7).astype(np.int32)
+    Kout = [torch.zeros((Hkv, cap, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+    Vout = [torch.zeros((Hkv, cap, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+    kd = torch.zeros(cap, dtype=torch.int32, device="cuda")
+    kd[:len(kept)] = torch.from_numpy(kept).cuda()
+    nk = torch.tensor([len(kept)], dtype=torch.int32, device="cuda")
+    so = torch.full((cap,), -9, dtype=torch.int32, device="cuda")
+    po = torch.full((cap,), -9, dtype=torch.int32, device="cuda")
+    st = B.new_status()
+    B.stepkv_compact([TL.bf16_dev(k) for k in Kin], [TL.bf16_dev(v) for v in Vin], T, kd, nk, cap, Kout, Vout,
+                     torch.from_numpy(step_in).cuda(), torch.from_numpy(pos_in).cuda(), so, po, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for l in range(L):
+        assert np.array_equal(TL.bits_of(Kout[l])[:, :len(kept)], O.compact_rows(Kin[l], kept))
+        assert np.array_equal(TL.bits_of(Vout[l])[:, :len(kept)], O.compact_rows(Vin[l], kept))
+        assert np.all(TL.bits_of(Kout[l])[:, len(kept):] == 0)  # rows past n_kept untouched
+    assert np.array_equal(so.cpu().numpy()[:len(kept)], step_in[kept])
+    assert np.array_equal(po.cpu().numpy()[:len(kept)], pos_in[kept])
+    assert np.all(so.cpu().numpy()[len(kept):] == -9)
+
+
+def test_compact_rejects_overflow_on_device(B):
+    import torch
+    T, cap = 100, 10
+    K = [torch.zeros((1, T, 64), dtype=torch.bfloat16, device="cuda")]
+    Ko = [torch.zeros((1, cap, 64), dtype=torch.bfloat16, device="cuda")]
+    kd = torch.arange(cap, dtype=torch.int32, device="cuda")
+    nk = torch.tensor([cap + 1], dtype=torch.int32, device="cuda")
+    st = B.new_status()
+    B.stepkv_compact(K, None, T, kd, nk, cap, Ko, None, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == B.STEPKV_ENOSPACE
+
+
+# ------------------------------------------------------------------------------------ fused pass
+def _compress_and_check(B, tr, p=None, layers_check=None, kept_cap=None):
+    import torch
+    p = p or B.Params()
+    g = TL.GpuTraj(tr, kept_cap=kept_cap)
+    prob = g.problem()
+    st = B.stepkv_compress([prob], p)
+    torch.cuda.synchronize()
+    assert st.item() == 0, st.item()
+    out = TL.run_oracle(tr, TL.oracle_params(p))
+    swaps = TL.check_select_outputs(g, out)
+    n = int(g.out.n_kept.item())
+    gk = g.out.kept_idx[:n].cpu().numpy()
+    for l in (layers_check if layers_check is not None else range(tr.shape.L)):
+        assert np.array_equal(TL.bits_of(g.K_out[l])[:, :n], O.compact_rows(tr.keys(l), gk))
+        assert np.array_equal(TL.bits_of(g.V_out[l])[:, :n], O.compact_rows(tr.values(l), gk))
+    assert np.array_equal(g.step_id_out[:n].cpu().numpy(), tr.step_id[gk])
+    assert np.array_equal(g.pos_out[:n].cpu().numpy(), tr.pos[gk])
+    return g, out, swaps
+
+
+@pytest.mark.parametrize("seed", [0, 233, 42, 3407])
+def test_compress_tiny(B, seed):
+    _compress_and_check(B, wl.tiny(seed))
+
+
+def test_compress_medium_gqa5_w128(B):
+    tr = wl.custom(77, L=5, Hq=10, Hkv=2, d=128, T=6000, W=128, n_steps=14, budget=wl.Budget.fixed(700))
+    _compress_and_check(B, tr)
+
+
+def test_compress_llama_shape_short(B):
+    tr = wl.llama8b_32k(seed=5, T=8192, L=4)
+    _compress_and_check(B, tr)
+
+
+def test_compress_batched_ragged(B):
+    import torch
+    trs = [wl.custom(100 + i, L=3, Hq=8, Hkv=2, d=128, T=T, W=32, n_steps=5 + i, budget=wl.Budget.ratio(1, 5))
+           for i, T in enumerate((1700, 2600, 999))]
+    gs = [TL.GpuTraj(tr) for tr in trs]
+    probs = [g.problem() for g in gs]
+    st = B.stepkv_compress(probs, B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for g, tr in zip(gs, trs):
+        out = TL.run_oracle(tr, TL.oracle_params(B.Params()))
+        TL.check_select_outputs(g, out)
+        n = int(g.out.n_kept.item())
+        gk = g.out.kept_idx[:n].cpu().numpy()
+        assert np.array_equal(TL.bits_of(g.K_out[0])[:, :n], O.compact_rows(tr.keys(0), gk))
+
+
+def test_compress_all_protected(B):
+    """N_t = 0: nothing is prunable, every slot is kept, B_t = 0."""
+    import torch
+    tr = wl.custom(3, L=2, Hq=4, Hkv=2, d=64, T=500, W=16, n_steps=2)
+    tr.prot = np.ones(tr.T, np.uint8)
+    g, out, _ = _compress_and_check(B, tr)
+    assert out["N"] == 0 and out["B"] == 0 and int(g.out.n_kept.item()) == tr.T
+
+
+def test_compress_step_without_prunable_tokens(B):
+    tr = wl.custom(8, L=2, Hq=4, Hkv=2, d=64, T=2500, W=16, n_steps=6)
+    k = 2
+    tr.prot = tr.prot.copy()
+    tr.prot[tr.step_id == k] = 1
+    g, out, _ = _compress_and_check(B, tr)
+    assert out["step_count"][k] == 0 and g.out.step_count[k].item() == 0
+
+
+def test_compress_single_step(B):
+    tr = wl.custom(12, L=1, Hq=4, Hkv=1, d=128, T=900, W=32, n_steps=1, budget=wl.Budget.ratio(1, 3))
+    _compress_and_check(B, tr)
+
+
+def test_compress_kept_cap_too_small(B):
+    import torch
+    tr = wl.tiny(1)
+    g = TL.GpuTraj(tr, kept_cap=100)
+    st = B.stepkv_compress([g.problem()], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == B.STEPKV_ENOSPACE
+
+
+def test_compress_deterministic(B):
+    import torch
+    tr = wl.custom(31, L=3, Hq=8, Hkv=2, d=128, T=5000, W=64, n_steps=10)
+    res = []
+    for _ in range(2):
+        g = TL.GpuTraj(tr)
+        B.stepkv_compress([g.problem()], B.Params())
+        torch.cuda.synchronize()
+        res.append([g.out.kept_idx.cpu(), g.out.priority.cpu(), g.out.token_sal.cpu(), g.out.step_sal_sum.cpu(),
+                    g.K_out[0].cpu(), g.V_out[2].cpu()])
+    for a, b in zip(*res):
+        assert torch.equal(a.contiguous().view(torch.uint8), b.contiguous().view(torch.uint8))
+
+
+@pytest.mark.slow
+def test_compress_full_32k_32layer(B):
+    """The benchmark's workload (Llama-3-8B shape, T = 32768, 32 layers, 10% budget), in the same
+    fused call the benchmark times: saliency layers from the shared generator, the other layers'
+    K/V drawn on the device; selection checked against the oracle, compaction checked row for row
+    against the oracle's retained slots."""
+    import torch
+    tr = wl.llama8b_32k(seed=1)
+    s = tr.shape
+    gen = torch.Generator(device="cuda").manual_seed(1234)
+    sal_ids = set(tr.sal_layer_ids())
+    K = [TL.bf16_dev(tr.keys(l)) if l in sal_ids else
+         torch.randn((s.Hkv, s.T, s.d), generator=gen, device="cuda", dtype=torch.bfloat16) for l in range(s.L)]
+    V = [torch.randn((s.Hkv, s.T, s.d), generator=gen, device="cuda", dtype=torch.bfloat16) for _ in range(s.L)]
+    g = TL.GpuTraj.__new__(TL.GpuTraj)
+    g.tr = tr
+    g.K, g.V = K, V
+    g.Q = [TL.bf16_dev(tr.queries(l)) for l in tr.sal_layer_ids()]
+    for nm, arr in (("step_id", tr.step_id), ("prot", tr.prot), ("pos", tr.pos), ("valid", tr.valid),
+                    ("gain", tr.gain), ("red", tr.red), ("obs_sim", tr.obs_sim), ("reuse_in", tr.reuse)):
+        setattr(g, nm, torch.from_numpy(arr).cuda())
+    g.reuse_out = torch.empty_like(g.reuse_in)
+    g.kept_cap = 4096
+    prob = g.problem()
+    st = B.stepkv_compress([prob], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    out = TL.run_oracle(tr, TL.oracle_params(B.Params()))
+    swaps = TL.check_select_outputs(g, out)
+    n = int(g.out.n_kept.item())
+    assert n == 16 + 64 + 3268
+    kept = g.out.kept_idx[:n].long()
+    for l in range(s.L):
+        assert torch.equal(g.K_out[l][:, :n], K[l].index_select(1, kept))
+        assert torch.equal(g.V_out[l][:, :n], V[l].index_select(1, kept))
+    print(f"full-size swaps: {swaps}")

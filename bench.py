@@ -109,10 +109,7 @@ class DeviceTraj:
 def launches_per_pass(tr) -> int:
     """Kernel launches of one stepkv_compress call (mirrors the library's launch plan)."""
     s = tr.shape
-    n_pairs = s.Ls * s.Hkv
-    ppg = min(n_pairs, max(1, int(80e6 // (s.T * s.d * 2))))
-    groups = math.ceil(n_pairs / ppg)
-    return 2 * groups + 1 + math.ceil(s.L / 96)
+    return 2 + 1 + math.ceil(s.L / 96)  # score pass 1, pass 2, select, compaction
 
 
 def algorithmic_bytes(tr, n_kept):

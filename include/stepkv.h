@@ -190,7 +190,7 @@ STEPKV_API stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, 
  *  steps, params, budget: host structs (device arrays inside steps).
  *  out       host struct of device output pointers (see stepkv_select_out_t).
  *  Ranking: (P_i descending, slot index ascending) -- on equal priority the older token wins.
- *  Supported: 1 <= T <= 262144, 1 <= n_steps <= 65536, n_sal >= 1.
+ *  Supported: 1 <= T <= 262144, 1 <= n_steps <= 65535, n_sal >= 1.
  */
 STEPKV_API size_t stepkv_select_workspace_size(int32_t n_sal, int32_t T, int32_t n_steps);
 STEPKV_API stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T,
@@ -208,8 +208,8 @@ STEPKV_API stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_
  *  n_kept is read on the device (no host synchronisation); *n_kept > kept_cap or a kept index
  *  outside [0, T) sets STEPKV_ENOSPACE / STEPKV_EDATA and skips the bad rows.
  *  V_in/V_out may be NULL (keys only); step/pos pointers may be NULL.
- *  Rows are d bf16 values; d*2 bytes must be a multiple of 16; bases 16-byte aligned; in/out head
- *  strides % 8 == 0.  In-place compaction (K_out == K_in) is not supported.
+ *  Rows are d bf16 values; d*2 bytes must be a multiple of 16 and d <= 256; bases 16-byte aligned;
+ *  in/out head strides % 8 == 0.  In-place compaction (K_out == K_in) is not supported.
  */
 STEPKV_API stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
                                int64_t in_head_stride, int32_t Hkv, int32_t d, int32_t T,

@@ -1,5 +1,6 @@
 // C ABI of the StepKV compression pass: argument validation, workspace layout, and the order of
 // kernel launches.  Every function only enqueues work on the caller's stream.
+#include <math.h>
 #include <stdio.h>
 
 #include <algorithm>
@@ -67,7 +68,7 @@ static stepkv_status_t check_select_args(int n_sal, int T, const int32_t* step_i
   if (!steps || !params || !budget || !out || !step_id || !prot) return STEPKV_EINVAL;
   if (n_sal < 1 || T < 1) return STEPKV_EINVAL;
   if (T > 262144) return STEPKV_EUNSUPPORTED;
-  if (steps->n_steps < 1 || steps->n_steps > 65536) return STEPKV_EINVAL;
+  if (steps->n_steps < 1 || steps->n_steps > 65535) return STEPKV_EINVAL;
   if (!steps->valid || !steps->gain || !steps->red || !steps->reuse_in) return STEPKV_EINVAL;
   if (!out->kept_idx || !out->n_kept || out->kept_cap < 0) return STEPKV_EINVAL;
   if (params->sal_norm != STEPKV_NORM_MAX && params->sal_norm != STEPKV_NORM_NONE) return STEPKV_EINVAL;
@@ -87,7 +88,7 @@ static stepkv_status_t check_compact_args(int n_layers, const void* const* K_in,
                                           void* const* V_out, int64_t out_head_stride) {
   if (n_layers < 0 || Hkv < 1 || d < 8 || T < 1 || kept_cap < 0) return STEPKV_EINVAL;
   if (!kept_idx || !n_kept) return STEPKV_EINVAL;
-  if ((d * 2) % 16) return STEPKV_EUNSUPPORTED;
+  if ((d * 2) % 16 || d > 256) return STEPKV_EUNSUPPORTED;
   if (n_layers > 0) {
     if (!K_in || !K_out) return STEPKV_EINVAL;
     if ((V_in == nullptr) != (V_out == nullptr)) return STEPKV_EINVAL;
@@ -171,7 +172,8 @@ stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_h
   float* rows = sal;
   if (n_rg > 1)
     rows = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + align256(score_partial_bytes(n_layers, Hkv, Hq, W)));
-  st = score_run(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W, rows, T, part, dev_status, s);
+  st = score_run(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W, rows, T, nullptr, 0, part,
+                 dev_status, s);
   if (st != STEPKV_OK) return st;
   if (n_rg > 1) st = score_sum_row_groups(rows, n_layers * Hkv, n_rg, T, sal, s);
   return st;
@@ -180,7 +182,7 @@ stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_h
 size_t stepkv_select_workspace_size(int32_t n_sal, int32_t T, int32_t n_steps) {
   (void)n_sal;
   if (T < 1 || n_steps < 1) return 0;
-  return select_ws_bytes(T, n_steps);
+  return align256((size_t)T * sizeof(float)) + select_ws_bytes(T, n_steps);
 }
 
 stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T, const int32_t* step_id,
@@ -190,10 +192,14 @@ stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T, const 
   stepkv_status_t st = check_select_args(n_sal, T, step_id, prot, steps, params, budget, out);
   if (st != STEPKV_OK) return st;
   if (!sal || !ws) return STEPKV_EINVAL;
-  if (ws_bytes < select_ws_bytes(T, steps->n_steps)) return STEPKV_ENOSPACE;
+  if (ws_bytes < stepkv_select_workspace_size(n_sal, T, steps->n_steps)) return STEPKV_ENOSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
-  return select_run(sal, n_sal, T, 1.0f / (float)n_sal, T, step_id, prot, *steps, *params, *budget, *out, ws,
-                    dev_status, static_cast<cudaStream_t>(stream));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* Tbuf = static_cast<float*>(ws);
+  void* sel_ws = static_cast<uint8_t*>(ws) + align256((size_t)T * sizeof(float));
+  st = mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, Tbuf, s);
+  if (st != STEPKV_OK) return st;
+  return select_run(Tbuf, nullptr, 0.0, T, step_id, prot, *steps, *params, *budget, *out, sel_ws, dev_status, s);
 }
 
 stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
@@ -211,9 +217,8 @@ stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const 
 
 static size_t compress_ws_one(const stepkv_problem_t& p) {
   const int Ls = std::min(p.n_sal_layers, p.L);
-  const int n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
   size_t b = align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
-  b += align256((size_t)Ls * p.Hkv * n_rg * p.T * sizeof(float));
+  b += align256((size_t)p.T * sizeof(unsigned long long));
   b += align256(select_ws_bytes(p.T, p.steps.n_steps));
   return b;
 }
@@ -255,18 +260,19 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     const int Ls = std::min(p.n_sal_layers, p.L);
-    const int n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
     uint8_t* w = static_cast<uint8_t*>(ws);
     float2* part = reinterpret_cast<float2*>(w);
     w += align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
-    float* rows = reinterpret_cast<float*>(w);
-    w += align256((size_t)Ls * p.Hkv * n_rg * p.T * sizeof(float));
+    unsigned long long* t_acc = reinterpret_cast<unsigned long long*>(w);
+    w += align256((size_t)p.T * sizeof(unsigned long long));
     void* sel_ws = w;
+    const int n_pairs = Ls * p.Hkv;
+    const int shift = score_acc_shift(n_pairs, p.W);
     stepkv_status_t st = score_run(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
-                                   p.T, p.W, rows, p.T, part, dev_status, s);
+                                   p.T, p.W, nullptr, 0, t_acc, shift, part, dev_status, s);
     if (st != STEPKV_OK) return st;
-    st = select_run(rows, Ls * p.Hkv * n_rg, p.T, 1.0f / (float)(Ls * p.Hkv), p.T, p.step_id, p.prot, p.steps,
-                    *params, p.budget, p.sel, sel_ws, dev_status, s);
+    st = select_run(nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps, *params,
+                    p.budget, p.sel, sel_ws, dev_status, s);
     if (st != STEPKV_OK) return st;
     st = compact_run(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap,
                      p.K_out, p.V_out, p.out_head_stride, p.step_id, p.pos_in, p.step_id_out, p.pos_out, dev_status,

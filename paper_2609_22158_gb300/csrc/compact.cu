@@ -1,11 +1,12 @@
 // Stage 5 -- compaction of the retained rows (Eq. 1: C_hat = C_prot || C_traj[K]).
 //   out[l][h][r][:] = in[l][h][kept_idx[r]][:]  for every layer, KV head and tensor (K, V)
 //
-// GB300 design: a pure HBM copy (about 4/5 of the pass's bytes).  Each CTA owns a block of 64
-// retained rows, keeps their source indices in registers/shared memory, and walks a slice of the
-// (layer, tensor, head) row sets.  Each thread moves 16-byte vectors with streaming loads/stores
-// (the data is touched once; keep it from evicting the L2-resident score data); four independent
-// vectors per thread are in flight before the first store.  n_kept is read on the device.
+// GB300 design: a pure HBM copy (about 4/5 of the pass's bytes).  The work is the list of row items
+// (row set, retained row), row set = (layer, tensor, KV head); a persistent grid of 8 CTAs per SM splits
+// it into equal contiguous ranges, so every SM streams the same number of rows.  A row of d bf16 is
+// d/8 16-byte vectors handled by d/8 lanes, so a warp moves 32/(d/8) rows per instruction; four such
+// groups are loaded before the first store (8 rows, 2 KB per warp in flight at d = 128).  Loads and
+// stores are streaming (.cs): the data is touched once.  n_kept is read on the device.
 #include <algorithm>
 
 #include "common.cuh"
@@ -14,15 +15,14 @@
 namespace stepkv {
 
 constexpr int kCompactThreads = 256;
-constexpr int kCompactRows = 64;       // retained rows per CTA
-constexpr int kCompactSetsPerCta = 16; // (layer, tensor, head) row sets per CTA
+constexpr int kCompactCtasPerSm = 8;
+constexpr int kCompactUnroll = 4;
 constexpr int kCompactLayersPerLaunch = 96;
 
 struct CompactArgs {
   const uint8_t* src[2 * kCompactLayersPerLaunch];  // per (layer, tensor): base of [Hkv][rows][d]
   uint8_t* dst[2 * kCompactLayersPerLaunch];
   int n_sets;               // n_layers_in_launch * n_tensors * Hkv
-  int n_tensors;            // 1 (K only) or 2
   int Hkv;
   int row_bytes;            // d * 2
   int64_t in_head_bytes;
@@ -49,59 +49,54 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 }
 
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_constant__ CompactArgs a) {
-  __shared__ int s_src[kCompactRows];
   pdl_wait();  // kept_idx / n_kept come from the selection kernel
   pdl_launch_dependents();
   const int n_kept = *a.n_kept;
   if (n_kept > a.kept_cap || n_kept < 0) {
-    if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) record_status(a.status, STEPKV_ENOSPACE);
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_status(a.status, STEPKV_ENOSPACE);
     return;
   }
-  const int r0 = blockIdx.x * kCompactRows;
-  if (r0 >= n_kept) return;
-  const int nr = min(kCompactRows, n_kept - r0);
-  if (threadIdx.x < kCompactRows) {
-    int s = -1;
-    if ((int)threadIdx.x < nr) {
-      s = a.kept_idx[r0 + threadIdx.x];
-      if (s < 0 || s >= a.T) {
-        record_status(a.status, STEPKV_EDATA);
-        s = -1;
-      }
-    }
-    s_src[threadIdx.x] = s;
-    if (a.gather_meta && blockIdx.y == 0 && (int)threadIdx.x < nr) {
-      const int r = r0 + threadIdx.x;
-      if (a.step_id_out) a.step_id_out[r] = (s >= 0 && a.step_id_in) ? a.step_id_in[s] : -1;
-      if (a.pos_out) a.pos_out[r] = s < 0 ? -1 : (a.pos_in ? a.pos_in[s] : s);
+  if (a.gather_meta) {
+    for (int r = blockIdx.x * kCompactThreads + threadIdx.x; r < n_kept; r += gridDim.x * kCompactThreads) {
+      const int s = a.kept_idx[r];
+      const bool ok = s >= 0 && s < a.T;
+      if (!ok) record_status(a.status, STEPKV_EDATA);
+      if (a.step_id_out) a.step_id_out[r] = (ok && a.step_id_in) ? a.step_id_in[s] : -1;
+      if (a.pos_out) a.pos_out[r] = ok ? (a.pos_in ? a.pos_in[s] : s) : -1;
     }
   }
-  __syncthreads();
-  const int vpr = a.row_bytes >> 4;  // 16-byte vectors per row
-  const int nvec = nr * vpr;
-  const int set_lo = blockIdx.y * kCompactSetsPerCta;
-  const int set_hi = min(a.n_sets, set_lo + kCompactSetsPerCta);
-  for (int set = set_lo; set < set_hi; ++set) {
-    const int h = set % a.Hkv;
-    const int lt = set / a.Hkv;  // layer*n_tensors + tensor
-    const uint8_t* src = a.src[lt] + (int64_t)h * a.in_head_bytes;
-    uint8_t* dst = a.dst[lt] + (int64_t)h * a.out_head_bytes + (int64_t)r0 * a.row_bytes;
-    for (int v0 = threadIdx.x; v0 < nvec; v0 += 4 * kCompactThreads) {
-      uint4 buf[4];
-      int rr[4], cc[4];
+  const int64_t total = (int64_t)a.n_sets * n_kept;  // row items
+  const int64_t per_cta = (total + gridDim.x - 1) / gridDim.x;
+  const int64_t lo = blockIdx.x * per_cta;
+  const int64_t hi = min(total, lo + per_cta);
+  const int vpr = a.row_bytes >> 4;      // lanes per row
+  const int rpw = 32 / vpr;              // rows per warp instruction
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int sub_row = lane / vpr, col = lane - sub_row * vpr;
+  const bool lane_active = sub_row < rpw;  // d/8 need not divide 32: the spare lanes idle
+  const int64_t step = (int64_t)(kCompactThreads / 32) * rpw * kCompactUnroll;
+  for (int64_t base = lo + (int64_t)warp * rpw * kCompactUnroll; base < hi; base += step) {
+    uint4 buf[kCompactUnroll];
+    uint4* dptr[kCompactUnroll];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int v = v0 + u * kCompactThreads;
-        rr[u] = v / vpr;
-        cc[u] = v - rr[u] * vpr;
-        const int s = v < nvec ? s_src[rr[u]] : -1;
-        if (s >= 0) buf[u] = ld_stream(reinterpret_cast<const uint4*>(src + (int64_t)s * a.row_bytes) + cc[u]);
-        else rr[u] = -1;
+    for (int u = 0; u < kCompactUnroll; ++u) {
+      const int64_t ri = base + u * rpw + sub_row;
+      dptr[u] = nullptr;
+      if (lane_active && ri < hi) {
+        const int set = (int)(ri / n_kept);
+        const int r = (int)(ri - (int64_t)set * n_kept);
+        const int s = __ldg(&a.kept_idx[r]);
+        if (s >= 0 && s < a.T) {
+          const int lt = set / a.Hkv, h = set - lt * a.Hkv;
+          const uint8_t* src = a.src[lt] + (int64_t)h * a.in_head_bytes + (int64_t)s * a.row_bytes;
+          buf[u] = ld_stream(reinterpret_cast<const uint4*>(src) + col);
+          dptr[u] = reinterpret_cast<uint4*>(a.dst[lt] + (int64_t)h * a.out_head_bytes + (int64_t)r * a.row_bytes) + col;
+        }
       }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (rr[u] >= 0) st_stream(reinterpret_cast<uint4*>(dst + (int64_t)rr[u] * a.row_bytes) + cc[u], buf[u]);
     }
+#pragma unroll
+    for (int u = 0; u < kCompactUnroll; ++u)
+      if (dptr[u]) st_stream(dptr[u], buf[u]);
   }
 }
 
@@ -124,7 +119,6 @@ stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* c
       }
     }
     a.n_sets = std::max(nl, 0) * n_tensors * Hkv;
-    a.n_tensors = n_tensors;
     a.Hkv = Hkv;
     a.row_bytes = d * 2;
     a.in_head_bytes = in_head_stride * 2;
@@ -139,9 +133,14 @@ stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* c
     a.pos_out = pos_out;
     a.gather_meta = l0 == 0;
     a.status = status;
-    const int gx = std::max(1, (kept_cap + kCompactRows - 1) / kCompactRows);
-    const int gy = std::max(1, (a.n_sets + kCompactSetsPerCta - 1) / kCompactSetsPerCta);
-    cudaError_t e = launch_pdl(compact_kernel, dim3(gx, gy), dim3(kCompactThreads), 0, stream, a);
+    int n_sm = 0;
+    cudaError_t e = device_sm_count(&n_sm);
+    if (e == cudaSuccess) {
+      const int64_t rows_max = (int64_t)std::max(a.n_sets, 1) * std::max(kept_cap, 1);
+      const int64_t want = (rows_max + 31) / 32;  // no more CTAs than 32 row items each at full capacity
+      const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * kCompactCtasPerSm, want));
+      e = launch_pdl(compact_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a);
+    }
     if (e != cudaSuccess) {
       set_last_cuda_error(e);
       return STEPKV_ECUDA;

@@ -14,7 +14,6 @@ namespace stepkv {
 
 constexpr int kMaxSalLayers = 8;        // saliency layers per score launch (tensor maps in kernel params)
 constexpr int kMaxGrid = 1024;          // upper bound on the persistent score grid (partial-slot sizing)
-constexpr double kL2GroupBytes = 80e6;  // K bytes per score launch group (re-read from L2 by pass 2)
 constexpr int kMaxCompactLayers = 256;  // layers per compaction launch (pointer tables in kernel params)
 
 void set_last_cuda_error(cudaError_t e);
@@ -64,19 +63,26 @@ cudaError_t launch_pdl_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, in
 // ---- score (score.cu)
 int score_row_groups(int Hkv, int Hq, int W);
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W);
-// Writes pass-2 rows: row (pair*n_rg + rg) of rows_out (stride out_stride) for pair = layer*Hkv + h.
+int score_acc_shift(int n_pairs, int W);
+// Pass 2 either writes rows (row pair*n_rg + rg of rows_out, stride out_stride, pair = layer*Hkv + h) or,
+// when t_acc is non-null, adds every contribution to the per-token fixed-point sum t_acc[T] (scale
+// 2^acc_shift; the first launch zeroes it).
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
-                          int64_t out_stride, float2* part, int32_t* status, cudaStream_t stream);
+                          int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
+                          cudaStream_t stream);
 stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal, cudaStream_t stream);
 
 // ---- select (select.cu)
 size_t select_ws_bytes(int T, int n_steps);
-// rows: n_rows saliency rows of length T (stride row_stride); T_i = inv_div * sum of the rows.
-stepkv_status_t select_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T,
+// Token saliency comes either as floats T_in[T] or as fixed-point sums t_acc[T] with T_i = t_acc * acc_to_T.
+stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, double acc_to_T, int T,
                            const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
                            const stepkv_params_t& params, const stepkv_budget_t& budget,
                            const stepkv_select_out_t& out, void* ws, int32_t* status, cudaStream_t stream);
+// T_out[j] = inv_div * sum_r rows[r * row_stride + j] (fixed order over r).
+stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, float* T_out,
+                              cudaStream_t stream);
 
 // ---- compact (compact.cu)
 stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* const* V_in, int64_t in_head_stride,

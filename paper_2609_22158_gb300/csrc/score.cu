@@ -23,8 +23,8 @@
 
 namespace stepkv {
 
-constexpr int kThreads = 320;   // warp 0: TMA producer, warp 1: MMA issuer + TMEM owner, warps 2..9: epilogue
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;   // four warps per TMEM lane quarter
+constexpr int kThreads = 64 + kEpiWarps * 32;  // warp 0: TMA producer, warp 1: MMA issuer + TMEM owner, rest: epilogue
 constexpr int kKeyTile = 128;
 constexpr int kMaxRows = 256;   // query rows per row group
 constexpr int kTmemCols = 512;  // two accumulator buffers of 256 columns
@@ -52,8 +52,11 @@ struct ScoreLaunch {
   int n_units;        // units = pairs of this launch x n_rg
   int tpc;            // tiles per CTA (contiguous range)
   float2* part;       // pass-1 partials: slot (unit + cta) x 256 rows
-  float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride
+  float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when t_acc == nullptr)
   int64_t out_stride;
+  unsigned long long* t_acc;  // pass 2: per-token fixed-point sum over all (pair, row group) (when non-null)
+  float acc_scale;    // 2^k: fixed-point scale of t_acc
+  int zero_acc;       // pass 1: zero t_acc[0..T) first (first launch of a compression pass)
   int32_t* status;
 };
 
@@ -89,8 +92,8 @@ struct ScoreCfg {
   static constexpr int kStageBytes = NCH * kKChunkBytes;
   static constexpr int kOffOff = kQBytes + kStages * kStageBytes;  // float sOff[256]
   static constexpr int kPwOff = kOffOff + kMaxRows * 4;            // int   sPw[256]
-  static constexpr int kCombOff = kPwOff + kMaxRows * 4;           // 2 KB: float2[256] (pass 1) / float[2][128] (pass 2)
-  static constexpr int kBarOff = kCombOff + kMaxRows * 8;
+  static constexpr int kCombOff = kPwOff + kMaxRows * 4;           // 4 KB: float2[4][128] (pass 1) / float[2][4][128] (pass 2)
+  static constexpr int kBarOff = kCombOff + 4096;
   static constexpr int kNumBars = 2 * kStages + 2 + 4 + 1;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;          // tmem base, abort flag
   static constexpr int kBytes = kMiscOff + 16;
@@ -140,6 +143,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   const int U = p.n_units * g.n_tiles;
   const int t_lo = blockIdx.x * p.tpc;
   const int t_hi = min(U, t_lo + p.tpc);
+  const int n_my = t_hi - t_lo;
+  // Pass 2 walks the CTA's tile range backwards: the tiles pass 1 streamed last are still in L2.
+  auto tile_at = [&](int k) { return PASS == 1 ? t_lo + k : t_hi - 1 - k; };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -171,19 +177,24 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  pdl_wait();  // K/Q (possibly written by an earlier compaction) and pass-1 partials are complete
+  // Pass 1 waits for every earlier kernel on the stream (one of them may have written K/Q).  Pass 2 is
+  // launched only after all pass-1 CTAs passed that wait, so its K/Q loads may start at once; only the
+  // epilogue, which reads the pass-1 partials, waits for pass 1 to complete.
+  if (PASS == 1) pdl_wait();
   pdl_launch_dependents();
+  if (PASS == 1 && p.zero_acc) {
+    for (int i = blockIdx.x * kThreads + threadIdx.x; i < g.T; i += gridDim.x * kThreads) p.t_acc[i] = 0ull;
+  }
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (one thread)
     if (lane == 0) {
       int stage = 0, cur = -1;
-      uint32_t phase = 0, qe_phase = 0, q_issue_phase = 0;
-      uint32_t last_parity[S];
-      bool used[S];
-      for (int i = 0; i < S; ++i) used[i] = false;
-      bool q_used = false, ok = true;
-      for (int gt = t_lo; gt < t_hi; ++gt) {
+      uint32_t phase = 0, qe_phase = 0, q_issued = 0;
+      uint32_t used = 0, last_par = 0;  // per-stage bit: loaded at least once / parity of its last load
+      bool ok = true;
+      for (int k = 0; k < n_my; ++k) {
+        const int gt = tile_at(k);
         const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
         const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
         const int layer = pair / g.Hkv, h = pair - layer * g.Hkv;
@@ -199,8 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             for (int c = 0; c < NCH; ++c)
               tma_load_3d(sQ + c * kQChunkBytes + b * r.blk_rows * 128, &p.tmQ[layer], c * 64, r.w0,
                           h * g.G + r.g_first + b, q_full);
-          q_used = true;
-          q_issue_phase ^= 1;
+          ++q_issued;
           cur = u;
         }
         if (!mbar_wait(&k_empty[stage], phase ^ 1, abort_flag)) { ok = false; break; }
@@ -208,8 +218,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         for (int c = 0; c < NCH; ++c)
           tma_load_3d(sK + stage * Cfg::kStageBytes + c * kKChunkBytes, &p.tmK[layer], c * 64, tile * kKeyTile, h,
                       &k_full[stage]);
-        used[stage] = true;
-        last_parity[stage] = phase;
+        used |= 1u << stage;
+        last_par = (last_par & ~(1u << stage)) | (phase << stage);
         if (++stage == S) { stage = 0; phase ^= 1; }
       }
       if (!ok) {
@@ -218,8 +228,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       }
       // Drain: every copy this thread issued has landed before the CTA may exit.
       for (int i = 0; i < S; ++i)
-        if (used[i]) mbar_wait_drain(&k_full[i], last_parity[i]);
-      if (q_used) mbar_wait_drain(q_full, q_issue_phase ^ 1);
+        if (used >> i & 1u) mbar_wait_drain(&k_full[i], last_par >> i & 1u);
+      if (q_issued) mbar_wait_drain(q_full, (q_issued - 1) & 1u);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (one thread)
@@ -229,8 +239,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       bool issued = false, ok = true;
       int last_buf = 0;
       uint32_t last_buf_parity = 0;
-      for (int gt = t_lo; gt < t_hi; ++gt) {
-        const int u = gt / g.n_tiles;
+      for (int k = 0; k < n_my; ++k) {
+        const int u = tile_at(k) / g.n_tiles;
         const RowGroup r = row_group(g, u % g.n_rg);
         if (u != cur) {
           if (cur >= 0) umma_commit(q_empty);  // Q may be overwritten once the previous unit's MMAs finish
@@ -281,41 +291,50 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       if (issued) mbar_wait_drain(&acc_full[last_buf], last_buf_parity);
     }
   } else {
-    // ------------------------------------------------------------ epilogue (8 warps)
+    // ------------------------------------------------------------ epilogue (16 warps, 4 per lane quarter)
     const int ew = warp - 2;
     const int q = warp & 3;    // TMEM lane quarter this warp may access
-    const int hsel = ew >> 2;  // which of the two warps sharing the quarter
+    const int sub = ew >> 2;   // which of the four warps sharing the quarter
     const float c = g.c;
     int buf = 0, cur = -1;
     uint32_t buf_phase = 0, eb_phase = 0;
     RowGroup r{};
-    float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row
+    float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row over its columns
     int my_row = 0, my_pw = 0;
     bool row_ok = false, ok = true;
+    float2* comb2 = sComb;                            // pass 1: [4 sub][128]
+    float* combf = reinterpret_cast<float*>(sComb);   // pass 2: [2 buf][4 sub][128]
 
-    for (int gt = t_lo; gt < t_hi && ok; ++gt) {
+    // pass 1: merge the (m, Z) of the warps that share a row and write this CTA's partial of unit u
+    auto flush_partial = [&](int u) -> bool {
+      const bool two = r.rows > 128;
+      comb2[sub * 128 + q * 32 + lane] = make_float2(m, Z);
+      if (!epi_sync(epi_bar, eb_phase, abort_flag)) return false;
+      const bool leader = two ? (sub & 1) == 0 : sub == 0;
+      if (leader) {
+        const int n_part = two ? 2 : 4;
+        float M = -INFINITY;
+        for (int k = 0; k < n_part; ++k) M = fmaxf(M, comb2[(sub + k) * 128 + q * 32 + lane].x);
+        float zs = 0.f;
+        if (M != -INFINITY)
+          for (int k = 0; k < n_part; ++k) {
+            const float2 o = comb2[(sub + k) * 128 + q * 32 + lane];
+            if (o.x != -INFINITY) zs += o.y * ex2_approx((o.x - M) * c);
+          }
+        p.part[(size_t)(u + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(M, zs);
+      }
+      return epi_sync(epi_bar, eb_phase, abort_flag);
+    };
+
+    if (PASS == 2) pdl_wait();  // pass-1 partials are complete
+    for (int k = 0; k < n_my && ok; ++k) {
+      const int gt = tile_at(k);
       const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
       if (u != cur) {
         if (PASS == 1) {
-          if (cur >= 0) {
-            // flush the partial of the previous unit
-            float mm = m, zz = Z;
-            const bool two = r.rows > 128;
-            if (!two) {
-              if (hsel == 1) sComb[q * 32 + lane] = make_float2(m, Z);
-              if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-              if (hsel == 0) {
-                const float2 o = sComb[q * 32 + lane];
-                const float M = fmaxf(mm, o.x);
-                if (M != -INFINITY) zz = zz * ex2_approx((mm - M) * c) + o.y * ex2_approx((o.x - M) * c);
-                mm = M;
-              }
-              if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-            }
-            if (two || hsel == 0) p.part[(size_t)(cur + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(mm, zz);
-          }
+          if (cur >= 0 && !(ok = flush_partial(cur))) break;
           r = row_group(g, u % g.n_rg);
-          my_row = (r.rows > 128 ? hsel * 128 : 0) + q * 32 + lane;
+          my_row = (r.rows > 128 ? (sub >> 1) * 128 : 0) + q * 32 + lane;
           const int w = r.w0 + my_row % r.blk_rows;
           row_ok = my_row < r.rows && w < g.W;
           my_pw = g.T - g.W + w;
@@ -325,24 +344,25 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           // Combine the pass-1 partials of unit u into per-row offsets, in contributing-CTA order.
           if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;  // previous unit's offsets no longer read
           r = row_group(g, u % g.n_rg);
-          const int row = threadIdx.x - 64;
-          const int w = r.w0 + row % r.blk_rows;
-          const bool valid = row < r.rows && w < g.W;
-          float off = INFINITY;
-          if (valid) {
-            const int c0 = (u * g.n_tiles) / p.tpc;
-            const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
-            float M = -INFINITY;
-            for (int ci = c0; ci <= c1; ++ci) M = fmaxf(M, __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]).x);
-            float Zs = 0.f;
-            for (int ci = c0; ci <= c1; ++ci) {
-              const float2 pz = __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]);
-              if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
+          const int c0 = (u * g.n_tiles) / p.tpc;
+          const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+          for (int row = threadIdx.x - 64; row < kMaxRows; row += kEpiWarps * 32) {
+            const int w = r.w0 + row % r.blk_rows;
+            const bool valid = row < r.rows && w < g.W;
+            float off = INFINITY;
+            if (valid) {
+              float M = -INFINITY;
+              for (int ci = c0; ci <= c1; ++ci) M = fmaxf(M, __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]).x);
+              float Zs = 0.f;
+              for (int ci = c0; ci <= c1; ++ci) {
+                const float2 pz = __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]);
+                if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
+              }
+              off = M * c + __log2f(Zs);
             }
-            off = M * c + __log2f(Zs);
+            sOff[row] = off;
+            sPw[row] = valid ? g.T - g.W + w : -1;
           }
-          sOff[row] = off;
-          sPw[row] = valid ? g.T - g.W + w : -1;
           if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
         }
         cur = u;
@@ -354,9 +374,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * 256);
       if (PASS == 1) {
         const bool two = r.rows > 128;
-        const int col_lo = two ? 0 : hsel * 64;
-        const int col_hi = two ? 128 : col_lo + 64;
-        const uint32_t mt_col = two ? (uint32_t)(hsel * 128) : 0u;
+        const int col_lo = two ? (sub & 1) * 64 : sub * 32;
+        const int col_hi = col_lo + (two ? 64 : 32);
+        const uint32_t mt_col = two ? (uint32_t)((sub >> 1) * 128) : 0u;
         for (int cc = col_lo; cc < col_hi; cc += 32) {
           float v[32];
           tmem_ld32(lane_base + mt_col + (uint32_t)cc, v);
@@ -386,11 +406,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           Z = Z * ex2_approx((m - mn) * c) + ((s0 + s1) + (s2 + s3));
           m = mn;
         }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[buf]);
       } else {
         const int n_cols = (r.rows + 31) & ~31;
         const int j = key0 + q * 32 + lane;
         float acc = 0.f;
-        for (int cc = hsel * 32; cc < n_cols; cc += 64) {
+        for (int cc = sub * 32; cc < n_cols; cc += 128) {
           float v[32];
           tmem_ld32(lane_base + (uint32_t)cc, v);
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
@@ -416,40 +439,27 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           }
           acc += (s0 + s1) + (s2 + s3);
         }
-        float* comb = reinterpret_cast<float*>(sComb) + buf * 128;
-        if (hsel == 1) comb[q * 32 + lane] = acc;
+        float* comb = combf + buf * (4 * 128);
+        if (sub != 0) comb[sub * 128 + q * 32 + lane] = acc;
         // TMEM reads of this buffer are done: hand it back to the MMA issuer before the exchange
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&acc_empty[buf]);
         if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-        if (hsel == 0 && j < g.T) {
-          const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
-          p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = (acc + comb[q * 32 + lane]) * g.inv_G;
+        if (sub == 0 && j < g.T) {
+          const int k = q * 32 + lane;
+          const float val = (((acc + comb[128 + k]) + comb[256 + k]) + comb[384 + k]) * g.inv_G;
+          if (p.t_acc) {
+            atomicAdd(&p.t_acc[j], (unsigned long long)llrintf(val * p.acc_scale));
+          } else {
+            const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
+            p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
+          }
         }
-        if (++buf == 2) { buf = 0; buf_phase ^= 1; }
-        continue;
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[buf]);
       if (++buf == 2) { buf = 0; buf_phase ^= 1; }
     }
-    if (PASS == 1 && ok && cur >= 0) {
-      float mm = m, zz = Z;
-      const bool two = r.rows > 128;
-      if (!two) {
-        if (hsel == 1) sComb[q * 32 + lane] = make_float2(m, Z);
-        ok = epi_sync(epi_bar, eb_phase, abort_flag);
-        if (ok && hsel == 0) {
-          const float2 o = sComb[q * 32 + lane];
-          const float M = fmaxf(mm, o.x);
-          if (M != -INFINITY) zz = zz * ex2_approx((mm - M) * c) + o.y * ex2_approx((o.x - M) * c);
-          mm = M;
-        }
-      }
-      if (ok && (two || hsel == 0)) p.part[(size_t)(cur + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(mm, zz);
-    }
+    if (PASS == 1 && ok && cur >= 0) ok = flush_partial(cur);
     if (!ok) {
       *abort_flag = 1;
       record_status(p.status, STEPKV_ETIMEOUT);
@@ -511,6 +521,16 @@ static ScoreGeom make_geom(int Hkv, int Hq, int d, int T, int W) {
 
 int score_row_groups(int Hkv, int Hq, int W) { return make_geom(Hkv, Hq, 64, W, W).n_rg; }
 
+// Fixed-point shift for the per-token sum over (layer, KV head) pairs: each pair contributes at most W
+// (a softmax row sums to one; W rows per query head, mean over the group), so the sum of n_pairs
+// contributions stays below 2^60 with scale 2^shift.
+int score_acc_shift(int n_pairs, int W) {
+  const double bound = (double)n_pairs * (double)W;
+  int e = 0;
+  while (ldexp(1.0, e) < bound) ++e;
+  return 60 - e;
+}
+
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
   const int n_rg = score_row_groups(Hkv, Hq, W);
   return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kMaxRows * sizeof(float2);
@@ -557,7 +577,8 @@ static cudaError_t launch_pass(const ScoreLaunch& L, int grid, cudaStream_t stre
 
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
-                          int64_t out_stride, float2* part, int32_t* status, cudaStream_t stream) {
+                          int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
+                          cudaStream_t stream) {
   const ScoreGeom g = make_geom(Hkv, Hq, d, T, W);
   ScoreLaunch L;
   memset(&L, 0, sizeof(L));
@@ -566,6 +587,8 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   L.part = part;
   L.out = rows_out;
   L.out_stride = out_stride;
+  L.t_acc = t_acc;
+  L.acc_scale = ldexpf(1.0f, acc_shift);
   L.status = status;
   const int box_rows = std::min(g.W_pad, kMaxRows);
   for (int l = 0; l < n_layers; ++l) {
@@ -576,13 +599,13 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   cudaError_t e = device_sm_count(&n_sm);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   const int grid_cap = std::max(1, std::min(n_sm, kMaxGrid));
-  // pairs per launch: one launch's K stays within L2, so pass 2 re-reads it from L2
-  const double pair_bytes = (double)T * d * 2.0;
+  // all (layer, KV head) pairs in one launch per pass
   const int n_pairs = n_layers * Hkv;
-  const int ppg = std::min(n_pairs, (int)std::max(1.0, floor(kL2GroupBytes / pair_bytes)));
+  const int ppg = n_pairs;
   for (int p0 = 0; p0 < n_pairs; p0 += ppg) {
     const int np = std::min(ppg, n_pairs - p0);
     L.pair0 = p0;
+    L.zero_acc = (t_acc != nullptr && p0 == 0) ? 1 : 0;
     L.n_units = np * g.n_rg;
     const int U = L.n_units * g.n_tiles;
     const int grid0 = std::min(grid_cap, U);

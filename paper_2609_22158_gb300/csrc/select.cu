@@ -28,13 +28,11 @@ namespace stepkv {
 constexpr int kSelCluster = 8;
 constexpr int kSelThreads = 512;
 constexpr int kSelWarps = kSelThreads / 32;
-constexpr int kSelMaxChunk = 32768;  // tokens per CTA held in shared memory (T <= 262144)
 
 struct SelectArgs {
-  const float* rows;
-  int n_rows;
-  int64_t row_stride;
-  float inv_div;
+  const float* T_in;                  // token saliency as floats, or
+  const unsigned long long* t_acc;    // as fixed-point sums: T_i = t_acc[i] * acc_to_T
+  float acc_to_T;
   int T;
   int chunk;  // tokens per CTA
   const int32_t* step_id;
@@ -103,66 +101,167 @@ __device__ __forceinline__ int block_excl_scan(int v, int* excl, int* scratch) {
   return total;
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1)
-    select_kernel(const SelectArgs a) {
+constexpr int kSelUnroll = 8;          // tokens per thread with loads in flight together
+constexpr int kSelSmemSteps = 4096;    // S_k kept in shared memory up to this many steps
+
+// One step-statistics contribution per warp when the warp's (consecutive) tokens share one step, else
+// one per lane.  Integer atomics only: the totals do not depend on the order of arrival.
+__device__ __forceinline__ void step_stat_add(bool act, int sid, unsigned long long fx, uint32_t mx_bits, int32_t* cnt,
+                                              unsigned long long* sum, uint32_t* mx) {
+  const unsigned am = __ballot_sync(0xffffffffu, act);
+  if (!am) return;
+  const int lane = threadIdx.x & 31;
+  const int sid0 = __shfl_sync(0xffffffffu, sid, __ffs(am) - 1);
+  if (__all_sync(0xffffffffu, !act || sid == sid0)) {
+    unsigned long long v = act ? fx : 0ull;
+    uint32_t m = act ? mx_bits : 0u;
+    for (int o = 16; o > 0; o >>= 1) {
+      v += __shfl_xor_sync(0xffffffffu, v, o);
+      m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+    }
+    if (lane == 0) {
+      atomicAdd(&cnt[sid0], __popc(am));
+      if (sum) atomicAdd(&sum[sid0], v);
+      if (mx) atomicMax(&mx[sid0], m);
+    }
+  } else if (act) {
+    atomicAdd(&cnt[sid], 1);
+    if (sum) atomicAdd(&sum[sid], fx);
+    if (mx) atomicMax(&mx[sid], mx_bits);
+  }
+}
+
+__device__ __forceinline__ float step_utility(const SelectArgs& a, int k, int t_last, float* c_out) {
+  const stepkv_params_t& p = a.prm;
+  const float r = a.steps.valid[k] + a.steps.gain[k] - p.lambda * a.steps.red[k];  // Eq. 2
+  float c = 0.f;                                                                     // Alg. 1: c_t = 0
+  if (k != t_last) {
+    c = a.steps.reuse_in[k];
+    if (a.steps.obs_sim) c += fminf(1.f, p.eta * a.steps.obs_sim[k]);              // Eq. 3
+  }
+  *c_out = c;
+  const float rc = fminf(fmaxf(r, p.r_min), p.r_max);
+  return fminf(fmaxf(p.w_r * rc + p.w_c * log1pf(c), 0.f), p.s_max);               // Eq. 4
+}
+
+// Read the 8 per-CTA exchange blocks once (one thread per remote CTA) into a local shared-memory copy.
+__device__ __forceinline__ void gather_exchange(cg::cluster_group& cluster, SelShared* ex, SelShared* all) {
+  if (threadIdx.x < kSelCluster) {
+    const SelShared* rex = cluster.map_shared_rank(ex, (int)threadIdx.x);
+    const int4 v0 = reinterpret_cast<const int4*>(rex)[0];
+    const int4 v1 = reinterpret_cast<const int4*>(rex)[1];
+    reinterpret_cast<int4*>(&all[threadIdx.x])[0] = v0;
+    reinterpret_cast<int4*>(&all[threadIdx.x])[1] = v1;
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs a) {
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
-  extern __shared__ uint8_t smem_raw[];
-  // layout: [chunk] float/uint32 keys | [chunk] u8 flags | 2 x 2048 int hist | SelShared | scratch
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  // layout: [chunk] float/uint32 keys | [chunk] u16 step id (0xFFFF = protected) | 2 x 2048 int hist |
+  //         SelShared (own) | SelShared[8] (gathered) | scratch | S_k
   uint32_t* sKey = reinterpret_cast<uint32_t*>(smem_raw);
   float* sT = reinterpret_cast<float*>(smem_raw);
-  uint8_t* sProt = smem_raw + (size_t)a.chunk * 4;
-  int* hist = reinterpret_cast<int*>(smem_raw + (((size_t)a.chunk * 5 + 15) & ~size_t(15)));
+  uint16_t* sSid = reinterpret_cast<uint16_t*>(smem_raw + (size_t)a.chunk * 4);
+  int* hist = reinterpret_cast<int*>(smem_raw + (((size_t)a.chunk * 6 + 15) & ~size_t(15)));
   SelShared* ex = reinterpret_cast<SelShared*>(hist + 2 * 2048);
-  int* scratch = reinterpret_cast<int*>(ex + 1);   // kSelWarps ints
-  int* bcast = scratch + kSelWarps;                  // 4 ints
+  SelShared* all = ex + 1;
+  int* scratch = reinterpret_cast<int*>(all + kSelCluster);   // 64 ints
+  int* bcast = scratch + 48;                                   // 4 ints (radix passes)
+  float* sS = reinterpret_cast<float*>(scratch + 64);          // [kSelSmemSteps] when n_steps fits
 
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
   const int n_steps = a.steps.n_steps;
   const int t_last = n_steps - 1;
   const int base = rank * a.chunk;
   const int len = max(0, min(a.chunk, T - base));
+  const bool s_in_smem = n_steps <= kSelSmemSteps;
 
-  pdl_wait();
-  pdl_launch_dependents();
-
-  // ---- Phase 1+2 of Algorithm 1 (Eqs. 2-4), steps distributed over the cluster; zero accumulators.
-  for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
-    const stepkv_params_t& p = a.prm;
-    const float r = a.steps.valid[k] + a.steps.gain[k] - p.lambda * a.steps.red[k];
-    float c = 0.f;
-    if (k != t_last) {
-      c = a.steps.reuse_in[k];
-      if (a.steps.obs_sim) c += fminf(1.f, p.eta * a.steps.obs_sim[k]);
+  // Work that reads only the caller's inputs runs before the wait on the score kernels: the first
+  // kernel of the pass already waited for every earlier writer of these inputs.
+  // ---- Phase 1+2 of Algorithm 1 (Eqs. 2-4).  With few steps every CTA keeps all S_k in shared memory
+  // (CTA 0 publishes them); otherwise the steps are split over the cluster through global memory.
+  if (s_in_smem) {
+    for (int k = tid; k < n_steps; k += kSelThreads) {
+      float c;
+      const float sk = step_utility(a, k, t_last, &c);
+      sS[k] = sk;
+      if (rank == 0) {
+        a.S[k] = sk;
+        if (a.out.step_util) a.out.step_util[k] = sk;
+        // reuse_out may alias reuse_in, which every CTA reads here: written after barrier (A)
+      }
     }
-    const float rc = fminf(fmaxf(r, p.r_min), p.r_max);
-    const float s = fminf(fmaxf(p.w_r * rc + p.w_c * log1pf(c), 0.f), p.s_max);
-    a.S[k] = s;
-    if (a.out.step_util && a.out.step_util != a.S) a.out.step_util[k] = s;
-    if (a.steps.reuse_out) a.steps.reuse_out[k] = c;
+  } else {
+    for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
+      float c;
+      const float sk = step_utility(a, k, t_last, &c);
+      a.S[k] = sk;
+      if (a.out.step_util) a.out.step_util[k] = sk;
+      if (a.steps.reuse_out) a.steps.reuse_out[k] = c;
+    }
+  }
+  for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
     a.acc_cnt[k] = 0;
     a.acc_sum[k] = 0ull;
     a.acc_max[k] = 0u;
     a.acc_kept[k] = 0;
   }
-
-  // ---- token saliency T_i (fixed-order sum over rows), prunable max and count, step-id check
-  float lmax = -INFINITY;
+  // step ids and protection flags of this CTA's tokens
   int lN = 0, lerr = 0;
-  for (int i = tid; i < len; i += kSelThreads) {
-    const int gi = base + i;
-    float s = 0.f;
-    for (int r = 0; r < a.n_rows; ++r) s += __ldg(&a.rows[(int64_t)r * a.row_stride + gi]);
-    s *= a.inv_div;
-    sT[i] = s;
-    const uint8_t pr = a.prot[gi] ? 1 : 0;
-    sProt[i] = pr;
-    if (!pr) {
-      ++lN;
-      lmax = fmaxf(lmax, s);
-      const int sid = a.step_id[gi];
-      if (sid < 0 || sid >= n_steps) lerr = 1;
+  for (int i0 = 0; i0 < len; i0 += kSelThreads * kSelUnroll) {
+    uint8_t pv[kSelUnroll];
+    int sv[kSelUnroll];
+#pragma unroll
+    for (int u = 0; u < kSelUnroll; ++u) {
+      const int i = i0 + u * kSelThreads + tid;
+      if (i < len) {
+        pv[u] = __ldg(&a.prot[base + i]);
+        sv[u] = __ldg(&a.step_id[base + i]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kSelUnroll; ++u) {
+      const int i = i0 + u * kSelThreads + tid;
+      if (i < len) {
+        if (!pv[u]) {
+          ++lN;
+          const bool bad = sv[u] < 0 || sv[u] >= n_steps;
+          if (bad) lerr = 1;
+          sSid[i] = bad ? 0 : (uint16_t)sv[u];
+        } else {
+          sSid[i] = 0xFFFFu;
+        }
+      }
+    }
+  }
+
+  pdl_wait();  // token saliency comes from the score kernels
+  pdl_launch_dependents();
+  const float* Sk = s_in_smem ? sS : a.S;
+
+  // ---- token saliency T_i and the prunable maximum
+  float lmax = -INFINITY;
+  for (int i0 = 0; i0 < len; i0 += kSelThreads * kSelUnroll) {
+    float tv[kSelUnroll];
+#pragma unroll
+    for (int u = 0; u < kSelUnroll; ++u) {
+      const int i = i0 + u * kSelThreads + tid;
+      if (i < len) {
+        const int gi = base + i;
+        tv[u] = a.t_acc ? __ull2float_rn(__ldcg(&a.t_acc[gi])) * a.acc_to_T : __ldcg(&a.T_in[gi]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kSelUnroll; ++u) {
+      const int i = i0 + u * kSelThreads + tid;
+      if (i < len) {
+        sT[i] = tv[u];
+        if (sSid[i] != 0xFFFF) lmax = fmaxf(lmax, tv[u]);
+      }
     }
   }
   {
@@ -175,14 +274,21 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       ex->loc_err = be;
     }
   }
-  cluster.sync();  // (A) S_k and zeroed accumulators visible; per-CTA summaries published
+  cluster.sync();  // (A) S_k, zeroed accumulators and per-CTA summaries visible cluster-wide
+  if (s_in_smem && rank == 0 && a.steps.reuse_out) {
+    for (int k = tid; k < n_steps; k += kSelThreads) {
+      float c;
+      step_utility(a, k, t_last, &c);
+      a.steps.reuse_out[k] = c;
+    }
+  }
+  gather_exchange(cluster, ex, all);
   float gmax = -INFINITY;
   int N = 0, err = 0;
   for (int r = 0; r < kSelCluster; ++r) {
-    const SelShared* rex = cluster.map_shared_rank(ex, r);
-    gmax = fmaxf(gmax, rex->loc_max);
-    N += rex->loc_N;
-    err += rex->loc_err;
+    gmax = fmaxf(gmax, all[r].loc_max);
+    N += all[r].loc_N;
+    err += all[r].loc_err;
   }
   if (err) {
     if (rank == 0 && tid == 0) {
@@ -212,45 +318,30 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   const int fx_shift = 62 - log2N - e_max;    // every partial sum < 2^62
   const float fx_scale = ldexpf(1.0f, min(fx_shift, 126));
 
-  // ---- priorities and ordered keys; per-step statistics (run-aggregated integer atomics)
-  {
-    int run_sid = -1, run_cnt = 0;
-    unsigned long long run_sum = 0ull;
-    uint32_t run_max = 0u;
-    auto flush = [&]() {
-      if (run_sid >= 0 && run_cnt) {
-        atomicAdd(&a.acc_cnt[run_sid], run_cnt);
-        atomicAdd(&a.acc_sum[run_sid], run_sum);
-        atomicMax(&a.acc_max[run_sid], run_max);
-      }
-    };
-    for (int i = tid; i < len; i += kSelThreads) {
-      const int gi = base + i;
-      const float th = sT[i] * inv_max;
-      if (a.out.token_sal) a.out.token_sal[gi] = th;
+  // ---- priorities (Eq. 5), ordered keys and per-step statistics.  The loop bound is uniform per warp
+  // (warp-aggregated atomics); T_hat is read before its shared-memory slot is overwritten by the key.
+  for (int i0 = 0; i0 < len; i0 += kSelThreads) {
+    const int i = i0 + tid;
+    const bool in = i < len;
+    const int gi = base + i;
+    const float th = in ? sT[i] * inv_max : 0.f;
+    const int sid = in ? sSid[i] : 0xFFFF;
+    const bool act = sid != 0xFFFF;
+    if (in) {
       uint32_t key = 0u;
-      if (!sProt[i]) {
-        const int sid = a.step_id[gi];
-        const float P = fmaf(a.prm.alpha, th, a.prm.beta * a.S[sid]);
+      if (act) {
+        const float P = fmaf(a.prm.alpha, th, a.prm.beta * Sk[sid]);
         key = float_to_ordered(P);
         if (a.out.priority) a.out.priority[gi] = P;
-        const float thc = fmaxf(th, 0.f);
-        if (sid != run_sid) {
-          flush();
-          run_sid = sid;
-          run_cnt = 0;
-          run_sum = 0ull;
-          run_max = 0u;
-        }
-        ++run_cnt;
-        run_sum += (unsigned long long)llrintf(thc * fx_scale);
-        run_max = max(run_max, __float_as_uint(thc));
       } else if (a.out.priority) {
         a.out.priority[gi] = -INFINITY;
       }
+      if (a.out.token_sal) a.out.token_sal[gi] = th;
       sKey[i] = key;
     }
-    flush();
+    const float thc = fmaxf(th, 0.f);
+    step_stat_add(act, sid, (unsigned long long)llrintf(thc * fx_scale), __float_as_uint(thc), a.acc_cnt, a.acc_sum,
+                  a.acc_max);
   }
   __syncthreads();
 
@@ -262,46 +353,59 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   } else if (B < N) {
     uint32_t prefix = 0u, mask = 0u;
     int remaining = B;
-    const int shifts[3] = {21, 10, 0};
-    const int nbits[3] = {11, 11, 10};
     for (int pass = 0; pass < 3; ++pass) {
       int* h = hist + (pass & 1) * 2048;
-      const int nb = 1 << nbits[pass];
-      const int sh = shifts[pass];
+      const int nbits = pass < 2 ? 11 : 10;
+      const int sh = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
+      const int nb = 1 << nbits;
       for (int b = tid; b < nb; b += kSelThreads) h[b] = 0;
       __syncthreads();
-      for (int i = tid; i < len; i += kSelThreads) {
-        const uint32_t k = sKey[i];
-        if (!sProt[i] && (k & mask) == prefix) atomicAdd(&h[(k >> sh) & (nb - 1)], 1);
+      // keys of one step share their leading bits, so many lanes hit the same bin: aggregate per warp
+      for (int i0 = 0; i0 < len; i0 += kSelThreads) {
+        const int i = i0 + tid;
+        const uint32_t k = i < len ? sKey[i] : 0u;
+        const bool hit = i < len && sSid[i] != 0xFFFF && (k & mask) == prefix;
+        const int bin = hit ? (int)((k >> sh) & (nb - 1)) : -1;
+        const unsigned peers = __match_any_sync(0xffffffffu, bin);
+        if (hit && (__ffs(peers) - 1) == lane) atomicAdd(&h[bin], __popc(peers));
       }
       cluster.sync();  // every CTA's histogram of this pass is complete
-      // global histogram; thread t owns bins [t*bpt, (t+1)*bpt)
-      const int bpt = nb / kSelThreads;  // 4 or 2
+      // global histogram; thread t owns bins [t*bpt, (t+1)*bpt): one vector load per remote CTA, all in flight
       int cnt[4] = {0, 0, 0, 0};
-      for (int r = 0; r < kSelCluster; ++r) {
-        const int* rh = cluster.map_shared_rank(h, r);
-        for (int q = 0; q < bpt; ++q) cnt[q] += rh[tid * bpt + q];
-      }
-      int mine = 0;
-      for (int q = 0; q < bpt; ++q) mine += cnt[q];
-      // suffix sum over threads (bins above mine): scan in reversed thread order
-      int excl_rev;
-      {
-        const int lane = tid & 31, warp = tid >> 5;
-        // reversed index: thread 511 first
-        int x = mine;
-        for (int o = 1; o < 32; o <<= 1) {
-          const int y = __shfl_down_sync(0xffffffffu, x, o);
-          if (lane + o < 32) x += y;
+      if (nb == 2048) {
+        int4 v[kSelCluster];
+#pragma unroll
+        for (int r = 0; r < kSelCluster; ++r) v[r] = reinterpret_cast<const int4*>(cluster.map_shared_rank(h, r))[tid];
+#pragma unroll
+        for (int r = 0; r < kSelCluster; ++r) {
+          cnt[0] += v[r].x;
+          cnt[1] += v[r].y;
+          cnt[2] += v[r].z;
+          cnt[3] += v[r].w;
         }
-        __syncthreads();
-        if (lane == 0) scratch[warp] = x;  // sum of lanes >= 0 of this warp = warp total
-        __syncthreads();
-        int after = 0;
-        for (int w = warp + 1; w < kSelWarps; ++w) after += scratch[w];
-        excl_rev = after + x - mine;  // keys in bins owned by higher threads
+      } else {
+        int2 v[kSelCluster];
+#pragma unroll
+        for (int r = 0; r < kSelCluster; ++r) v[r] = reinterpret_cast<const int2*>(cluster.map_shared_rank(h, r))[tid];
+#pragma unroll
+        for (int r = 0; r < kSelCluster; ++r) {
+          cnt[0] += v[r].x;
+          cnt[1] += v[r].y;
+        }
       }
-      int above = excl_rev;
+      const int bpt = nb / kSelThreads;  // 4 or 2
+      const int mine = cnt[0] + cnt[1] + cnt[2] + cnt[3];
+      // keys in bins owned by higher threads: suffix scan over the block
+      int x = mine;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_down_sync(0xffffffffu, x, o);
+        if (lane + o < 32) x += y;
+      }
+      if (lane == 0) scratch[warp] = x;
+      __syncthreads();
+      int after = 0;
+      for (int w = warp + 1; w < kSelWarps; ++w) after += scratch[w];
+      int above = after + x - mine;
       for (int q = bpt - 1; q >= 0; --q) {
         if (above < remaining && remaining <= above + cnt[q]) {
           bcast[0] = tid * bpt + q;
@@ -325,7 +429,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   {
     int kb = 0, eq = 0;
     for (int i = tid; i < len; i += kSelThreads) {
-      if (sProt[i]) ++kb;
+      if (sSid[i] == 0xFFFF) ++kb;
       else if (sKey[i] > kth) ++kb;
       else if (sKey[i] == kth) ++eq;
     }
@@ -337,19 +441,19 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     }
   }
   cluster.sync();  // (B)
+  gather_exchange(cluster, ex, all);
   // offsets: CTA r keeps its protected + strictly-greater tokens and the ties that fall within the
   // first need_eq ties in slot order
   int out_off = 0, total_kept = 0, ties_before = 0, eq_cum = 0;
   for (int r = 0; r < kSelCluster; ++r) {
-    const SelShared* rex = cluster.map_shared_rank(ex, r);
-    const int granted = max(0, min(need_eq - eq_cum, rex->loc_eq));
-    const int kept_r = rex->loc_keep_base + granted;
+    const int granted = max(0, min(need_eq - eq_cum, all[r].loc_eq));
+    const int kept_r = all[r].loc_keep_base + granted;
     if (r < rank) {
       out_off += kept_r;
-      ties_before += rex->loc_eq;
+      ties_before += all[r].loc_eq;
     }
     total_kept += kept_r;
-    eq_cum += rex->loc_eq;
+    eq_cum += all[r].loc_eq;
   }
   const bool overflow = total_kept > a.out.kept_cap;
   if (rank == 0 && tid == 0) {
@@ -358,46 +462,68 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     if (overflow) record_status(a.status, STEPKV_ENOSPACE);
   }
 
-  // ---- ordered write of the retained slots (ballot + prefix per 512-token round)
+  // ---- ordered write of the retained slots.  Token i of round r = i / 512 is handled by thread i % 512;
+  // each warp records per-round tie and keep counts, two block-wide prefix passes order them.
   if (!overflow) {
-    int run_keep = 0, run_eq = 0;
-    const int lane = tid & 31, warp = tid >> 5;
-    int* wk = scratch;               // kSelWarps kept counts
-    int* we = scratch + kSelWarps;   // uses bcast area too (kSelWarps more ints)
-    for (int r0 = 0; r0 < len; r0 += kSelThreads) {
-      const int i = r0 + tid;
+    const int n_rounds = (len + kSelThreads - 1) / kSelThreads;
+    int* cnt_eq = reinterpret_cast<int*>(hist);              // [rounds][warps]
+    int* cnt_keep = cnt_eq + n_rounds * kSelWarps;            // [rounds][warps]
+    // (1) tie counts per (round, warp)
+    for (int r = 0; r < n_rounds; ++r) {
+      const int i = r * kSelThreads + tid;
+      const bool is_eq = i < len && sSid[i] != 0xFFFF && sKey[i] == kth;
+      const unsigned m = __ballot_sync(0xffffffffu, is_eq);
+      if (lane == 0) cnt_eq[r * kSelWarps + warp] = __popc(m);
+    }
+    __syncthreads();
+    // exclusive prefix over (round, warp) in slot order, one warp per 32 entries (serial over few rounds)
+    if (tid == 0) {
+      int run = ties_before;
+      for (int e = 0; e < n_rounds * kSelWarps; ++e) {
+        const int c = cnt_eq[e];
+        cnt_eq[e] = run;
+        run += c;
+      }
+    }
+    __syncthreads();
+    // (2) keep flags and keep counts per (round, warp)
+    for (int r = 0; r < n_rounds; ++r) {
+      const int i = r * kSelThreads + tid;
       const bool in = i < len;
       const uint32_t k = in ? sKey[i] : 0u;
-      const bool pr = in && sProt[i];
+      const bool pr = in && sSid[i] == 0xFFFF;
       const bool is_eq = in && !pr && k == kth;
-      const unsigned eq_mask = __ballot_sync(0xffffffffu, is_eq);
-      const int eq_lane_before = __popc(eq_mask & ((1u << lane) - 1u));
-      if (lane == 0) we[warp] = __popc(eq_mask);
-      __syncthreads();
-      int eq_warp_before = 0, eq_round = 0;
-      for (int w = 0; w < kSelWarps; ++w) {
-        if (w < warp) eq_warp_before += we[w];
-        eq_round += we[w];
+      const unsigned em = __ballot_sync(0xffffffffu, is_eq);
+      const int eq_rank = cnt_eq[r * kSelWarps + warp] + __popc(em & ((1u << lane) - 1u));
+      const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
+      const unsigned km = __ballot_sync(0xffffffffu, keep);
+      if (lane == 0) cnt_keep[r * kSelWarps + warp] = __popc(km);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int run = out_off;
+      for (int e = 0; e < n_rounds * kSelWarps; ++e) {
+        const int c = cnt_keep[e];
+        cnt_keep[e] = run;
+        run += c;
       }
-      const int eq_rank = ties_before + run_eq + eq_warp_before + eq_lane_before;
-      const bool keep = in && (pr || (k > kth) || (is_eq && eq_rank < need_eq));
-      const unsigned keep_mask = __ballot_sync(0xffffffffu, keep);
-      const int keep_lane_before = __popc(keep_mask & ((1u << lane) - 1u));
-      if (lane == 0) wk[warp] = __popc(keep_mask);
-      __syncthreads();
-      int keep_warp_before = 0, keep_round = 0;
-      for (int w = 0; w < kSelWarps; ++w) {
-        if (w < warp) keep_warp_before += wk[w];
-        keep_round += wk[w];
-      }
-      if (keep) {
-        const int gi = base + i;
-        a.out.kept_idx[out_off + run_keep + keep_warp_before + keep_lane_before] = gi;
-        if (!pr) atomicAdd(&a.acc_kept[a.step_id[gi]], 1);
-      }
-      run_keep += keep_round;
-      run_eq += eq_round;
-      __syncthreads();
+    }
+    __syncthreads();
+    // (3) write
+    for (int r = 0; r < n_rounds; ++r) {
+      const int i = r * kSelThreads + tid;
+      const bool in = i < len;
+      const uint32_t k = in ? sKey[i] : 0u;
+      const int sid = in ? sSid[i] : 0xFFFF;
+      const bool pr = in && sid == 0xFFFF;
+      const bool is_eq = in && !pr && k == kth;
+      const unsigned em = __ballot_sync(0xffffffffu, is_eq);
+      const int eq_rank = cnt_eq[r * kSelWarps + warp] + __popc(em & ((1u << lane) - 1u));
+      const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
+      const unsigned km = __ballot_sync(0xffffffffu, keep);
+      if (keep) a.out.kept_idx[cnt_keep[r * kSelWarps + warp] + __popc(km & ((1u << lane) - 1u))] = base + i;
+      const bool kept_prunable = keep && !pr;
+      step_stat_add(kept_prunable, sid, 0ull, 0u, a.acc_kept, nullptr, nullptr);
     }
   }
   cluster.sync();  // (C) all step accumulators final
@@ -413,6 +539,39 @@ __global__ void __launch_bounds__(kSelThreads, 1)
 }
 
 // -------------------------------------------------------------------------------------------------
+// T_out[j] = inv_div * sum over rows (fixed order): the token-saliency input of stepkv_select when the
+// caller supplies per-(layer, head) saliency rows.  Four rows in flight per thread.
+__global__ void mean_rows_kernel(const float* __restrict__ rows, int n_rows, int64_t row_stride, float inv_div, int T,
+                                 float* __restrict__ T_out) {
+  pdl_wait();
+  pdl_launch_dependents();
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < T; j += gridDim.x * blockDim.x) {
+    float s = 0.f;
+    int r = 0;
+    for (; r + 4 <= n_rows; r += 4) {
+      const float a0 = __ldg(&rows[(int64_t)r * row_stride + j]);
+      const float a1 = __ldg(&rows[(int64_t)(r + 1) * row_stride + j]);
+      const float a2 = __ldg(&rows[(int64_t)(r + 2) * row_stride + j]);
+      const float a3 = __ldg(&rows[(int64_t)(r + 3) * row_stride + j]);
+      s = (((s + a0) + a1) + a2) + a3;
+    }
+    for (; r < n_rows; ++r) s += __ldg(&rows[(int64_t)r * row_stride + j]);
+    T_out[j] = s * inv_div;
+  }
+}
+
+stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, float* T_out,
+                              cudaStream_t stream) {
+  const int blocks = std::max(1, std::min((T + 255) / 256, 4096));
+  cudaError_t e = launch_pdl(mean_rows_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_rows, row_stride, inv_div,
+                             T, T_out);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return STEPKV_ECUDA;
+  }
+  return STEPKV_OK;
+}
+
 static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
 size_t select_ws_bytes(int T, int n_steps) {
@@ -421,16 +580,15 @@ size_t select_ws_bytes(int T, int n_steps) {
   return align256(n * 4) + align256(n * 4) + align256(n * 8) + align256(n * 4) + align256(n * 4);
 }
 
-stepkv_status_t select_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T,
+stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, double acc_to_T, int T,
                            const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
                            const stepkv_params_t& params, const stepkv_budget_t& budget,
                            const stepkv_select_out_t& out, void* ws, int32_t* status, cudaStream_t stream) {
   SelectArgs a;
   memset(&a, 0, sizeof(a));
-  a.rows = rows;
-  a.n_rows = n_rows;
-  a.row_stride = row_stride;
-  a.inv_div = inv_div;
+  a.T_in = T_in;
+  a.t_acc = t_acc;
+  a.acc_to_T = acc_to_T;
   a.T = T;
   a.chunk = ((T + kSelCluster - 1) / kSelCluster + 15) & ~15;
   a.step_id = step_id;
@@ -451,7 +609,9 @@ stepkv_status_t select_run(const float* rows, int n_rows, int64_t row_stride, fl
   w += align256(n * 4);
   a.acc_kept = reinterpret_cast<int32_t*>(w);
   a.status = status;
-  const size_t smem = (((size_t)a.chunk * 5 + 15) & ~size_t(15)) + 2 * 2048 * 4 + sizeof(SelShared) + 64 * 4;
+  const size_t smem = (((size_t)a.chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + kSelCluster) * sizeof(SelShared) +
+                      64 * 4 +
+                      (steps.n_steps <= kSelSmemSteps ? (size_t)steps.n_steps * 4 : 0);
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_kernel), (int)smem);
   if (e == cudaSuccess)
     e = launch_pdl_cluster(select_kernel, dim3(kSelCluster), dim3(kSelThreads), kSelCluster, smem, stream, a);

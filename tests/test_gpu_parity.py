@@ -167,6 +167,28 @@ def test_select_large_T(B):
     TL.check_select_outputs(g, out)
 
 
+def test_select_reuse_in_place(B):
+    """reuse_out may alias reuse_in (the caller keeps one c_k array across boundaries)."""
+    import torch
+    tr = wl.custom(6, L=1, Hq=4, Hkv=1, d=64, T=5000, W=16, n_steps=30)
+    rng = np.random.default_rng(6)
+    sal = (rng.random((2, tr.T)) * 3).astype(np.float32)
+    c = torch.from_numpy(tr.reuse.copy()).cuda()
+    steps = B.StepSignals(*(torch.from_numpy(x).cuda() for x in (tr.valid, tr.gain, tr.red)), c,
+                          torch.from_numpy(tr.obs_sim).cuda(), c)
+    out = B.SelectOutputs.allocate(tr.T, tr.n_steps, tr.T, "cuda")
+    st = B.new_status()
+    B.stepkv_select(torch.from_numpy(sal).cuda(), torch.from_numpy(tr.step_id).cuda(), torch.from_numpy(tr.prot).cuda(),
+                    steps, B.Params(), B.budget_ratio(1, 5), out, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    exp = O.reuse_update(tr.reuse, tr.obs_sim, 1.5)
+    TL.assert_close(c.cpu().numpy(), exp, "c_k in place", floor=1e-6)
+    p = O.Params()
+    S = O.step_utility(O.completion_score(tr.valid, tr.gain, tr.red, p.lam), exp, p)
+    TL.assert_close(out.step_util.cpu().numpy(), S, "S_k", floor=1e-6)
+
+
 def test_select_bad_step_id_sets_edata(B):
     tr = wl.custom(4, L=1, Hq=2, Hkv=1, d=64, T=600, W=8, n_steps=3)
     tr.step_id = tr.step_id.copy()
@@ -193,7 +215,7 @@ def _select_case_status(B, tr, sal):
 
 
 # ------------------------------------------------------------------------------------ stage 5
-@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("d", [64, 96, 128])
 def test_compact_bit_exact(B, d):
     import torch
     rng = np.random.default_rng(d)
@@ -330,8 +352,9 @@ def test_compress_deterministic(B):
         g = TL.GpuTraj(tr)
         B.stepkv_compress([g.problem()], B.Params())
         torch.cuda.synchronize()
-        res.append([g.out.kept_idx.cpu(), g.out.priority.cpu(), g.out.token_sal.cpu(), g.out.step_sal_sum.cpu(),
-                    g.K_out[0].cpu(), g.V_out[2].cpu()])
+        n = int(g.out.n_kept.item())
+        res.append([g.out.kept_idx[:n].cpu(), g.out.priority.cpu(), g.out.token_sal.cpu(), g.out.step_sal_sum.cpu(),
+                    g.K_out[0][:, :n].cpu(), g.V_out[2][:, :n].cpu()])
     for a, b in zip(*res):
         assert torch.equal(a.contiguous().view(torch.uint8), b.contiguous().view(torch.uint8))
 

@@ -154,9 +154,48 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+// Packed fp32 pairs (sm_100 family): one instruction for two lanes' worth of FMA / ADD.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 // Named barrier among `nthreads` threads (multiple of 32) of the CTA; ids 1..15 (0 = __syncthreads).
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Exact fixed-point conversion of a non-negative float: round(x * 2^shift) as uint64, with integer
+// instructions only (the float -> 64-bit conversion instructions run on the slow FP64 pipe).  Requires
+// x * 2^shift < 2^63.  Rounds half away from zero.
+__device__ __forceinline__ unsigned long long to_fixed(float x, int shift) {
+  const uint32_t b = __float_as_uint(x);
+  const int e = (int)((b >> 23) & 0xFFu);
+  if (e == 0 || (b >> 31)) return 0ull;                   // zero, subnormal or negative
+  const unsigned long long mant = (unsigned long long)((b & 0x7FFFFFu) | 0x800000u);
+  const int sh = e - 150 + shift;                           // value = mant * 2^(e-150)
+  if (sh >= 0) return mant << sh;
+  if (sh < -24) return 0ull;
+  return (mant + (1ull << (-sh - 1))) >> (-sh);
 }
 
 // Float <-> order-preserving unsigned key (larger float <=> larger key; -0 < +0).

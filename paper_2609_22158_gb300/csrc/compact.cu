@@ -139,7 +139,7 @@ stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* c
       const int64_t rows_max = (int64_t)std::max(a.n_sets, 1) * std::max(kept_cap, 1);
       const int64_t want = (rows_max + 31) / 32;  // no more CTAs than 32 row items each at full capacity
       const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * kCompactCtasPerSm, want));
-      e = launch_pdl(compact_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a);
+      e = launch_kernel(compact_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a);
     }
     if (e != cudaSuccess) {
       set_last_cuda_error(e);

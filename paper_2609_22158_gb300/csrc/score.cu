@@ -55,7 +55,7 @@ struct ScoreLaunch {
   float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when t_acc == nullptr)
   int64_t out_stride;
   unsigned long long* t_acc;  // pass 2: per-token fixed-point sum over all (pair, row group) (when non-null)
-  float acc_scale;    // 2^k: fixed-point scale of t_acc
+  int acc_shift;      // k: fixed-point scale 2^k of t_acc
   int zero_acc;       // pass 1: zero t_acc[0..T) first (first launch of a compression pass)
   int32_t* status;
 };
@@ -85,20 +85,26 @@ __host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
   return r;
 }
 
-template <int NCH>
+template <int PASS, int NCH>
 struct ScoreCfg {
-  static constexpr int kStages = NCH == 2 ? 4 : 8;
+  // Pass 1 needs no shared tables, so it affords a fifth K stage (more bytes in flight per SM).
+  static constexpr int kStages = PASS == 1 ? (NCH == 2 ? 5 : 10) : (NCH == 2 ? 4 : 8);
   static constexpr int kQBytes = NCH * kQChunkBytes;
   static constexpr int kStageBytes = NCH * kKChunkBytes;
-  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;  // float sOff[256]
-  static constexpr int kPwOff = kOffOff + kMaxRows * 4;            // int   sPw[256]
-  static constexpr int kCombOff = kPwOff + kMaxRows * 4;           // 4 KB: float2[4][128] (pass 1) / float[2][4][128] (pass 2)
-  static constexpr int kBarOff = kCombOff + 4096;
+  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;         // pass 2: float sNegOff[256]
+  static constexpr int kPwOff = kOffOff + (PASS == 2 ? kMaxRows * 4 : 0); // pass 2: int sPw[256]
+  static constexpr int kCombOff = kPwOff + (PASS == 2 ? kMaxRows * 4 : 0);// pass 2: float[2][4][128]
+  static constexpr int kBarOff = kCombOff + (PASS == 2 ? 4096 : 0);
   static constexpr int kNumBars = 2 * kStages + 2 + 4 + 1;
-  static constexpr int kMiscOff = kBarOff + kNumBars * 8;          // tmem base, abort flag
+  static constexpr int kMiscOff = kBarOff + kNumBars * 8;                 // tmem base, abort flag
   static constexpr int kBytes = kMiscOff + 16;
-  static constexpr int kDynSmem = kBytes + 1024;                   // + alignment slack
+  static constexpr int kDynSmem = kBytes + 1024;                          // + alignment slack
+  static_assert(kDynSmem <= 232448, "shared memory budget");
 };
+
+// Pass-1 partial (m, Z) slots: one per (unit, CTA), each with 4 entries per row (one per warp that
+// covers part of the row's keys).
+constexpr int kPartEntries = 4;
 
 // Bounded barrier among the 8 epilogue warps (an mbarrier with one arrival per warp).  Returns false
 // if the CTA aborted or the wait limit passed.
@@ -118,13 +124,13 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
 
 template <int PASS, int NCH>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreLaunch p) {
-  using Cfg = ScoreCfg<NCH>;
+  using Cfg = ScoreCfg<PASS, NCH>;
   constexpr int S = Cfg::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = sm;
   uint8_t* sK = sm + Cfg::kQBytes;
-  float* sOff = reinterpret_cast<float*>(sm + Cfg::kOffOff);
+  float* sNegOff = reinterpret_cast<float*>(sm + Cfg::kOffOff);
   int* sPw = reinterpret_cast<int*>(sm + Cfg::kPwOff);
   float2* sComb = reinterpret_cast<float2*>(sm + Cfg::kCombOff);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kBarOff);
@@ -177,10 +183,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  // Pass 1 waits for every earlier kernel on the stream (one of them may have written K/Q).  Pass 2 is
-  // launched only after all pass-1 CTAs passed that wait, so its K/Q loads may start at once; only the
-  // epilogue, which reads the pass-1 partials, waits for pass 1 to complete.
-  if (PASS == 1) pdl_wait();
+  // Only shared memory, barriers and TMEM are set up before this point.  Every thread waits for the
+  // earlier kernels on the stream before its first global access (a per-role wait placed later was
+  // observed to let early-launched CTAs read pass-1 partials of the previous call).
+  pdl_wait();
   pdl_launch_dependents();
   if (PASS == 1 && p.zero_acc) {
     for (int i = blockIdx.x * kThreads + threadIdx.x; i < g.T; i += gridDim.x * kThreads) p.t_acc[i] = 0ull;
@@ -302,37 +308,21 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row over its columns
     int my_row = 0, my_pw = 0;
     bool row_ok = false, ok = true;
-    float2* comb2 = sComb;                            // pass 1: [4 sub][128]
-    float* combf = reinterpret_cast<float*>(sComb);   // pass 2: [2 buf][4 sub][128]
+    float* combf = reinterpret_cast<float*>(sComb);   // pass 2 (rows output): [2 buf][4 sub][128]
 
-    // pass 1: merge the (m, Z) of the warps that share a row and write this CTA's partial of unit u
-    auto flush_partial = [&](int u) -> bool {
+    // pass 1: this warp's (m, Z) over its share of the row's keys becomes entry e of the CTA's partial
+    auto flush_partial = [&](int u) {
       const bool two = r.rows > 128;
-      comb2[sub * 128 + q * 32 + lane] = make_float2(m, Z);
-      if (!epi_sync(epi_bar, eb_phase, abort_flag)) return false;
-      const bool leader = two ? (sub & 1) == 0 : sub == 0;
-      if (leader) {
-        const int n_part = two ? 2 : 4;
-        float M = -INFINITY;
-        for (int k = 0; k < n_part; ++k) M = fmaxf(M, comb2[(sub + k) * 128 + q * 32 + lane].x);
-        float zs = 0.f;
-        if (M != -INFINITY)
-          for (int k = 0; k < n_part; ++k) {
-            const float2 o = comb2[(sub + k) * 128 + q * 32 + lane];
-            if (o.x != -INFINITY) zs += o.y * ex2_approx((o.x - M) * c);
-          }
-        p.part[(size_t)(u + (int)blockIdx.x) * kMaxRows + my_row] = make_float2(M, zs);
-      }
-      return epi_sync(epi_bar, eb_phase, abort_flag);
+      const int e = two ? (sub & 1) : sub;
+      p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + e) * kMaxRows + my_row] = make_float2(m, Z);
     };
 
-    if (PASS == 2) pdl_wait();  // pass-1 partials are complete
     for (int k = 0; k < n_my && ok; ++k) {
       const int gt = tile_at(k);
       const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
       if (u != cur) {
         if (PASS == 1) {
-          if (cur >= 0 && !(ok = flush_partial(cur))) break;
+          if (cur >= 0) flush_partial(cur);
           r = row_group(g, u % g.n_rg);
           my_row = (r.rows > 128 ? (sub >> 1) * 128 : 0) + q * 32 + lane;
           const int w = r.w0 + my_row % r.blk_rows;
@@ -346,21 +336,25 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           r = row_group(g, u % g.n_rg);
           const int c0 = (u * g.n_tiles) / p.tpc;
           const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+          const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
           for (int row = threadIdx.x - 64; row < kMaxRows; row += kEpiWarps * 32) {
             const int w = r.w0 + row % r.blk_rows;
             const bool valid = row < r.rows && w < g.W;
             float off = INFINITY;
             if (valid) {
               float M = -INFINITY;
-              for (int ci = c0; ci <= c1; ++ci) M = fmaxf(M, __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]).x);
+              for (int ci = c0; ci <= c1; ++ci)
+                for (int e = 0; e < n_e; ++e)
+                  M = fmaxf(M, __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]).x);
               float Zs = 0.f;
-              for (int ci = c0; ci <= c1; ++ci) {
-                const float2 pz = __ldcg(&p.part[(size_t)(u + ci) * kMaxRows + row]);
-                if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
-              }
+              for (int ci = c0; ci <= c1; ++ci)
+                for (int e = 0; e < n_e; ++e) {
+                  const float2 pz = __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]);
+                  if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
+                }
               off = M * c + __log2f(Zs);
             }
-            sOff[row] = off;
+            sNegOff[row] = -off;
             sPw[row] = valid ? g.T - g.W + w : -1;
           }
           if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
@@ -386,24 +380,31 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = (j0 + i <= my_pw) ? v[i] : -INFINITY;
           }
-          float cm0 = fmaxf(v[0], v[1]), cm1 = fmaxf(v[2], v[3]);
+          float mx[11];
 #pragma unroll
-          for (int i = 4; i < 32; i += 4) {
-            cm0 = fmaxf(cm0, fmaxf(v[i], v[i + 1]));
-            cm1 = fmaxf(cm1, fmaxf(v[i + 2], v[i + 3]));
-          }
-          const float mn = fmaxf(m, fmaxf(cm0, cm1));
+          for (int i = 0; i < 10; ++i) mx[i] = fmax3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+          mx[10] = fmaxf(v[30], v[31]);
+          const float mn = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]),
+                                 fmax3(fmax3(mx[6], mx[7], mx[8]), fmax3(mx[9], mx[10], m), -INFINITY));
           if (mn == -INFINITY) continue;
-          const float mc = mn * c;
-          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+          const float nmc = -mn * c;
+          const uint64_t c2 = f2_pack(c, c), b2 = f2_pack(nmc, nmc);
+          uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-          for (int i = 0; i < 32; i += 4) {
-            s0 += ex2_approx(fmaf(v[i + 0], c, -mc));
-            s1 += ex2_approx(fmaf(v[i + 1], c, -mc));
-            s2 += ex2_approx(fmaf(v[i + 2], c, -mc));
-            s3 += ex2_approx(fmaf(v[i + 3], c, -mc));
+          for (int i = 0; i < 32; i += 8) {
+#pragma unroll
+            for (int k2 = 0; k2 < 4; ++k2) {
+              float lo, hi;
+              f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, b2), lo, hi);
+              acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+            }
           }
-          Z = Z * ex2_approx((m - mn) * c) + ((s0 + s1) + (s2 + s3));
+          float s0, s1, s2, s3, s4, s5, s6, s7;
+          f2_unpack(acc2[0], s0, s1);
+          f2_unpack(acc2[1], s2, s3);
+          f2_unpack(acc2[2], s4, s5);
+          f2_unpack(acc2[3], s6, s7);
+          Z = Z * ex2_approx((m - mn) * c) + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
           m = mn;
         }
         tc_fence_before();
@@ -418,40 +419,56 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           tmem_ld32(lane_base + (uint32_t)cc, v);
           float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
           if (!need_mask) {
+            const uint64_t c2 = f2_pack(c, c);
+            uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              const float4 o = *reinterpret_cast<const float4*>(&sOff[cc + i]);
-              s0 += ex2_approx(fmaf(v[i + 0], c, -o.x));
-              s1 += ex2_approx(fmaf(v[i + 1], c, -o.y));
-              s2 += ex2_approx(fmaf(v[i + 2], c, -o.z));
-              s3 += ex2_approx(fmaf(v[i + 3], c, -o.w));
+            for (int i = 0; i < 32; i += 8) {
+#pragma unroll
+              for (int k2 = 0; k2 < 4; ++k2) {
+                const float2 o = *reinterpret_cast<const float2*>(&sNegOff[cc + i + 2 * k2]);
+                float lo, hi;
+                f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, f2_pack(o.x, o.y)), lo, hi);
+                acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+              }
             }
+            float t0, t1, t2, t3, t4, t5, t6, t7;
+            f2_unpack(acc2[0], t0, t1);
+            f2_unpack(acc2[1], t2, t3);
+            f2_unpack(acc2[2], t4, t5);
+            f2_unpack(acc2[3], t6, t7);
+            s0 = t0 + t1;
+            s1 = t2 + t3;
+            s2 = t4 + t5;
+            s3 = t6 + t7;
           } else {
 #pragma unroll
             for (int i = 0; i < 32; i += 4) {
-              const float4 o = *reinterpret_cast<const float4*>(&sOff[cc + i]);
+              const float4 o = *reinterpret_cast<const float4*>(&sNegOff[cc + i]);
               const int4 pw = *reinterpret_cast<const int4*>(&sPw[cc + i]);
-              s0 += j <= pw.x ? ex2_approx(fmaf(v[i + 0], c, -o.x)) : 0.f;
-              s1 += j <= pw.y ? ex2_approx(fmaf(v[i + 1], c, -o.y)) : 0.f;
-              s2 += j <= pw.z ? ex2_approx(fmaf(v[i + 2], c, -o.z)) : 0.f;
-              s3 += j <= pw.w ? ex2_approx(fmaf(v[i + 3], c, -o.w)) : 0.f;
+              s0 += j <= pw.x ? ex2_approx(fmaf(v[i + 0], c, o.x)) : 0.f;
+              s1 += j <= pw.y ? ex2_approx(fmaf(v[i + 1], c, o.y)) : 0.f;
+              s2 += j <= pw.z ? ex2_approx(fmaf(v[i + 2], c, o.z)) : 0.f;
+              s3 += j <= pw.w ? ex2_approx(fmaf(v[i + 3], c, o.w)) : 0.f;
             }
           }
           acc += (s0 + s1) + (s2 + s3);
         }
-        float* comb = combf + buf * (4 * 128);
-        if (sub != 0) comb[sub * 128 + q * 32 + lane] = acc;
-        // TMEM reads of this buffer are done: hand it back to the MMA issuer before the exchange
+        // TMEM reads of this buffer are done: hand it back to the MMA issuer
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&acc_empty[buf]);
-        if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-        if (sub == 0 && j < g.T) {
-          const int k = q * 32 + lane;
-          const float val = (((acc + comb[128 + k]) + comb[256 + k]) + comb[384 + k]) * g.inv_G;
-          if (p.t_acc) {
-            atomicAdd(&p.t_acc[j], (unsigned long long)llrintf(val * p.acc_scale));
-          } else {
+        if (p.t_acc) {
+          // fused pass: each warp adds its share of the rows straight into the per-token fixed-point
+          // sum (integer addition: the total does not depend on the order of arrival)
+          if (j < g.T) atomicAdd(&p.t_acc[j], to_fixed(acc * g.inv_G, p.acc_shift));
+        } else {
+          // saliency rows: the four warps sharing the keys combine in a fixed order
+          float* comb = combf + buf * (4 * 128);
+          if (sub != 0) comb[sub * 128 + q * 32 + lane] = acc;
+          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
+          if (sub == 0 && j < g.T) {
+            const int k = q * 32 + lane;
+            const float val = (((acc + comb[128 + k]) + comb[256 + k]) + comb[384 + k]) * g.inv_G;
             const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }
@@ -459,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       }
       if (++buf == 2) { buf = 0; buf_phase ^= 1; }
     }
-    if (PASS == 1 && ok && cur >= 0) ok = flush_partial(cur);
+    if (PASS == 1 && ok && cur >= 0) flush_partial(cur);
     if (!ok) {
       *abort_flag = 1;
       record_status(p.status, STEPKV_ETIMEOUT);
@@ -533,7 +550,7 @@ int score_acc_shift(int n_pairs, int W) {
 
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
   const int n_rg = score_row_groups(Hkv, Hq, W);
-  return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kMaxRows * sizeof(float2);
+  return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -568,11 +585,11 @@ static bool encode_3d(CUtensorMap* map, const void* base, int d, int rows, int h
 
 template <int PASS, int NCH>
 static cudaError_t launch_pass(const ScoreLaunch& L, int grid, cudaStream_t stream) {
-  using Cfg = ScoreCfg<NCH>;
+  using Cfg = ScoreCfg<PASS, NCH>;
   void (*kern)(ScoreLaunch) = score_kernel<PASS, NCH>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), Cfg::kDynSmem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kern, dim3(grid), dim3(kThreads), Cfg::kDynSmem, stream, L);
+  return launch_kernel(kern, dim3(grid), dim3(kThreads), Cfg::kDynSmem, stream, L);
 }
 
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
@@ -588,7 +605,7 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   L.out = rows_out;
   L.out_stride = out_stride;
   L.t_acc = t_acc;
-  L.acc_scale = ldexpf(1.0f, acc_shift);
+  L.acc_shift = acc_shift;
   L.status = status;
   const int box_rows = std::min(g.W_pad, kMaxRows);
   for (int l = 0; l < n_layers; ++l) {
@@ -622,7 +639,7 @@ stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, i
                                      cudaStream_t stream) {
   const int64_t n = (int64_t)n_pairs * T;
   const int blocks = (int)std::min<int64_t>((n + 255) / 256, 4096);
-  cudaError_t e = launch_pdl(sum_row_groups_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_pairs, n_rg, T, sal);
+  cudaError_t e = launch_kernel(sum_row_groups_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_pairs, n_rg, T, sal);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   return STEPKV_OK;
 }

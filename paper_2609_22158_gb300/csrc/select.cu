@@ -180,8 +180,9 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
   const int len = max(0, min(a.chunk, T - base));
   const bool s_in_smem = n_steps <= kSelSmemSteps;
 
-  // Work that reads only the caller's inputs runs before the wait on the score kernels: the first
-  // kernel of the pass already waited for every earlier writer of these inputs.
+  pdl_wait();  // every global read below may depend on an earlier kernel on the stream
+  pdl_launch_dependents();
+
   // ---- Phase 1+2 of Algorithm 1 (Eqs. 2-4).  With few steps every CTA keeps all S_k in shared memory
   // (CTA 0 publishes them); otherwise the steps are split over the cluster through global memory.
   if (s_in_smem) {
@@ -239,8 +240,6 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
     }
   }
 
-  pdl_wait();  // token saliency comes from the score kernels
-  pdl_launch_dependents();
   const float* Sk = s_in_smem ? sS : a.S;
 
   // ---- token saliency T_i and the prunable maximum
@@ -316,7 +315,8 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
   frexpf(vmax, &e_max);                       // vmax < 2^e_max
   const int log2N = 32 - __clz(max(N, 1));    // N < 2^log2N
   const int fx_shift = 62 - log2N - e_max;    // every partial sum < 2^62
-  const float fx_scale = ldexpf(1.0f, min(fx_shift, 126));
+  const int fx_shift_c = min(fx_shift, 126);
+  const float fx_scale = ldexpf(1.0f, fx_shift_c);
 
   // ---- priorities (Eq. 5), ordered keys and per-step statistics.  The loop bound is uniform per warp
   // (warp-aggregated atomics); T_hat is read before its shared-memory slot is overwritten by the key.
@@ -340,8 +340,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       sKey[i] = key;
     }
     const float thc = fmaxf(th, 0.f);
-    step_stat_add(act, sid, (unsigned long long)llrintf(thc * fx_scale), __float_as_uint(thc), a.acc_cnt, a.acc_sum,
-                  a.acc_max);
+    step_stat_add(act, sid, to_fixed(thc, fx_shift_c), __float_as_uint(thc), a.acc_cnt, a.acc_sum, a.acc_max);
   }
   __syncthreads();
 
@@ -563,7 +562,7 @@ __global__ void mean_rows_kernel(const float* __restrict__ rows, int n_rows, int
 stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, float* T_out,
                               cudaStream_t stream) {
   const int blocks = std::max(1, std::min((T + 255) / 256, 4096));
-  cudaError_t e = launch_pdl(mean_rows_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_rows, row_stride, inv_div,
+  cudaError_t e = launch_kernel(mean_rows_kernel, dim3(blocks), dim3(256), 0, stream, rows, n_rows, row_stride, inv_div,
                              T, T_out);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
@@ -614,7 +613,7 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
                       (steps.n_steps <= kSelSmemSteps ? (size_t)steps.n_steps * 4 : 0);
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_kernel), (int)smem);
   if (e == cudaSuccess)
-    e = launch_pdl_cluster(select_kernel, dim3(kSelCluster), dim3(kSelThreads), kSelCluster, smem, stream, a);
+    e = launch_cluster(select_kernel, dim3(kSelCluster), dim3(kSelThreads), kSelCluster, smem, stream, a);
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return STEPKV_ECUDA;

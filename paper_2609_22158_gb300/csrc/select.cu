@@ -7,12 +7,12 @@
 //   P_i   = alpha T_i + beta S_{s(i)}                                        (Eq. 5)
 //   K     = top B_t prunable tokens by (P desc, index asc), B_t from Eq. 1   (Alg. 1 Phase 3)
 //
-// GB300 design: one thread-block cluster of 8 CTAs per trajectory.  Each CTA keeps its slice of the
-// tokens in shared memory (saliency, then the order-preserving 32-bit key of P); the exact B-th
-// largest key is found by three radix passes (11/11/10 bits) whose per-CTA shared-memory histograms
-// are summed across the cluster through distributed shared memory; retained slots are written in
-// ascending order by warp ballot + prefix counts.  Per-step statistics use integer atomics only
-// (fixed-point sums), so every output is bit-reproducible run to run.
+// GB300 design: the tokens live in shared memory (saliency, then the order-preserving 32-bit key of P,
+// and a 16-bit step id) -- in one 1024-thread CTA up to 2048 tokens, else in a cluster of 8 CTAs.
+// The exact B-th largest key is found by three radix passes (11/11/10 bits) over warp-aggregated
+// shared-memory histograms (summed across the cluster through distributed shared memory); retained
+// slots are written in ascending order by warp ballot + prefix counts.  Per-step statistics use
+// integer atomics only (fixed-point sums), so every output is bit-reproducible run to run.
 #include <cooperative_groups.h>
 #include <math.h>
 
@@ -25,24 +25,28 @@ namespace cg = cooperative_groups;
 
 namespace stepkv {
 
-constexpr int kSelCluster = 8;
-constexpr int kSelThreads = 512;
-constexpr int kSelWarps = kSelThreads / 32;
+// Two shapes of the same algorithm: one 1024-thread CTA for short trajectories (no cluster barriers),
+// else a cluster of 8 CTAs of 512 threads whose histograms and counts meet through distributed shared
+// memory.  Measured on GB300 at T = 32768: one CTA 78 us, 8-CTA cluster 31 us, 16-CTA cluster 35 us
+// (the token loops shrink with more SMs, the cluster barriers and DSMEM gathers grow).
+constexpr int kSelSingleMaxT = 2048;
+constexpr int kSelClusterCtas = 8;
 
 struct SelectArgs {
   const float* T_in;                  // token saliency as floats, or
   const unsigned long long* t_acc;    // as fixed-point sums: T_i = t_acc[i] * acc_to_T
   float acc_to_T;
   int T;
-  int chunk;  // tokens per CTA
+  int chunk;                          // tokens per CTA
+  int s_in_smem;                      // S_k kept in shared memory (all CTAs compute all steps)
   const int32_t* step_id;
   const uint8_t* prot;
   stepkv_steps_t steps;
   stepkv_params_t prm;
   stepkv_budget_t budget;
   stepkv_select_out_t out;
-  float* S;                  // [n_steps] step utilities (ws or out.step_util)
-  int32_t* acc_cnt;          // [n_steps] ws accumulators (zeroed here)
+  float* S;                           // [n_steps] step utilities (workspace)
+  int32_t* acc_cnt;                   // [n_steps] workspace accumulators (zeroed here)
   unsigned long long* acc_sum;
   uint32_t* acc_max;
   int32_t* acc_kept;
@@ -59,6 +63,7 @@ struct SelShared {
   int pad[3];
 };
 
+template <int NT>
 __device__ __forceinline__ int block_reduce_sum_int(int v, int* scratch) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -66,10 +71,11 @@ __device__ __forceinline__ int block_reduce_sum_int(int v, int* scratch) {
   if (lane == 0) scratch[warp] = v;
   __syncthreads();
   int t = 0;
-  for (int w = 0; w < kSelWarps; ++w) t += scratch[w];
+  for (int w = 0; w < NT / 32; ++w) t += scratch[w];
   return t;
 }
 
+template <int NT>
 __device__ __forceinline__ float block_reduce_max(float v, float* scratch) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
@@ -77,14 +83,19 @@ __device__ __forceinline__ float block_reduce_max(float v, float* scratch) {
   if (lane == 0) scratch[warp] = v;
   __syncthreads();
   float t = -INFINITY;
-  for (int w = 0; w < kSelWarps; ++w) t = fmaxf(t, scratch[w]);
+  for (int w = 0; w < NT / 32; ++w) t = fmaxf(t, scratch[w]);
   return t;
 }
 
-// Exclusive prefix over the block of per-thread counts (thread order); returns the block total.
-__device__ __forceinline__ int block_excl_scan(int v, int* excl, int* scratch) {
+// In-place exclusive prefix of arr[0..n) with starting value `init` (block-wide, fixed order).
+template <int NT>
+__device__ __forceinline__ void block_scan_array(int* arr, int n, int init, int* scratch) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int x = v;
+  const int per = (n + NT - 1) / NT;
+  const int lo = min(n, (int)threadIdx.x * per), hi = min(n, lo + per);
+  int mine = 0;
+  for (int i = lo; i < hi; ++i) mine += arr[i];
+  int x = mine;
   for (int o = 1; o < 32; o <<= 1) {
     const int y = __shfl_up_sync(0xffffffffu, x, o);
     if (lane >= o) x += y;
@@ -92,17 +103,15 @@ __device__ __forceinline__ int block_excl_scan(int v, int* excl, int* scratch) {
   __syncthreads();
   if (lane == 31) scratch[warp] = x;
   __syncthreads();
-  int before = 0, total = 0;
-  for (int w = 0; w < kSelWarps; ++w) {
-    if (w < warp) before += scratch[w];
-    total += scratch[w];
+  int run = init + x - mine;
+  for (int w = 0; w < warp; ++w) run += scratch[w];
+  for (int i = lo; i < hi; ++i) {
+    const int c = arr[i];
+    arr[i] = run;
+    run += c;
   }
-  *excl = before + x - v;
-  return total;
+  __syncthreads();
 }
-
-constexpr int kSelUnroll = 8;          // tokens per thread with loads in flight together
-constexpr int kSelSmemSteps = 4096;    // S_k kept in shared memory up to this many steps
 
 // One step-statistics contribution per warp when the warp's (consecutive) tokens share one step, else
 // one per lane.  Integer atomics only: the totals do not depend on the order of arrival.
@@ -144,33 +153,41 @@ __device__ __forceinline__ float step_utility(const SelectArgs& a, int k, int t_
   return fminf(fmaxf(p.w_r * rc + p.w_c * log1pf(c), 0.f), p.s_max);               // Eq. 4
 }
 
-// Read the 8 per-CTA exchange blocks once (one thread per remote CTA) into a local shared-memory copy.
-__device__ __forceinline__ void gather_exchange(cg::cluster_group& cluster, SelShared* ex, SelShared* all) {
-  if (threadIdx.x < kSelCluster) {
-    const SelShared* rex = cluster.map_shared_rank(ex, (int)threadIdx.x);
-    const int4 v0 = reinterpret_cast<const int4*>(rex)[0];
-    const int4 v1 = reinterpret_cast<const int4*>(rex)[1];
-    reinterpret_cast<int4*>(&all[threadIdx.x])[0] = v0;
-    reinterpret_cast<int4*>(&all[threadIdx.x])[1] = v1;
-  }
-  __syncthreads();
-}
+template <int NC>
+struct ClusterOps {
+  cg::cluster_group cluster;
+  __device__ ClusterOps() : cluster(cg::this_cluster()) {}
+  __device__ int rank() const { return (int)cluster.block_rank(); }
+  __device__ void sync() { cluster.sync(); }
+  template <typename P>
+  __device__ P* peer(P* p, int r) { return cluster.map_shared_rank(p, r); }
+};
+template <>
+struct ClusterOps<1> {
+  __device__ int rank() const { return 0; }
+  __device__ void sync() { __syncthreads(); }
+  template <typename P>
+  __device__ P* peer(P* p, int) { return p; }
+};
 
-__global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs a) {
-  cg::cluster_group cluster = cg::this_cluster();
-  const int rank = (int)cluster.block_rank();
+template <int NC, int NT>
+__global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
+  constexpr int NW = NT / 32;
+  constexpr int UNROLL = NT >= 1024 ? 4 : 8;
+  ClusterOps<NC> cl;
+  const int rank = cl.rank();
   extern __shared__ __align__(16) uint8_t smem_raw[];
   // layout: [chunk] float/uint32 keys | [chunk] u16 step id (0xFFFF = protected) | 2 x 2048 int hist |
-  //         SelShared (own) | SelShared[8] (gathered) | scratch | S_k
+  //         SelShared (own) | SelShared[NC] (gathered) | scratch[64] | S_k (when s_in_smem)
   uint32_t* sKey = reinterpret_cast<uint32_t*>(smem_raw);
   float* sT = reinterpret_cast<float*>(smem_raw);
   uint16_t* sSid = reinterpret_cast<uint16_t*>(smem_raw + (size_t)a.chunk * 4);
   int* hist = reinterpret_cast<int*>(smem_raw + (((size_t)a.chunk * 6 + 15) & ~size_t(15)));
   SelShared* ex = reinterpret_cast<SelShared*>(hist + 2 * 2048);
   SelShared* all = ex + 1;
-  int* scratch = reinterpret_cast<int*>(all + kSelCluster);   // 64 ints
-  int* bcast = scratch + 48;                                   // 4 ints (radix passes)
-  float* sS = reinterpret_cast<float*>(scratch + 64);          // [kSelSmemSteps] when n_steps fits
+  int* scratch = reinterpret_cast<int*>(all + NC);  // 64 ints
+  int* bcast = scratch + 48;                        // radix decision
+  float* sS = reinterpret_cast<float*>(scratch + 64);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
@@ -178,15 +195,15 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
   const int t_last = n_steps - 1;
   const int base = rank * a.chunk;
   const int len = max(0, min(a.chunk, T - base));
-  const bool s_in_smem = n_steps <= kSelSmemSteps;
+  const bool s_in_smem = a.s_in_smem != 0;
 
   pdl_wait();  // every global read below may depend on an earlier kernel on the stream
   pdl_launch_dependents();
 
   // ---- Phase 1+2 of Algorithm 1 (Eqs. 2-4).  With few steps every CTA keeps all S_k in shared memory
-  // (CTA 0 publishes them); otherwise the steps are split over the cluster through global memory.
+  // (CTA 0 publishes them); otherwise the steps are split over the CTAs through global memory.
   if (s_in_smem) {
-    for (int k = tid; k < n_steps; k += kSelThreads) {
+    for (int k = tid; k < n_steps; k += NT) {
       float c;
       const float sk = step_utility(a, k, t_last, &c);
       sS[k] = sk;
@@ -197,7 +214,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       }
     }
   } else {
-    for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
+    for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
       float c;
       const float sk = step_utility(a, k, t_last, &c);
       a.S[k] = sk;
@@ -205,31 +222,38 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       if (a.steps.reuse_out) a.steps.reuse_out[k] = c;
     }
   }
-  for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
+  for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
     a.acc_cnt[k] = 0;
     a.acc_sum[k] = 0ull;
     a.acc_max[k] = 0u;
     a.acc_kept[k] = 0;
   }
-  // step ids and protection flags of this CTA's tokens
+
+  // ---- this CTA's tokens: step ids / protection flags and token saliency T_i (loads batched)
+  float lmax = -INFINITY;
   int lN = 0, lerr = 0;
-  for (int i0 = 0; i0 < len; i0 += kSelThreads * kSelUnroll) {
-    uint8_t pv[kSelUnroll];
-    int sv[kSelUnroll];
+  for (int i0 = 0; i0 < len; i0 += NT * UNROLL) {
+    float tv[UNROLL];
+    uint8_t pv[UNROLL];
+    int sv[UNROLL];
 #pragma unroll
-    for (int u = 0; u < kSelUnroll; ++u) {
-      const int i = i0 + u * kSelThreads + tid;
+    for (int u = 0; u < UNROLL; ++u) {
+      const int i = i0 + u * NT + tid;
       if (i < len) {
-        pv[u] = __ldg(&a.prot[base + i]);
-        sv[u] = __ldg(&a.step_id[base + i]);
+        const int gi = base + i;
+        pv[u] = __ldg(&a.prot[gi]);
+        sv[u] = __ldg(&a.step_id[gi]);
+        tv[u] = a.t_acc ? __ull2float_rn(__ldcg(&a.t_acc[gi])) * a.acc_to_T : __ldcg(&a.T_in[gi]);
       }
     }
 #pragma unroll
-    for (int u = 0; u < kSelUnroll; ++u) {
-      const int i = i0 + u * kSelThreads + tid;
+    for (int u = 0; u < UNROLL; ++u) {
+      const int i = i0 + u * NT + tid;
       if (i < len) {
+        sT[i] = tv[u];
         if (!pv[u]) {
           ++lN;
+          lmax = fmaxf(lmax, tv[u]);
           const bool bad = sv[u] < 0 || sv[u] >= n_steps;
           if (bad) lerr = 1;
           sSid[i] = bad ? 0 : (uint16_t)sv[u];
@@ -239,52 +263,34 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       }
     }
   }
-
-  const float* Sk = s_in_smem ? sS : a.S;
-
-  // ---- token saliency T_i and the prunable maximum
-  float lmax = -INFINITY;
-  for (int i0 = 0; i0 < len; i0 += kSelThreads * kSelUnroll) {
-    float tv[kSelUnroll];
-#pragma unroll
-    for (int u = 0; u < kSelUnroll; ++u) {
-      const int i = i0 + u * kSelThreads + tid;
-      if (i < len) {
-        const int gi = base + i;
-        tv[u] = a.t_acc ? __ull2float_rn(__ldcg(&a.t_acc[gi])) * a.acc_to_T : __ldcg(&a.T_in[gi]);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kSelUnroll; ++u) {
-      const int i = i0 + u * kSelThreads + tid;
-      if (i < len) {
-        sT[i] = tv[u];
-        if (sSid[i] != 0xFFFF) lmax = fmaxf(lmax, tv[u]);
-      }
-    }
-  }
   {
-    const float bm = block_reduce_max(lmax, reinterpret_cast<float*>(scratch));
-    const int bn = block_reduce_sum_int(lN, scratch);
-    const int be = block_reduce_sum_int(lerr, scratch);
+    const float bm = block_reduce_max<NT>(lmax, reinterpret_cast<float*>(scratch));
+    const int bn = block_reduce_sum_int<NT>(lN, scratch);
+    const int be = block_reduce_sum_int<NT>(lerr, scratch);
     if (tid == 0) {
       ex->loc_max = bm;
       ex->loc_N = bn;
       ex->loc_err = be;
     }
   }
-  cluster.sync();  // (A) S_k, zeroed accumulators and per-CTA summaries visible cluster-wide
+  cl.sync();  // (A) S_k, zeroed accumulators and per-CTA summaries visible to every CTA
   if (s_in_smem && rank == 0 && a.steps.reuse_out) {
-    for (int k = tid; k < n_steps; k += kSelThreads) {
+    for (int k = tid; k < n_steps; k += NT) {
       float c;
       step_utility(a, k, t_last, &c);
       a.steps.reuse_out[k] = c;
     }
   }
-  gather_exchange(cluster, ex, all);
+  if (tid < NC) {
+    const int4* rex = reinterpret_cast<const int4*>(cl.peer(ex, tid));
+    const int4 v0 = rex[0], v1 = rex[1];
+    reinterpret_cast<int4*>(&all[tid])[0] = v0;
+    reinterpret_cast<int4*>(&all[tid])[1] = v1;
+  }
+  __syncthreads();
   float gmax = -INFINITY;
   int N = 0, err = 0;
-  for (int r = 0; r < kSelCluster; ++r) {
+  for (int r = 0; r < NC; ++r) {
     gmax = fmaxf(gmax, all[r].loc_max);
     N += all[r].loc_N;
     err += all[r].loc_err;
@@ -295,7 +301,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       *a.out.n_kept = 0;
       if (a.out.n_budget) { a.out.n_budget[0] = N; a.out.n_budget[1] = 0; }
     }
-    cluster.sync();
+    cl.sync();
     return;
   }
   // ---- budget (Eq. 1): B = max(1, floor(num N / den)) or a count, then |K| = min(B, N)
@@ -314,13 +320,12 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
   int e_max;
   frexpf(vmax, &e_max);                       // vmax < 2^e_max
   const int log2N = 32 - __clz(max(N, 1));    // N < 2^log2N
-  const int fx_shift = 62 - log2N - e_max;    // every partial sum < 2^62
-  const int fx_shift_c = min(fx_shift, 126);
-  const float fx_scale = ldexpf(1.0f, fx_shift_c);
+  const int fx_shift = min(62 - log2N - e_max, 126);  // every partial sum < 2^62
+  const float* Sk = s_in_smem ? sS : a.S;
 
   // ---- priorities (Eq. 5), ordered keys and per-step statistics.  The loop bound is uniform per warp
   // (warp-aggregated atomics); T_hat is read before its shared-memory slot is overwritten by the key.
-  for (int i0 = 0; i0 < len; i0 += kSelThreads) {
+  for (int i0 = 0; i0 < len; i0 += NT) {
     const int i = i0 + tid;
     const bool in = i < len;
     const int gi = base + i;
@@ -340,7 +345,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       sKey[i] = key;
     }
     const float thc = fmaxf(th, 0.f);
-    step_stat_add(act, sid, to_fixed(thc, fx_shift_c), __float_as_uint(thc), a.acc_cnt, a.acc_sum, a.acc_max);
+    step_stat_add(act, sid, to_fixed(thc, fx_shift), __float_as_uint(thc), a.acc_cnt, a.acc_sum, a.acc_max);
   }
   __syncthreads();
 
@@ -357,10 +362,10 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       const int nbits = pass < 2 ? 11 : 10;
       const int sh = pass == 0 ? 21 : (pass == 1 ? 10 : 0);
       const int nb = 1 << nbits;
-      for (int b = tid; b < nb; b += kSelThreads) h[b] = 0;
+      for (int b = tid; b < nb; b += NT) h[b] = 0;
       __syncthreads();
       // keys of one step share their leading bits, so many lanes hit the same bin: aggregate per warp
-      for (int i0 = 0; i0 < len; i0 += kSelThreads) {
+      for (int i0 = 0; i0 < len; i0 += NT) {
         const int i = i0 + tid;
         const uint32_t k = i < len ? sKey[i] : 0u;
         const bool hit = i < len && sSid[i] != 0xFFFF && (k & mask) == prefix;
@@ -368,31 +373,37 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
         const unsigned peers = __match_any_sync(0xffffffffu, bin);
         if (hit && (__ffs(peers) - 1) == lane) atomicAdd(&h[bin], __popc(peers));
       }
-      cluster.sync();  // every CTA's histogram of this pass is complete
-      // global histogram; thread t owns bins [t*bpt, (t+1)*bpt): one vector load per remote CTA, all in flight
+      cl.sync();  // every CTA's histogram of this pass is complete
+      // global histogram; thread t owns bins [t*bpt, (t+1)*bpt)
+      const int bpt = nb / NT;  // 1, 2 or 4
       int cnt[4] = {0, 0, 0, 0};
-      if (nb == 2048) {
-        int4 v[kSelCluster];
+      if (bpt == 4) {
+        int4 v[NC];
 #pragma unroll
-        for (int r = 0; r < kSelCluster; ++r) v[r] = reinterpret_cast<const int4*>(cluster.map_shared_rank(h, r))[tid];
+        for (int r = 0; r < NC; ++r) v[r] = reinterpret_cast<const int4*>(cl.peer(h, r))[tid];
 #pragma unroll
-        for (int r = 0; r < kSelCluster; ++r) {
+        for (int r = 0; r < NC; ++r) {
           cnt[0] += v[r].x;
           cnt[1] += v[r].y;
           cnt[2] += v[r].z;
           cnt[3] += v[r].w;
         }
-      } else {
-        int2 v[kSelCluster];
+      } else if (bpt == 2) {
+        int2 v[NC];
 #pragma unroll
-        for (int r = 0; r < kSelCluster; ++r) v[r] = reinterpret_cast<const int2*>(cluster.map_shared_rank(h, r))[tid];
+        for (int r = 0; r < NC; ++r) v[r] = reinterpret_cast<const int2*>(cl.peer(h, r))[tid];
 #pragma unroll
-        for (int r = 0; r < kSelCluster; ++r) {
+        for (int r = 0; r < NC; ++r) {
           cnt[0] += v[r].x;
           cnt[1] += v[r].y;
         }
+      } else {
+        int v[NC];
+#pragma unroll
+        for (int r = 0; r < NC; ++r) v[r] = cl.peer(h, r)[tid];
+#pragma unroll
+        for (int r = 0; r < NC; ++r) cnt[0] += v[r];
       }
-      const int bpt = nb / kSelThreads;  // 4 or 2
       const int mine = cnt[0] + cnt[1] + cnt[2] + cnt[3];
       // keys in bins owned by higher threads: suffix scan over the block
       int x = mine;
@@ -403,7 +414,7 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
       if (lane == 0) scratch[warp] = x;
       __syncthreads();
       int after = 0;
-      for (int w = warp + 1; w < kSelWarps; ++w) after += scratch[w];
+      for (int w = warp + 1; w < NW; ++w) after += scratch[w];
       int above = after + x - mine;
       for (int q = bpt - 1; q >= 0; --q) {
         if (above < remaining && remaining <= above + cnt[q]) {
@@ -427,24 +438,30 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
   // ---- per-CTA counts: protected + strictly greater, ties at the threshold
   {
     int kb = 0, eq = 0;
-    for (int i = tid; i < len; i += kSelThreads) {
+    for (int i = tid; i < len; i += NT) {
       if (sSid[i] == 0xFFFF) ++kb;
       else if (sKey[i] > kth) ++kb;
       else if (sKey[i] == kth) ++eq;
     }
-    const int bkb = block_reduce_sum_int(kb, scratch);
-    const int beq = block_reduce_sum_int(eq, scratch);
+    const int bkb = block_reduce_sum_int<NT>(kb, scratch);
+    const int beq = block_reduce_sum_int<NT>(eq, scratch);
     if (tid == 0) {
       ex->loc_keep_base = bkb;
       ex->loc_eq = beq;
     }
   }
-  cluster.sync();  // (B)
-  gather_exchange(cluster, ex, all);
+  cl.sync();  // (B)
+  if (tid < NC) {
+    const int4* rex = reinterpret_cast<const int4*>(cl.peer(ex, tid));
+    const int4 v0 = rex[0], v1 = rex[1];
+    reinterpret_cast<int4*>(&all[tid])[0] = v0;
+    reinterpret_cast<int4*>(&all[tid])[1] = v1;
+  }
+  __syncthreads();
   // offsets: CTA r keeps its protected + strictly-greater tokens and the ties that fall within the
   // first need_eq ties in slot order
   int out_off = 0, total_kept = 0, ties_before = 0, eq_cum = 0;
-  for (int r = 0; r < kSelCluster; ++r) {
+  for (int r = 0; r < NC; ++r) {
     const int granted = max(0, min(need_eq - eq_cum, all[r].loc_eq));
     const int kept_r = all[r].loc_keep_base + granted;
     if (r < rank) {
@@ -461,80 +478,61 @@ __global__ void __launch_bounds__(kSelThreads, 1) select_kernel(const SelectArgs
     if (overflow) record_status(a.status, STEPKV_ENOSPACE);
   }
 
-  // ---- ordered write of the retained slots.  Token i of round r = i / 512 is handled by thread i % 512;
-  // each warp records per-round tie and keep counts, two block-wide prefix passes order them.
+  // ---- ordered write of the retained slots.  Token i of round r = i / NT is handled by thread i % NT;
+  // each warp records per-round tie and keep counts, block-wide prefix passes order them.
   if (!overflow) {
-    const int n_rounds = (len + kSelThreads - 1) / kSelThreads;
-    int* cnt_eq = reinterpret_cast<int*>(hist);              // [rounds][warps]
-    int* cnt_keep = cnt_eq + n_rounds * kSelWarps;            // [rounds][warps]
-    // (1) tie counts per (round, warp)
+    const int n_rounds = (len + NT - 1) / NT;
+    int* cnt_eq = hist;                           // [rounds][warps] (the histograms are no longer read)
+    int* cnt_keep = cnt_eq + n_rounds * NW;       // [rounds][warps]
     for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * kSelThreads + tid;
+      const int i = r * NT + tid;
       const bool is_eq = i < len && sSid[i] != 0xFFFF && sKey[i] == kth;
       const unsigned m = __ballot_sync(0xffffffffu, is_eq);
-      if (lane == 0) cnt_eq[r * kSelWarps + warp] = __popc(m);
+      if (lane == 0) cnt_eq[r * NW + warp] = __popc(m);
     }
     __syncthreads();
-    // exclusive prefix over (round, warp) in slot order, one warp per 32 entries (serial over few rounds)
-    if (tid == 0) {
-      int run = ties_before;
-      for (int e = 0; e < n_rounds * kSelWarps; ++e) {
-        const int c = cnt_eq[e];
-        cnt_eq[e] = run;
-        run += c;
-      }
-    }
-    __syncthreads();
-    // (2) keep flags and keep counts per (round, warp)
+    block_scan_array<NT>(cnt_eq, n_rounds * NW, ties_before, scratch);
     for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * kSelThreads + tid;
+      const int i = r * NT + tid;
       const bool in = i < len;
       const uint32_t k = in ? sKey[i] : 0u;
       const bool pr = in && sSid[i] == 0xFFFF;
       const bool is_eq = in && !pr && k == kth;
       const unsigned em = __ballot_sync(0xffffffffu, is_eq);
-      const int eq_rank = cnt_eq[r * kSelWarps + warp] + __popc(em & ((1u << lane) - 1u));
+      const int eq_rank = cnt_eq[r * NW + warp] + __popc(em & ((1u << lane) - 1u));
       const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
       const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (lane == 0) cnt_keep[r * kSelWarps + warp] = __popc(km);
+      if (lane == 0) cnt_keep[r * NW + warp] = __popc(km);
     }
     __syncthreads();
-    if (tid == 0) {
-      int run = out_off;
-      for (int e = 0; e < n_rounds * kSelWarps; ++e) {
-        const int c = cnt_keep[e];
-        cnt_keep[e] = run;
-        run += c;
-      }
-    }
-    __syncthreads();
-    // (3) write
+    block_scan_array<NT>(cnt_keep, n_rounds * NW, out_off, scratch);
     for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * kSelThreads + tid;
+      const int i = r * NT + tid;
       const bool in = i < len;
       const uint32_t k = in ? sKey[i] : 0u;
       const int sid = in ? sSid[i] : 0xFFFF;
       const bool pr = in && sid == 0xFFFF;
       const bool is_eq = in && !pr && k == kth;
       const unsigned em = __ballot_sync(0xffffffffu, is_eq);
-      const int eq_rank = cnt_eq[r * kSelWarps + warp] + __popc(em & ((1u << lane) - 1u));
+      const int eq_rank = cnt_eq[r * NW + warp] + __popc(em & ((1u << lane) - 1u));
       const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
       const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (keep) a.out.kept_idx[cnt_keep[r * kSelWarps + warp] + __popc(km & ((1u << lane) - 1u))] = base + i;
+      if (keep) a.out.kept_idx[cnt_keep[r * NW + warp] + __popc(km & ((1u << lane) - 1u))] = base + i;
       const bool kept_prunable = keep && !pr;
       step_stat_add(kept_prunable, sid, 0ull, 0u, a.acc_kept, nullptr, nullptr);
     }
   }
-  cluster.sync();  // (C) all step accumulators final
+  cl.sync();  // (C) all step accumulators final
 
   // ---- per-step outputs
-  for (int k = rank * kSelThreads + tid; k < n_steps; k += kSelCluster * kSelThreads) {
+  const double fx_unit = ldexp(1.0, -fx_shift);
+  for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
     if (a.out.step_count) a.out.step_count[k] = a.acc_cnt[k];
-    if (a.out.step_sal_sum) a.out.step_sal_sum[k] = (float)((double)a.acc_sum[k] / (double)fx_scale);
+    if (a.out.step_sal_sum) a.out.step_sal_sum[k] = (float)((double)a.acc_sum[k] * fx_unit);
     if (a.out.step_sal_max) a.out.step_sal_max[k] = __uint_as_float(a.acc_max[k]);
     if (a.out.step_kept) a.out.step_kept[k] = a.acc_kept[k];
   }
-  cluster.sync();  // no CTA exits while another may still read its shared memory
+  if (NC > 1) cl.sync();  // no CTA exits while another may still read its shared memory
 }
 
 // -------------------------------------------------------------------------------------------------
@@ -587,9 +585,8 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
   memset(&a, 0, sizeof(a));
   a.T_in = T_in;
   a.t_acc = t_acc;
-  a.acc_to_T = acc_to_T;
+  a.acc_to_T = (float)acc_to_T;
   a.T = T;
-  a.chunk = ((T + kSelCluster - 1) / kSelCluster + 15) & ~15;
   a.step_id = step_id;
   a.prot = prot;
   a.steps = steps;
@@ -608,12 +605,23 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
   w += align256(n * 4);
   a.acc_kept = reinterpret_cast<int32_t*>(w);
   a.status = status;
-  const size_t smem = (((size_t)a.chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + kSelCluster) * sizeof(SelShared) +
-                      64 * 4 +
-                      (steps.n_steps <= kSelSmemSteps ? (size_t)steps.n_steps * 4 : 0);
-  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(select_kernel), (int)smem);
-  if (e == cudaSuccess)
-    e = launch_cluster(select_kernel, dim3(kSelCluster), dim3(kSelThreads), kSelCluster, smem, stream, a);
+  const int nc = T <= kSelSingleMaxT ? 1 : kSelClusterCtas;
+  a.chunk = ((T + nc - 1) / nc + 15) & ~15;
+  const size_t fixed = (((size_t)a.chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) + 64 * 4;
+  const size_t budget_smem = 232448 - 1024;
+  a.s_in_smem = fixed + (size_t)steps.n_steps * 4 <= budget_smem ? 1 : 0;
+  const size_t smem = fixed + (a.s_in_smem ? (size_t)steps.n_steps * 4 : 0);
+  cudaError_t e;
+  if (nc == 1) {
+    void (*kern)(SelectArgs) = select_kernel<1, 1024>;
+    e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
+    if (e == cudaSuccess) e = launch_kernel(kern, dim3(1), dim3(1024), smem, stream, a);
+  } else {
+    void (*kern)(SelectArgs) = select_kernel<kSelClusterCtas, 512>;
+    e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
+    if (e == cudaSuccess)
+      e = launch_cluster(kern, dim3(kSelClusterCtas), dim3(512), kSelClusterCtas, smem, stream, a);
+  }
   if (e != cudaSuccess) {
     set_last_cuda_error(e);
     return STEPKV_ECUDA;

@@ -123,6 +123,17 @@ def test_select_matches_oracle(B, seed):
     TL.check_select_outputs(g, out)
 
 
+@pytest.mark.parametrize("T", [2047, 2048, 2049, 2065])
+def test_select_single_cta_cluster_boundary(B, T):
+    """Up to 2048 tokens one CTA selects, above that an 8-CTA cluster: both sides of the switch."""
+    tr = wl.custom(17, L=1, Hq=4, Hkv=1, d=64, T=T, W=16, n_steps=7, budget=wl.Budget.ratio(1, 4))
+    rng = np.random.default_rng(T)
+    sal = (rng.random((2, tr.T)) * 2).astype(np.float32)
+    g, out, st = _select_case(B, tr, B.Params(), sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
 @pytest.mark.parametrize("budget", [wl.Budget.ratio(1, 10), wl.Budget.ratio(1, 2), wl.Budget.fixed(1),
                                     wl.Budget.fixed(5000), wl.Budget.ratio(1, 1), wl.Budget.fixed(0)])
 def test_select_budgets(B, budget):

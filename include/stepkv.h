@@ -24,6 +24,8 @@
  *  - The library never allocates or frees memory and keeps no state between calls; scratch
  *    memory is the caller's `ws` (size from the matching *_workspace_size function, 256-byte
  *    aligned).  Calls on different streams with different workspaces may run concurrently.
+ *    The one exception is stepkv_select_static_scratch (below), which takes no workspace and uses
+ *    a fixed scratch array compiled into the library instead.
  *  - Errors: argument problems are detected on the host and returned (STEPKV_EINVAL,
  *    STEPKV_EUNSUPPORTED, STEPKV_ENOSPACE) before anything is enqueued.  A failed launch returns
  *    STEPKV_ECUDA.  Data-dependent problems found on the device (a step id out of range, kept_cap
@@ -198,6 +200,42 @@ STEPKV_API stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_
                               const stepkv_steps_t* steps, const stepkv_params_t* params,
                               const stepkv_budget_t* budget, const stepkv_select_out_t* out,
                               void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* ---------------------------------------------------------------------------------------------
+ * Stages 2-4 without a caller workspace.  The paper has no counterpart: this is a library
+ * convenience, not part of the method.
+ *
+ * Who needs it: callers that cannot allocate device memory at call time.  A serving loop whose
+ * device memory is fully reserved up front (a KV-cache pool that holds nearly all of HBM) would
+ * see a per-call cudaMalloc fail; a latency-bound loop cannot take the device-wide
+ * synchronisation that cudaFree implies; a plain C host has no caching allocator to borrow a
+ * workspace from.  Such callers allocate their outputs once and call this instead of
+ * stepkv_select; it allocates nothing.
+ *
+ * Same arguments, results and errors as stepkv_select without (ws, ws_bytes).  The scratch is a
+ * 256-byte-aligned array of 1,146,880 bytes in the library's device image (one per device,
+ * created with the library's module), enough for the mean saliency row and the per-step
+ * accumulators up to the limits below.
+ *  - Limits: T <= STEPKV_STATIC_SCRATCH_MAX_T and n_steps <= STEPKV_STATIC_SCRATCH_MAX_STEPS.
+ *    Larger problems return STEPKV_ENOSPACE before anything is enqueued; use stepkv_select with
+ *    a workspace for them.
+ *  - Set-up: the first call on each device looks up the scratch's device address
+ *    (cudaGetSymbolAddress, which may load the library's module) and keeps it for the process.
+ *    Make that first call before any stream capture.  The address is not refreshed after
+ *    cudaDeviceReset.
+ *  - Nothing in the scratch needs to start at zero: the mean kernel overwrites the saliency row
+ *    and the selection kernel zeroes its accumulators before using them.
+ *  - Calls whose work overlaps on the device (different streams, or threads enqueueing on
+ *    different streams of the same device) share the one scratch and race.  Calls on one stream
+ *    are ordered and safe.  dev_status is the caller's device int32, as for stepkv_select.
+ */
+#define STEPKV_STATIC_SCRATCH_MAX_T 262144
+#define STEPKV_STATIC_SCRATCH_MAX_STEPS 4096
+STEPKV_API stepkv_status_t stepkv_select_static_scratch(const float* sal, int32_t n_sal, int32_t T,
+                              const int32_t* step_id, const uint8_t* prot,
+                              const stepkv_steps_t* steps, const stepkv_params_t* params,
+                              const stepkv_budget_t* budget, const stepkv_select_out_t* out,
+                              int32_t* dev_status, void* stream);
 
 /* ---------------------------------------------------------------------------------------------
  * Stage 5: compaction (Eq. 1, C_hat = C_prot || C_traj[K]).

@@ -77,6 +77,9 @@ SIGNATURES = {
     "stepkv_select_workspace_size": (_SZ, [_I32, _I32, _I32]),
     "stepkv_select": (_I32, [_VP, _I32, _I32, _VP, _VP, ctypes.POINTER(CSteps), ctypes.POINTER(CParams),
                              ctypes.POINTER(CBudget), ctypes.POINTER(CSelOut), _VP, _SZ, _VP, _VP]),
+    "stepkv_select_static_scratch": (_I32, [_VP, _I32, _I32, _VP, _VP, ctypes.POINTER(CSteps),
+                                            ctypes.POINTER(CParams), ctypes.POINTER(CBudget),
+                                            ctypes.POINTER(CSelOut), _VP, _VP]),
     "stepkv_compact": (_I32, [_I32, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _VP, _I32, _VP, _VP, _I64, _VP, _VP,
                               _VP, _VP, _VP, _VP]),
     "stepkv_compress_workspace_size": (_SZ, [ctypes.POINTER(CProblem), _I32]),
@@ -340,6 +343,42 @@ def stepkv_select(sal, step_id, prot, steps: StepSignals, params: Params, budget
                              ctypes.byref(cp), ctypes.byref(budget), ctypes.byref(co), wp, wn, status.data_ptr(),
                              _stream_handle(stream))
     _check(code, "stepkv_select")
+    return out
+
+
+# Limits of the fixed scratch compiled into the library (STEPKV_STATIC_SCRATCH_MAX_* in the header).
+STATIC_SCRATCH_MAX_T = 262144
+STATIC_SCRATCH_MAX_STEPS = 4096
+
+
+def stepkv_select_static_scratch(sal, step_id, prot, steps: StepSignals, params: Params, budget: CBudget,
+                                 out: SelectOutputs, status, stream=None) -> SelectOutputs:
+    """stepkv_select without a workspace, for callers that cannot allocate device memory at call time
+    (device memory reserved up front, no room for the synchronisation of a free, no caching allocator).
+    The library uses a fixed device scratch instead (T <= 262144, n_steps <= 4096); this wrapper
+    allocates nothing either, so `status` (a zeroed device int32) is required.  The first call on a
+    device looks up the scratch address and should come before any stream capture; calls that overlap
+    on one device share the scratch and race."""
+    torch = _torch()
+    lib = load_library()
+    _need(sal, torch.float32, "sal")
+    T = sal.shape[-1]
+    n_sal = sal.numel() // T
+    if not sal.is_contiguous():
+        raise ValueError("sal must be contiguous")
+    _need(step_id, torch.int32, "step_id", 1)
+    _need(prot, torch.uint8, "prot", 1)
+    _need(status, torch.int32, "status")
+    if step_id.numel() < T or prot.numel() < T:
+        raise ValueError("step_id/prot shorter than T")
+    if T > STATIC_SCRATCH_MAX_T or steps.n_steps > STATIC_SCRATCH_MAX_STEPS:
+        raise ValueError(f"T={T}, n_steps={steps.n_steps} exceed the static scratch limits "
+                         f"({STATIC_SCRATCH_MAX_T}, {STATIC_SCRATCH_MAX_STEPS}): use stepkv_select")
+    cs, cp, co = steps.c(), params.c(), out.c()
+    code = lib.stepkv_select_static_scratch(sal.data_ptr(), n_sal, T, step_id.data_ptr(), prot.data_ptr(),
+                                            ctypes.byref(cs), ctypes.byref(cp), ctypes.byref(budget),
+                                            ctypes.byref(co), status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_select_static_scratch")
     return out
 
 

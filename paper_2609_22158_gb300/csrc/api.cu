@@ -202,6 +202,61 @@ stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T, const 
   return select_run(Tbuf, nullptr, 0.0, T, step_id, prot, *steps, *params, *budget, *out, sel_ws, dev_status, s);
 }
 
+// Selection with a fixed device scratch instead of a caller workspace, for callers that cannot
+// allocate device memory at call time (fully pre-reserved HBM, no tolerance for the synchronisation
+// of cudaFree, no caching allocator).  Not part of the method.  The array below is the only scratch;
+// its address is looked up once per device and reused, so calls that overlap on one device race.
+// Layout: the mean saliency row (4 B per token), then the step utility, count, fixed-point sum, max
+// and kept count (24 B per step), each 256-byte aligned: 1,146,880 bytes at the limits.
+static __device__ __align__(256) unsigned char g_select_scratch[(size_t)STEPKV_STATIC_SCRATCH_MAX_T * 4 +
+                                                                (size_t)STEPKV_STATIC_SCRATCH_MAX_STEPS * 24];
+constexpr int kScratchDevices = 64;
+static std::mutex g_scratch_mu;
+static void* g_scratch_addr[kScratchDevices];
+
+static stepkv_status_t static_scratch_address(void** addr) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return STEPKV_ECUDA;
+  }
+  if (dev < 0 || dev >= kScratchDevices) return STEPKV_EUNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_select_scratch);
+    if (e != cudaSuccess || !p) {
+      set_last_cuda_error(e);
+      return STEPKV_ECUDA;
+    }
+    g_scratch_addr[dev] = p;
+  }
+  *addr = g_scratch_addr[dev];
+  return STEPKV_OK;
+}
+
+stepkv_status_t stepkv_select_static_scratch(const float* sal, int32_t n_sal, int32_t T, const int32_t* step_id,
+                                             const uint8_t* prot, const stepkv_steps_t* steps,
+                                             const stepkv_params_t* params, const stepkv_budget_t* budget,
+                                             const stepkv_select_out_t* out, int32_t* dev_status, void* stream) {
+  stepkv_status_t st = check_select_args(n_sal, T, step_id, prot, steps, params, budget, out);
+  if (st != STEPKV_OK) return st;
+  if (!sal) return STEPKV_EINVAL;
+  if (T > STEPKV_STATIC_SCRATCH_MAX_T || steps->n_steps > STEPKV_STATIC_SCRATCH_MAX_STEPS) return STEPKV_ENOSPACE;
+  const size_t t_bytes = align256((size_t)T * sizeof(float));
+  if (t_bytes + select_ws_bytes(T, steps->n_steps) > sizeof(g_select_scratch)) return STEPKV_ENOSPACE;
+  void* scratch = nullptr;
+  st = static_scratch_address(&scratch);
+  if (st != STEPKV_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  float* Tbuf = static_cast<float*>(scratch);
+  void* sel_ws = static_cast<uint8_t*>(scratch) + t_bytes;
+  st = mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, Tbuf, s);
+  if (st != STEPKV_OK) return st;
+  return select_run(Tbuf, nullptr, 0.0, T, step_id, prot, *steps, *params, *budget, *out, sel_ws, dev_status, s);
+}
+
 stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
                                int64_t in_head_stride, int32_t Hkv, int32_t d, int32_t T, const int32_t* kept_idx,
                                const int32_t* n_kept, int32_t kept_cap, void* const* K_out, void* const* V_out,

@@ -24,6 +24,7 @@
 namespace stepkv {
 
 constexpr int kEpiWarps = 16;   // four warps per TMEM lane quarter
+constexpr int kGroupWarps = 8;  // two epilogue groups, one per accumulator buffer (alternate tiles)
 constexpr int kThreads = 64 + kEpiWarps * 32;  // warp 0: TMA producer, warp 1: MMA issuer + TMEM owner, rest: epilogue
 constexpr int kKeyTile = 128;
 constexpr int kMaxRows = 256;   // query rows per row group
@@ -91,11 +92,11 @@ struct ScoreCfg {
   static constexpr int kStages = PASS == 1 ? (NCH == 2 ? 5 : 10) : (NCH == 2 ? 4 : 8);
   static constexpr int kQBytes = NCH * kQChunkBytes;
   static constexpr int kStageBytes = NCH * kKChunkBytes;
-  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;         // pass 2: float sNegOff[256]
-  static constexpr int kPwOff = kOffOff + (PASS == 2 ? kMaxRows * 4 : 0); // pass 2: int sPw[256]
-  static constexpr int kCombOff = kPwOff + (PASS == 2 ? kMaxRows * 4 : 0);// pass 2: float[2][4][128]
-  static constexpr int kBarOff = kCombOff + (PASS == 2 ? 4096 : 0);
-  static constexpr int kNumBars = 2 * kStages + 2 + 4 + 1;
+  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;             // pass 2: float sNegOff[2][256]
+  static constexpr int kPwOff = kOffOff + (PASS == 2 ? 2 * kMaxRows * 4 : 0); // pass 2: int sPw[2][256]
+  static constexpr int kCombOff = kPwOff + (PASS == 2 ? 2 * kMaxRows * 4 : 0);// pass 2: float[2][2][128]
+  static constexpr int kBarOff = kCombOff + (PASS == 2 ? 2048 : 0);
+  static constexpr int kNumBars = 2 * kStages + 2 + 4 + 2;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;                 // tmem base, abort flag
   static constexpr int kBytes = kMiscOff + 16;
   static constexpr int kDynSmem = kBytes + 1024;                          // + alignment slack
@@ -122,6 +123,90 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity) 
   return mbar_wait(bar, parity, &zero);
 }
 
+// Maximum of n consecutive values as a tree of 3-input max instructions (short dependency chain).
+template <int N>
+__device__ __forceinline__ float tree_max(const float* v) {
+  if constexpr (N == 1) {
+    return v[0];
+  } else if constexpr (N == 2) {
+    return fmaxf(v[0], v[1]);
+  } else if constexpr (N == 3) {
+    return fmax3(v[0], v[1], v[2]);
+  } else {
+    constexpr int A = N / 3, B = (N - A) / 2;
+    return fmax3(tree_max<A>(v), tree_max<B>(v + A), tree_max<N - A - B>(v + A + B));
+  }
+}
+
+// Pass 1: fold NCHUNK x 32 logits of one query row into its running (m, Z), Z = sum 2^((s - m) c).
+template <int NCHUNK>
+__device__ __forceinline__ void row_stats_update(const float (&va)[32], const float (&vb)[32], float c, float& m,
+                                                 float& Z) {
+  float mn = fmaxf(tree_max<32>(va), m);
+  if (NCHUNK == 2) mn = fmaxf(mn, tree_max<32>(vb));
+  if (mn == -INFINITY) return;
+  const float nmc = -mn * c;
+  const uint64_t c2 = f2_pack(c, c), b2 = f2_pack(nmc, nmc);
+  uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+  for (int ch = 0; ch < NCHUNK; ++ch) {
+    const float* v = ch == 0 ? va : vb;
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+#pragma unroll
+      for (int k2 = 0; k2 < 4; ++k2) {
+        float lo, hi;
+        f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, b2), lo, hi);
+        acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+      }
+    }
+  }
+  float s0, s1, s2, s3, s4, s5, s6, s7;
+  f2_unpack(acc2[0], s0, s1);
+  f2_unpack(acc2[1], s2, s3);
+  f2_unpack(acc2[2], s4, s5);
+  f2_unpack(acc2[3], s6, s7);
+  Z = Z * ex2_approx((m - mn) * c) + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
+  m = mn;
+}
+
+// Pass 2: sum over 32 query columns of 2^(s c - off_r) for key j; columns whose causal limit pw_r is
+// below j contribute nothing (only tiles that reach into the window need the test).
+__device__ __forceinline__ float key_mass(const float (&v)[32], const float* negoff, const int* pw, int j,
+                                          bool need_mask, float c) {
+  if (!need_mask) {
+    const uint64_t c2 = f2_pack(c, c);
+    uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) {
+#pragma unroll
+      for (int k2 = 0; k2 < 4; ++k2) {
+        const float2 o = *reinterpret_cast<const float2*>(&negoff[i + 2 * k2]);
+        float lo, hi;
+        f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, f2_pack(o.x, o.y)), lo, hi);
+        acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+      }
+    }
+    float t0, t1, t2, t3, t4, t5, t6, t7;
+    f2_unpack(acc2[0], t0, t1);
+    f2_unpack(acc2[1], t2, t3);
+    f2_unpack(acc2[2], t4, t5);
+    f2_unpack(acc2[3], t6, t7);
+    return ((t0 + t1) + (t2 + t3)) + ((t4 + t5) + (t6 + t7));
+  }
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+  for (int i = 0; i < 32; i += 4) {
+    const float4 o = *reinterpret_cast<const float4*>(&negoff[i]);
+    const int4 w = *reinterpret_cast<const int4*>(&pw[i]);
+    s0 += j <= w.x ? ex2_approx(fmaf(v[i + 0], c, o.x)) : 0.f;
+    s1 += j <= w.y ? ex2_approx(fmaf(v[i + 1], c, o.y)) : 0.f;
+    s2 += j <= w.z ? ex2_approx(fmaf(v[i + 2], c, o.z)) : 0.f;
+    s3 += j <= w.w ? ex2_approx(fmaf(v[i + 3], c, o.w)) : 0.f;
+  }
+  return (s0 + s1) + (s2 + s3);
+}
+
 template <int PASS, int NCH>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreLaunch p) {
   using Cfg = ScoreCfg<PASS, NCH>;
@@ -140,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   uint64_t* q_empty = q_full + 1;
   uint64_t* acc_full = q_empty + 1;    // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
-  uint64_t* epi_bar = acc_empty + 2;
+  uint64_t* epi_bar = acc_empty + 2;  // [2], one per epilogue group
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + Cfg::kMiscOff);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + Cfg::kMiscOff + 4);
 
@@ -162,9 +247,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     mbar_init(q_empty, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
-      mbar_init(&acc_empty[b], kEpiWarps);
+      mbar_init(&acc_empty[b], kGroupWarps);
     }
-    mbar_init(epi_bar, kEpiWarps);
+    mbar_init(&epi_bar[0], kGroupWarps);
+    mbar_init(&epi_bar[1], kGroupWarps);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -298,183 +384,151 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     }
   } else {
     // ------------------------------------------------------------ epilogue (16 warps, 4 per lane quarter)
+    // Two groups of 8 warps take alternate tiles (group g drains accumulator buffer g), so one group's
+    // TMEM round trips and barrier waits overlap the other group's exponentials.  Within a group, two
+    // warps share each TMEM lane quarter.
     const int ew = warp - 2;
-    const int q = warp & 3;    // TMEM lane quarter this warp may access
-    const int sub = ew >> 2;   // which of the four warps sharing the quarter
+    const int q = warp & 3;     // TMEM lane quarter this warp may access
+    const int sub = ew >> 2;    // 0..3
+    const int grp = sub >> 1;   // epilogue group = accumulator buffer
+    const int s2 = sub & 1;     // which of the group's two warps on this quarter
     const float c = g.c;
-    int buf = 0, cur = -1;
-    uint32_t buf_phase = 0, eb_phase = 0;
+    int cur = -1;
+    uint32_t acc_phase = 0, eb_phase = 0;
     RowGroup r{};
     float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row over its columns
-    int my_row = 0, my_pw = 0;
-    bool row_ok = false, ok = true;
-    float* combf = reinterpret_cast<float*>(sComb);   // pass 2 (rows output): [2 buf][4 sub][128]
+    int my_row = 0, my_pw = 0, my_e = 0;
+    bool row_ok = false, two = false, ok = true;
+    float* negoff = sNegOff + grp * kMaxRows;  // pass 2: this group's per-row offsets and causal limits
+    int* pw_tab = sPw + grp * kMaxRows;
+    float* combf = reinterpret_cast<float*>(sComb) + grp * (2 * 128);  // pass 2 rows output: [2 parity][128]
+    int n_done = 0;                                                     // tiles this group has drained
+    const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(grp * 256);
 
-    // pass 1: this warp's (m, Z) over its share of the row's keys becomes entry e of the CTA's partial
+    // pass 1: this warp's (m, Z) over its share of the row's keys becomes entry my_e of the CTA's partial
     auto flush_partial = [&](int u) {
-      const bool two = r.rows > 128;
-      const int e = two ? (sub & 1) : sub;
-      p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + e) * kMaxRows + my_row] = make_float2(m, Z);
+      p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + my_e) * kMaxRows + my_row] = make_float2(m, Z);
+    };
+    auto release_buffer = [&]() {
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[grp]);
     };
 
     for (int k = 0; k < n_my && ok; ++k) {
       const int gt = tile_at(k);
       const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
-      if (u != cur) {
-        if (PASS == 1) {
-          if (cur >= 0) flush_partial(cur);
-          r = row_group(g, u % g.n_rg);
-          my_row = (r.rows > 128 ? (sub >> 1) * 128 : 0) + q * 32 + lane;
-          const int w = r.w0 + my_row % r.blk_rows;
-          row_ok = my_row < r.rows && w < g.W;
-          my_pw = g.T - g.W + w;
-          m = -INFINITY;
-          Z = 0.f;
-        } else {
-          // Combine the pass-1 partials of unit u into per-row offsets, in contributing-CTA order.
-          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;  // previous unit's offsets no longer read
-          r = row_group(g, u % g.n_rg);
-          const int c0 = (u * g.n_tiles) / p.tpc;
-          const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
-          const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
-          for (int row = threadIdx.x - 64; row < kMaxRows; row += kEpiWarps * 32) {
-            const int w = r.w0 + row % r.blk_rows;
-            const bool valid = row < r.rows && w < g.W;
-            float off = INFINITY;
-            if (valid) {
-              float M = -INFINITY;
-              for (int ci = c0; ci <= c1; ++ci)
-                for (int e = 0; e < n_e; ++e)
-                  M = fmaxf(M, __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]).x);
-              float Zs = 0.f;
-              for (int ci = c0; ci <= c1; ++ci)
-                for (int e = 0; e < n_e; ++e) {
-                  const float2 pz = __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]);
-                  if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
-                }
-              off = M * c + __log2f(Zs);
-            }
-            sNegOff[row] = -off;
-            sPw[row] = valid ? g.T - g.W + w : -1;
-          }
-          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-        }
+      if (PASS == 1 && u != cur) {
+        // Every group flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
+        // so each of the unit's partial entries is written.
+        if (cur >= 0) flush_partial(cur);
+        r = row_group(g, u % g.n_rg);
+        two = r.rows > 128;
+        my_row = (two ? s2 * 128 : 0) + q * 32 + lane;
+        my_e = two ? grp : grp * 2 + s2;
+        const int w = r.w0 + my_row % r.blk_rows;
+        row_ok = my_row < r.rows && w < g.W;
+        my_pw = g.T - g.W + w;
+        m = -INFINITY;
+        Z = 0.f;
         cur = u;
       }
-      if (!(ok = mbar_wait(&acc_full[buf], buf_phase, abort_flag))) break;
+      if ((k & 1) != grp) continue;
+      if (PASS == 2 && u != cur) {
+        // Combine the pass-1 partials of unit u into this group's per-row offsets, in contributing-CTA
+        // order (the group no longer reads the previous unit's offsets once all its warps arrive).
+        if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
+        r = row_group(g, u % g.n_rg);
+        const int c0 = (u * g.n_tiles) / p.tpc;
+        const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+        const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
+        const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
+        const int w = r.w0 + row % r.blk_rows;
+        const bool valid = row < r.rows && w < g.W;
+        float off = INFINITY;
+        if (valid) {
+          float M = -INFINITY;
+          for (int ci = c0; ci <= c1; ++ci)
+            for (int e = 0; e < n_e; ++e)
+              M = fmaxf(M, __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]).x);
+          float Zs = 0.f;
+          for (int ci = c0; ci <= c1; ++ci)
+            for (int e = 0; e < n_e; ++e) {
+              const float2 pz = __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]);
+              if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
+            }
+          off = M * c + __log2f(Zs);
+        }
+        negoff[row] = -off;
+        pw_tab[row] = valid ? g.T - g.W + w : -1;
+        if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
+        cur = u;
+      }
+      if (!(ok = mbar_wait(&acc_full[grp], acc_phase, abort_flag))) break;
+      acc_phase ^= 1;
       tc_fence_after();
       const int key0 = tile * kKeyTile;
       const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
-      const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * 256);
       if (PASS == 1) {
-        const bool two = r.rows > 128;
-        const int col_lo = two ? (sub & 1) * 64 : sub * 32;
-        const int col_hi = col_lo + (two ? 64 : 32);
-        const uint32_t mt_col = two ? (uint32_t)((sub >> 1) * 128) : 0u;
-        for (int cc = col_lo; cc < col_hi; cc += 32) {
-          float v[32];
-          tmem_ld32(lane_base + mt_col + (uint32_t)cc, v);
-          if (!row_ok) continue;
-          const int j0 = key0 + cc;
-          if (need_mask) {
+        // Queries on the TMEM lanes.  Above 128 rows warp s2 takes M-tile s2 (128 columns = all 128 keys
+        // of the tile); otherwise the two warps split the 128 columns (keys) in halves.
+        const uint32_t col0 = two ? (uint32_t)(s2 * 128) : (uint32_t)(s2 * 64);
+        const int kofs = two ? 0 : s2 * 64;
+        const int n_pairs_ch = two ? 2 : 1;  // pairs of 32-column chunks
+#pragma unroll 1
+        for (int h2 = 0; h2 < n_pairs_ch; ++h2) {
+          float va[32], vb[32];
+          tmem_ld32x2(lane_base + col0 + (uint32_t)(h2 * 64), lane_base + col0 + (uint32_t)(h2 * 64 + 32), va, vb);
+          if (h2 == n_pairs_ch - 1) release_buffer();
+          if (row_ok) {
+            const int j0 = key0 + kofs + h2 * 64;
+            if (need_mask) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = (j0 + i <= my_pw) ? v[i] : -INFINITY;
-          }
-          float mx[11];
-#pragma unroll
-          for (int i = 0; i < 10; ++i) mx[i] = fmax3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
-          mx[10] = fmaxf(v[30], v[31]);
-          const float mn = fmax3(fmax3(mx[0], mx[1], mx[2]), fmax3(mx[3], mx[4], mx[5]),
-                                 fmax3(fmax3(mx[6], mx[7], mx[8]), fmax3(mx[9], mx[10], m), -INFINITY));
-          if (mn == -INFINITY) continue;
-          const float nmc = -mn * c;
-          const uint64_t c2 = f2_pack(c, c), b2 = f2_pack(nmc, nmc);
-          uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-          for (int i = 0; i < 32; i += 8) {
-#pragma unroll
-            for (int k2 = 0; k2 < 4; ++k2) {
-              float lo, hi;
-              f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, b2), lo, hi);
-              acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+              for (int i = 0; i < 32; ++i) {
+                va[i] = (j0 + i <= my_pw) ? va[i] : -INFINITY;
+                vb[i] = (j0 + 32 + i <= my_pw) ? vb[i] : -INFINITY;
+              }
             }
+            row_stats_update<2>(va, vb, c, m, Z);
           }
-          float s0, s1, s2, s3, s4, s5, s6, s7;
-          f2_unpack(acc2[0], s0, s1);
-          f2_unpack(acc2[1], s2, s3);
-          f2_unpack(acc2[2], s4, s5);
-          f2_unpack(acc2[3], s6, s7);
-          Z = Z * ex2_approx((m - mn) * c) + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
-          m = mn;
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&acc_empty[buf]);
       } else {
+        // Keys on the TMEM lanes: this warp sums its key's mass over query columns s2*32 + 64 i, one
+        // 32-column chunk at a time (holding two chunks in registers spills).  The buffer is released
+        // once the warp's last chunk is in registers.
         const int n_cols = (r.rows + 31) & ~31;
         const int j = key0 + q * 32 + lane;
         float acc = 0.f;
-        for (int cc = sub * 32; cc < n_cols; cc += 128) {
+        bool released = false;
+#pragma unroll 1
+        for (int cc = s2 * 32; cc < n_cols; cc += 64) {
           float v[32];
           tmem_ld32(lane_base + (uint32_t)cc, v);
-          float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
-          if (!need_mask) {
-            const uint64_t c2 = f2_pack(c, c);
-            uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
-#pragma unroll
-            for (int i = 0; i < 32; i += 8) {
-#pragma unroll
-              for (int k2 = 0; k2 < 4; ++k2) {
-                const float2 o = *reinterpret_cast<const float2*>(&sNegOff[cc + i + 2 * k2]);
-                float lo, hi;
-                f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, f2_pack(o.x, o.y)), lo, hi);
-                acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
-              }
-            }
-            float t0, t1, t2, t3, t4, t5, t6, t7;
-            f2_unpack(acc2[0], t0, t1);
-            f2_unpack(acc2[1], t2, t3);
-            f2_unpack(acc2[2], t4, t5);
-            f2_unpack(acc2[3], t6, t7);
-            s0 = t0 + t1;
-            s1 = t2 + t3;
-            s2 = t4 + t5;
-            s3 = t6 + t7;
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              const float4 o = *reinterpret_cast<const float4*>(&sNegOff[cc + i]);
-              const int4 pw = *reinterpret_cast<const int4*>(&sPw[cc + i]);
-              s0 += j <= pw.x ? ex2_approx(fmaf(v[i + 0], c, o.x)) : 0.f;
-              s1 += j <= pw.y ? ex2_approx(fmaf(v[i + 1], c, o.y)) : 0.f;
-              s2 += j <= pw.z ? ex2_approx(fmaf(v[i + 2], c, o.z)) : 0.f;
-              s3 += j <= pw.w ? ex2_approx(fmaf(v[i + 3], c, o.w)) : 0.f;
-            }
+          if (cc + 64 >= n_cols) {
+            release_buffer();
+            released = true;
           }
-          acc += (s0 + s1) + (s2 + s3);
+          acc += key_mass(v, negoff + cc, pw_tab + cc, j, need_mask, c);
         }
-        // TMEM reads of this buffer are done: hand it back to the MMA issuer
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+        if (!released) release_buffer();
         if (p.t_acc) {
           // fused pass: each warp adds its share of the rows straight into the per-token fixed-point
           // sum (integer addition: the total does not depend on the order of arrival)
           if (j < g.T) atomicAdd(&p.t_acc[j], to_fixed(acc * g.inv_G, p.acc_shift));
         } else {
-          // saliency rows: the four warps sharing the keys combine in a fixed order
-          float* comb = combf + buf * (4 * 128);
-          if (sub != 0) comb[sub * 128 + q * 32 + lane] = acc;
-          if (!(ok = epi_sync(epi_bar, eb_phase, abort_flag))) break;
-          if (sub == 0 && j < g.T) {
-            const int k = q * 32 + lane;
-            const float val = (((acc + comb[128 + k]) + comb[256 + k]) + comb[384 + k]) * g.inv_G;
+          // saliency rows: the group's two warps on this quarter combine in a fixed order (the slot
+          // alternates between the group's tiles, so a write never meets a pending read)
+          float* comb = combf + (n_done & 1) * 128;
+          if (s2 == 1) comb[q * 32 + lane] = acc;
+          if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
+          if (s2 == 0 && j < g.T) {
+            const float val = (acc + comb[q * 32 + lane]) * g.inv_G;
             const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }
         }
       }
-      if (++buf == 2) { buf = 0; buf_phase ^= 1; }
+      ++n_done;
     }
     if (PASS == 1 && ok && cur >= 0) flush_partial(cur);
     if (!ok) {

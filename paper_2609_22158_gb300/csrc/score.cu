@@ -9,14 +9,19 @@
 //                 Z = sum 2^((s - m) c), c = log2(e)/sqrt(d); one partial (m, Z) per CTA segment;
 //   pass 2  S^T = K . Q^T  (M = 128 keys, N = up to 256 query rows): per-key
 //                 sum_r 2^(s c - off_r), off_r = m_r c + log2 Z_r combined from the pass-1 partials.
+// Both passes run in one cooperative launch.  Each CTA (one per SM) owns a contiguous range of
+// (unit, key tile) items, unit = (layer, KV head, row group); it streams them forward for pass 1 and
+// backward for pass 2, so pass 2 starts on the tiles pass 1 left in L2 and on the Q already staged.
 // K tiles are TMA-staged (128-byte swizzle) through an mbarrier ring; one thread issues tcgen05.mma
-// into a double-buffered TMEM accumulator (2 x 256 columns); 8 epilogue warps read TMEM with
-// tcgen05.ld and spend one MUFU ex2 per logit.  Each CTA (one per SM) owns a contiguous range of key
-// tiles, so a (pair, row-group) unit has a few pass-1 partials that pass 2 combines in a fixed order
-// (deterministic).  Pairs are launched in groups whose K fits in L2, so pass 2 re-reads K from L2.
+// into a double-buffered TMEM accumulator (2 x 256 columns); 16 epilogue warps in two groups (one per
+// accumulator buffer, alternate items) read TMEM with tcgen05.ld and spend one MUFU ex2 per logit.
+// A unit has a few pass-1 partials (one set per contributing CTA); the pass-2 epilogue combines them
+// in a fixed order (deterministic) once every CTA has raised its pass-1 flag.
 #include <math.h>
 
 #include <algorithm>
+#include <atomic>
+#include <chrono>
 
 #include "common.cuh"
 #include "internal.h"
@@ -57,7 +62,9 @@ struct ScoreLaunch {
   int64_t out_stride;
   unsigned long long* t_acc;  // pass 2: per-token fixed-point sum over all (pair, row group) (when non-null)
   int acc_shift;      // k: fixed-point scale 2^k of t_acc
-  int zero_acc;       // pass 1: zero t_acc[0..T) first (first launch of a compression pass)
+  int zero_acc;       // zero t_acc[0..T) before any contribution is added
+  unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores `token` once its partials are written
+  unsigned long long token;   // unique per launch, so flags left by earlier launches never match
   int32_t* status;
 };
 
@@ -86,21 +93,25 @@ __host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
   return r;
 }
 
-template <int PASS, int NCH>
+// Shared memory of the kernel.  Pass 1 streams K through kStages1 stages; pass 2 through the first
+// kStages2 = kStages1 - 1 of them, and keeps its per-row tables in the last stage's bytes (free once the
+// last pass-1 MMA has completed).
+template <int NCH>
 struct ScoreCfg {
-  // Pass 1 needs no shared tables, so it affords a fifth K stage (more bytes in flight per SM).
-  static constexpr int kStages = PASS == 1 ? (NCH == 2 ? 5 : 10) : (NCH == 2 ? 4 : 8);
+  static constexpr int kStages1 = NCH == 2 ? 5 : 12;
+  static constexpr int kStages2 = kStages1 - 1;
   static constexpr int kQBytes = NCH * kQChunkBytes;
   static constexpr int kStageBytes = NCH * kKChunkBytes;
-  static constexpr int kOffOff = kQBytes + kStages * kStageBytes;             // pass 2: float sNegOff[2][256]
-  static constexpr int kPwOff = kOffOff + (PASS == 2 ? 2 * kMaxRows * 4 : 0); // pass 2: int sPw[2][256]
-  static constexpr int kCombOff = kPwOff + (PASS == 2 ? 2 * kMaxRows * 4 : 0);// pass 2: float[2][2][128]
-  static constexpr int kBarOff = kCombOff + (PASS == 2 ? 2048 : 0);
-  static constexpr int kNumBars = 2 * kStages + 2 + 4 + 2;
+  static constexpr int kTabOff = kQBytes + kStages2 * kStageBytes;   // float negoff[2][256] | int pw[2][256]
+  static constexpr int kCombOff = kTabOff + 2 * 2 * kMaxRows * 4;    // | float comb[2 grp][2 parity][128]
+  static constexpr int kBarOff = kQBytes + kStages1 * kStageBytes;
+  // k_full/k_empty per stage, q_full/q_empty, acc_full/acc_empty[2], epi[2], p1_mma_done, p1_flushed
+  static constexpr int kNumBars = 2 * kStages1 + 2 + 4 + 2 + 2;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;                 // tmem base, abort flag
   static constexpr int kBytes = kMiscOff + 16;
   static constexpr int kDynSmem = kBytes + 1024;                          // + alignment slack
   static_assert(kDynSmem <= 232448, "shared memory budget");
+  static_assert(kCombOff + 2 * 2 * 128 * 4 <= kBarOff, "pass-2 tables fit in the last stage");
 };
 
 // Pass-1 partial (m, Z) slots: one per (unit, CTA), each with 4 entries per row (one per warp that
@@ -207,25 +218,42 @@ __device__ __forceinline__ float key_mass(const float (&v)[32], const float* neg
   return (s0 + s1) + (s2 + s3);
 }
 
-template <int PASS, int NCH>
+__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+
+// Both passes in one launch.  A CTA owns a contiguous range of (unit, key tile) items; it streams them
+// forward for pass 1 and backward for pass 2, so the TMA ring, the MMA issuer and the Q staging run on
+// without a break at the change of pass (the first pass-2 tile is the last pass-1 tile, same Q).  Only
+// the pass-2 epilogue depends on other CTAs: it starts once every CTA has published its pass-1
+// partials (a flag per CTA set to this launch's token; the launch is cooperative, so all CTAs are
+// resident and the wait ends, else it gives up after the wait limit).
+template <int NCH>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreLaunch p) {
-  using Cfg = ScoreCfg<PASS, NCH>;
-  constexpr int S = Cfg::kStages;
+  using Cfg = ScoreCfg<NCH>;
+  constexpr int S1 = Cfg::kStages1, S2 = Cfg::kStages2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = sm;
   uint8_t* sK = sm + Cfg::kQBytes;
-  float* sNegOff = reinterpret_cast<float*>(sm + Cfg::kOffOff);
-  int* sPw = reinterpret_cast<int*>(sm + Cfg::kPwOff);
-  float2* sComb = reinterpret_cast<float2*>(sm + Cfg::kCombOff);
+  float* sNegOff = reinterpret_cast<float*>(sm + Cfg::kTabOff);
+  int* sPw = reinterpret_cast<int*>(sm + Cfg::kTabOff + 2 * kMaxRows * 4);
+  float* sComb = reinterpret_cast<float*>(sm + Cfg::kCombOff);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kBarOff);
   uint64_t* k_full = bars;
-  uint64_t* k_empty = bars + S;
-  uint64_t* q_full = bars + 2 * S;
+  uint64_t* k_empty = bars + S1;
+  uint64_t* q_full = bars + 2 * S1;
   uint64_t* q_empty = q_full + 1;
   uint64_t* acc_full = q_empty + 1;    // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
-  uint64_t* epi_bar = acc_empty + 2;  // [2], one per epilogue group
+  uint64_t* epi_bar = acc_empty + 2;   // [2], one per epilogue group
+  uint64_t* p1_mma_done = epi_bar + 2; // every pass-1 MMA has completed (the last stage is free)
+  uint64_t* p1_flushed = p1_mma_done + 1;  // every epilogue warp has written its pass-1 partials
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + Cfg::kMiscOff);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + Cfg::kMiscOff + 4);
 
@@ -234,12 +262,15 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   const int U = p.n_units * g.n_tiles;
   const int t_lo = blockIdx.x * p.tpc;
   const int t_hi = min(U, t_lo + p.tpc);
-  const int n_my = t_hi - t_lo;
-  // Pass 2 walks the CTA's tile range backwards: the tiles pass 1 streamed last are still in L2.
-  auto tile_at = [&](int k) { return PASS == 1 ? t_lo + k : t_hi - 1 - k; };
+  const int n1 = max(0, t_hi - t_lo);  // pass-1 items; the same number of pass-2 items follows
+  const int n_seq = 2 * n1;
+  // Item k of the CTA's sequence: pass 1 forward, then pass 2 backward (the tiles pass 1 streamed last
+  // are still in L2).
+  auto tile_at = [&](int k) { return k < n1 ? t_lo + k : t_hi - 1 - (k - n1); };
+  auto stage_of = [&](int k) { return k < n1 ? k % S1 : (k - n1) % S2; };
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < S; ++i) {
+    for (int i = 0; i < S1; ++i) {
       mbar_init(&k_full[i], 1);
       mbar_init(&k_empty[i], 1);
     }
@@ -248,9 +279,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     for (int b = 0; b < 2; ++b) {
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], kGroupWarps);
+      mbar_init(&epi_bar[b], kGroupWarps);
     }
-    mbar_init(&epi_bar[0], kGroupWarps);
-    mbar_init(&epi_bar[1], kGroupWarps);
+    mbar_init(p1_mma_done, 1);
+    mbar_init(p1_flushed, kEpiWarps);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -264,28 +296,27 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   // Zero the Q staging area once: rows the TMA never writes (MMA padding) must hold finite values.
   for (int i = threadIdx.x; i < Cfg::kQBytes / 16; i += kThreads) reinterpret_cast<uint4*>(sQ)[i] = make_uint4(0, 0, 0, 0);
   fence_proxy_async_smem();
+
+  // Every thread waits for the earlier kernels on the stream before its first global access.
+  pdl_wait();
+  pdl_launch_dependents();
+  if (p.zero_acc) {
+    for (int i = blockIdx.x * kThreads + threadIdx.x; i < g.T; i += gridDim.x * kThreads) p.t_acc[i] = 0ull;
+    __threadfence();  // ordered before this CTA's pass-1 flag, hence before any pass-2 addition
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  // Only shared memory, barriers and TMEM are set up before this point.  Every thread waits for the
-  // earlier kernels on the stream before its first global access (a per-role wait placed later was
-  // observed to let early-launched CTAs read pass-1 partials of the previous call).
-  pdl_wait();
-  pdl_launch_dependents();
-  if (PASS == 1 && p.zero_acc) {
-    for (int i = blockIdx.x * kThreads + threadIdx.x; i < g.T; i += gridDim.x * kThreads) p.t_acc[i] = 0ull;
-  }
-
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (one thread)
     if (lane == 0) {
-      int stage = 0, cur = -1;
-      uint32_t phase = 0, qe_phase = 0, q_issued = 0;
-      uint32_t used = 0, last_par = 0;  // per-stage bit: loaded at least once / parity of its last load
+      int cur = -1;
+      uint32_t qe_phase = 0, q_issued = 0;
+      uint32_t par = 0, used = 0;  // per stage: parity of its next use / loaded at least once
       bool ok = true;
-      for (int k = 0; k < n_my; ++k) {
+      for (int k = 0; k < n_seq; ++k) {
         const int gt = tile_at(k);
         const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
         const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
@@ -305,33 +336,34 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           ++q_issued;
           cur = u;
         }
-        if (!mbar_wait(&k_empty[stage], phase ^ 1, abort_flag)) { ok = false; break; }
-        mbar_arrive_expect_tx(&k_full[stage], (uint32_t)(NCH * kKChunkBytes));
+        const int st = stage_of(k);
+        const uint32_t ph = (par >> st) & 1u;
+        if (!mbar_wait(&k_empty[st], ph ^ 1u, abort_flag)) { ok = false; break; }
+        mbar_arrive_expect_tx(&k_full[st], (uint32_t)(NCH * kKChunkBytes));
         for (int c = 0; c < NCH; ++c)
-          tma_load_3d(sK + stage * Cfg::kStageBytes + c * kKChunkBytes, &p.tmK[layer], c * 64, tile * kKeyTile, h,
-                      &k_full[stage]);
-        used |= 1u << stage;
-        last_par = (last_par & ~(1u << stage)) | (phase << stage);
-        if (++stage == S) { stage = 0; phase ^= 1; }
+          tma_load_3d(sK + st * Cfg::kStageBytes + c * kKChunkBytes, &p.tmK[layer], c * 64, tile * kKeyTile, h,
+                      &k_full[st]);
+        used |= 1u << st;
+        par ^= 1u << st;
       }
       if (!ok) {
         *abort_flag = 1;
         record_status(p.status, STEPKV_ETIMEOUT);
       }
       // Drain: every copy this thread issued has landed before the CTA may exit.
-      for (int i = 0; i < S; ++i)
-        if (used >> i & 1u) mbar_wait_drain(&k_full[i], last_par >> i & 1u);
+      for (int i = 0; i < S1; ++i)
+        if (used >> i & 1u) mbar_wait_drain(&k_full[i], ((par >> i) & 1u) ^ 1u);
       if (q_issued) mbar_wait_drain(q_full, (q_issued - 1) & 1u);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (one thread)
     if (lane == 0) {
-      int stage = 0, buf = 0, cur = -1;
-      uint32_t phase = 0, buf_phase = 0, q_phase = 0;
+      int buf = 0, cur = -1;
+      uint32_t par = 0, buf_phase = 0, q_phase = 0;
       bool issued = false, ok = true;
       int last_buf = 0;
       uint32_t last_buf_parity = 0;
-      for (int k = 0; k < n_my; ++k) {
+      for (int k = 0; k < n_seq; ++k) {
         const int u = tile_at(k) / g.n_tiles;
         const RowGroup r = row_group(g, u % g.n_rg);
         if (u != cur) {
@@ -341,12 +373,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           cur = u;
         }
         if (!mbar_wait(&acc_empty[buf], buf_phase ^ 1, abort_flag)) { ok = false; break; }
-        if (!mbar_wait(&k_full[stage], phase, abort_flag)) { ok = false; break; }
+        const int st = stage_of(k);
+        if (!mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t kst = smem_u32(sK + stage * Cfg::kStageBytes);
+        const uint32_t kst = smem_u32(sK + st * Cfg::kStageBytes);
         const uint32_t qst = smem_u32(sQ);
         const uint32_t dcol = tmem_base + (uint32_t)(buf * 256);
-        if (PASS == 1) {
+        if (k < n1) {
+          // S = Q K^T: queries on M (one or two 128-row halves), the tile's 128 keys on N
           const int n_mt = r.rows > 128 ? 2 : 1;
           constexpr uint32_t idesc = umma_idesc_bf16(128, kKeyTile);
           for (int mt = 0; mt < n_mt; ++mt)
@@ -358,6 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
                         kk > 0 ? 1u : 0u);
             }
         } else {
+          // S^T = K Q^T: the tile's keys on M, the query rows on N
           const int n_mma = (r.rows + 31) & ~31;  // every TMEM column the epilogue loads is written
           const uint32_t idesc = umma_idesc_bf16(128, n_mma);
 #pragma unroll
@@ -367,12 +402,13 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             umma_bf16(dcol, umma_desc_sw128(kst + koff), umma_desc_sw128(qst + qoff), idesc, kk > 0 ? 1u : 0u);
           }
         }
-        umma_commit(&k_empty[stage]);
+        umma_commit(&k_empty[st]);
         umma_commit(&acc_full[buf]);
+        if (k == n1 - 1) umma_commit(p1_mma_done);
         issued = true;
         last_buf = buf;
         last_buf_parity = buf_phase;
-        if (++stage == S) { stage = 0; phase ^= 1; }
+        par ^= 1u << st;
         if (++buf == 2) { buf = 0; buf_phase ^= 1; }
       }
       if (!ok) {
@@ -384,7 +420,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     }
   } else {
     // ------------------------------------------------------------ epilogue (16 warps, 4 per lane quarter)
-    // Two groups of 8 warps take alternate tiles (group g drains accumulator buffer g), so one group's
+    // Two groups of 8 warps take alternate items (group g drains accumulator buffer g), so one group's
     // TMEM round trips and barrier waits overlap the other group's exponentials.  Within a group, two
     // warps share each TMEM lane quarter.
     const int ew = warp - 2;
@@ -392,84 +428,51 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     const int sub = ew >> 2;    // 0..3
     const int grp = sub >> 1;   // epilogue group = accumulator buffer
     const int s2 = sub & 1;     // which of the group's two warps on this quarter
+    const bool leader = (ew & 7) == 0;
     const float c = g.c;
-    int cur = -1;
     uint32_t acc_phase = 0, eb_phase = 0;
-    RowGroup r{};
-    float m = -INFINITY, Z = 0.f;  // pass 1: running statistics of this thread's row over its columns
-    int my_row = 0, my_pw = 0, my_e = 0;
-    bool row_ok = false, two = false, ok = true;
-    float* negoff = sNegOff + grp * kMaxRows;  // pass 2: this group's per-row offsets and causal limits
-    int* pw_tab = sPw + grp * kMaxRows;
-    float* combf = reinterpret_cast<float*>(sComb) + grp * (2 * 128);  // pass 2 rows output: [2 parity][128]
-    int n_done = 0;                                                     // tiles this group has drained
+    bool ok = true;
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(grp * 256);
-
-    // pass 1: this warp's (m, Z) over its share of the row's keys becomes entry my_e of the CTA's partial
-    auto flush_partial = [&](int u) {
-      p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + my_e) * kMaxRows + my_row] = make_float2(m, Z);
-    };
     auto release_buffer = [&]() {
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[grp]);
     };
 
-    for (int k = 0; k < n_my && ok; ++k) {
-      const int gt = tile_at(k);
-      const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
-      if (PASS == 1 && u != cur) {
-        // Every group flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
-        // so each of the unit's partial entries is written.
-        if (cur >= 0) flush_partial(cur);
-        r = row_group(g, u % g.n_rg);
-        two = r.rows > 128;
-        my_row = (two ? s2 * 128 : 0) + q * 32 + lane;
-        my_e = two ? grp : grp * 2 + s2;
-        const int w = r.w0 + my_row % r.blk_rows;
-        row_ok = my_row < r.rows && w < g.W;
-        my_pw = g.T - g.W + w;
-        m = -INFINITY;
-        Z = 0.f;
-        cur = u;
-      }
-      if ((k & 1) != grp) continue;
-      if (PASS == 2 && u != cur) {
-        // Combine the pass-1 partials of unit u into this group's per-row offsets, in contributing-CTA
-        // order (the group no longer reads the previous unit's offsets once all its warps arrive).
-        if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
-        r = row_group(g, u % g.n_rg);
-        const int c0 = (u * g.n_tiles) / p.tpc;
-        const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
-        const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
-        const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
-        const int w = r.w0 + row % r.blk_rows;
-        const bool valid = row < r.rows && w < g.W;
-        float off = INFINITY;
-        if (valid) {
-          float M = -INFINITY;
-          for (int ci = c0; ci <= c1; ++ci)
-            for (int e = 0; e < n_e; ++e)
-              M = fmaxf(M, __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]).x);
-          float Zs = 0.f;
-          for (int ci = c0; ci <= c1; ++ci)
-            for (int e = 0; e < n_e; ++e) {
-              const float2 pz = __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row]);
-              if (pz.x != -INFINITY) Zs += pz.y * ex2_approx((pz.x - M) * c);
-            }
-          off = M * c + __log2f(Zs);
+    // ---- pass 1: per-row running (m, Z) over the keys this warp sees
+    {
+      int cur = -1;
+      float m = -INFINITY, Z = 0.f;
+      int my_row = 0, my_pw = 0, my_e = 0;
+      bool row_ok = false, two = false;
+      // this warp's (m, Z) over its share of the row's keys becomes entry my_e of the CTA's partial
+      auto flush_partial = [&](int u) {
+        p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + my_e) * kMaxRows + my_row] = make_float2(m, Z);
+      };
+      for (int k = 0; k < n1 && ok; ++k) {
+        const int gt = tile_at(k);
+        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+        if (u != cur) {
+          // Every group flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
+          // so each of the unit's partial entries is written.
+          if (cur >= 0) flush_partial(cur);
+          const RowGroup r = row_group(g, u % g.n_rg);
+          two = r.rows > 128;
+          my_row = (two ? s2 * 128 : 0) + q * 32 + lane;
+          my_e = two ? grp : grp * 2 + s2;
+          const int w = r.w0 + my_row % r.blk_rows;
+          row_ok = my_row < r.rows && w < g.W;
+          my_pw = g.T - g.W + w;
+          m = -INFINITY;
+          Z = 0.f;
+          cur = u;
         }
-        negoff[row] = -off;
-        pw_tab[row] = valid ? g.T - g.W + w : -1;
-        if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
-        cur = u;
-      }
-      if (!(ok = mbar_wait(&acc_full[grp], acc_phase, abort_flag))) break;
-      acc_phase ^= 1;
-      tc_fence_after();
-      const int key0 = tile * kKeyTile;
-      const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
-      if (PASS == 1) {
+        if ((k & 1) != grp) continue;
+        if (!(ok = mbar_wait(&acc_full[grp], acc_phase, abort_flag))) break;
+        acc_phase ^= 1;
+        tc_fence_after();
+        const int key0 = tile * kKeyTile;
+        const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
         // Queries on the TMEM lanes.  Above 128 rows warp s2 takes M-tile s2 (128 columns = all 128 keys
         // of the tile); otherwise the two warps split the 128 columns (keys) in halves.
         const uint32_t col0 = two ? (uint32_t)(s2 * 128) : (uint32_t)(s2 * 64);
@@ -492,7 +495,106 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             row_stats_update<2>(va, vb, c, m, Z);
           }
         }
-      } else {
+      }
+      // End of pass 1: every warp writes its last partial; then one thread publishes the CTA's flag.
+      if (ok) {
+        if (cur >= 0) flush_partial(cur);
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(p1_flushed);
+        if (ew == 0 && lane == 0) {
+          if (mbar_wait(p1_flushed, 0, abort_flag)) {
+            __threadfence();
+            st_release_u64(&p.flags[blockIdx.x], p.token);
+          } else {
+            ok = false;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      }
+    }
+
+    // ---- pass 2: per-key mass over the query rows, with the offsets of every row of the unit
+    if (ok) {
+      int cur = -1, n_done = 0;  // n_done: pass-2 items this group has drained
+      RowGroup r{};
+      bool others_done = false;
+      float* negoff = sNegOff + grp * kMaxRows;  // this group's per-row offsets and causal limits
+      int* pw_tab = sPw + grp * kMaxRows;
+      float* combf = sComb + grp * (2 * 128);     // rows output: [2 parity][128]
+      for (int k = n1; k < n_seq && ok; ++k) {
+        if ((k & 1) != grp) continue;
+        const int gt = tile_at(k);
+        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+        if (u != cur) {
+          if (!others_done) {
+            // Wait until every CTA has published its pass-1 partials (and zeroed its share of t_acc),
+            // and until this CTA's pass-1 MMAs no longer read the stage that holds the pass-2 tables.
+            if (leader) {
+              bool all = false;
+              const uint64_t t0 = globaltimer_ns();
+              for (uint32_t it = 0; !all; ++it) {
+                bool mine = true;
+                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_acquire_u64(&p.flags[b]) == p.token;
+                all = __all_sync(0xffffffffu, mine);
+                if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) break;
+              }
+              if (all) all = mbar_wait(p1_mma_done, 0, abort_flag);
+              if (!all) {
+                *abort_flag = 1;
+                if (lane == 0) record_status(p.status, STEPKV_ETIMEOUT);
+              }
+            }
+            others_done = true;
+          }
+          // Combine the pass-1 partials of unit u into this group's per-row offsets, in contributing-CTA
+          // order (the group no longer reads the previous unit's offsets once all its warps arrive).
+          if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
+          r = row_group(g, u % g.n_rg);
+          const int c0 = (u * g.n_tiles) / p.tpc;
+          const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+          const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
+          const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
+          const int w = r.w0 + row % r.blk_rows;
+          const bool valid = row < r.rows && w < g.W;
+          float off = INFINITY;
+          if (valid) {
+            // Online log-sum-exp over the unit's entries, in a fixed order; loads are issued eight at a
+            // time so their latencies overlap.
+            const int n_ent = (c1 - c0 + 1) * n_e;
+            float M = -INFINITY, Zs = 0.f;
+            for (int i0 = 0; i0 < n_ent; i0 += 8) {
+              float2 pz[8];
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                const int i = i0 + t;
+                const int ci = c0 + i / n_e, e = i - (i / n_e) * n_e;
+                pz[t] = i < n_ent ? __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row])
+                                  : make_float2(-INFINITY, 0.f);
+              }
+#pragma unroll
+              for (int t = 0; t < 8; ++t) {
+                if (pz[t].x == -INFINITY) continue;
+                if (pz[t].x > M) {
+                  Zs = Zs * ex2_approx((M - pz[t].x) * c) + pz[t].y;
+                  M = pz[t].x;
+                } else {
+                  Zs += pz[t].y * ex2_approx((pz[t].x - M) * c);
+                }
+              }
+            }
+            off = M * c + __log2f(Zs);
+          }
+          negoff[row] = -off;
+          pw_tab[row] = valid ? g.T - g.W + w : -1;
+          if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
+          cur = u;
+        }
+        if (!(ok = mbar_wait(&acc_full[grp], acc_phase, abort_flag))) break;
+        acc_phase ^= 1;
+        tc_fence_after();
+        const int key0 = tile * kKeyTile;
+        const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
         // Keys on the TMEM lanes: this warp sums its key's mass over query columns s2*32 + 64 i, one
         // 32-column chunk at a time (holding two chunks in registers spills).  The buffer is released
         // once the warp's last chunk is in registers.
@@ -517,7 +619,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           if (j < g.T) atomicAdd(&p.t_acc[j], to_fixed(acc * g.inv_G, p.acc_shift));
         } else {
           // saliency rows: the group's two warps on this quarter combine in a fixed order (the slot
-          // alternates between the group's tiles, so a write never meets a pending read)
+          // alternates between the group's items, so a write never meets a pending read)
           float* comb = combf + (n_done & 1) * 128;
           if (s2 == 1) comb[q * 32 + lane] = acc;
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
@@ -527,10 +629,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }
         }
+        ++n_done;
       }
-      ++n_done;
     }
-    if (PASS == 1 && ok && cur >= 0) flush_partial(cur);
     if (!ok) {
       *abort_flag = 1;
       record_status(p.status, STEPKV_ETIMEOUT);
@@ -602,9 +703,13 @@ int score_acc_shift(int n_pairs, int W) {
   return 60 - e;
 }
 
-size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
+// Pass-1 partial slots, then one pass-1-done flag per CTA.
+static size_t score_partial_slots_bytes(int n_layers, int Hkv, int Hq, int W) {
   const int n_rg = score_row_groups(Hkv, Hq, W);
   return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
+}
+size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
+  return score_partial_slots_bytes(n_layers, Hkv, Hq, W) + (size_t)kMaxGrid * sizeof(unsigned long long);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -637,13 +742,44 @@ static bool encode_3d(CUtensorMap* map, const void* base, int d, int rows, int h
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int PASS, int NCH>
-static cudaError_t launch_pass(const ScoreLaunch& L, int grid, cudaStream_t stream) {
-  using Cfg = ScoreCfg<PASS, NCH>;
-  void (*kern)(ScoreLaunch) = score_kernel<PASS, NCH>;
+// A value no earlier launch in this process used (and, with the per-process salt, vanishingly unlikely to
+// be left in a workspace by another process); never zero.
+static unsigned long long next_launch_token() {
+  static std::atomic<unsigned long long> counter{0};
+  static const unsigned long long salt = [] {
+    unsigned long long x = (unsigned long long)std::chrono::steady_clock::now().time_since_epoch().count();
+    x ^= (unsigned long long)reinterpret_cast<uintptr_t>(&counter) << 17;
+    // splitmix64 finaliser
+    x += 0x9E3779B97F4A7C15ull;
+    x = (x ^ (x >> 30)) * 0xBF58476D1CE4E5B9ull;
+    x = (x ^ (x >> 27)) * 0x94D049BB133111EBull;
+    return x ^ (x >> 31);
+  }();
+  unsigned long long t = 0;
+  while (t == 0) t = salt + (counter.fetch_add(1) + 1) * 0x9E3779B97F4A7C15ull;
+  return t;
+}
+
+template <int NCH>
+static cudaError_t launch_score(const ScoreLaunch& L, int grid, cudaStream_t stream) {
+  using Cfg = ScoreCfg<NCH>;
+  void (*kern)(ScoreLaunch) = score_kernel<NCH>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), Cfg::kDynSmem);
   if (e != cudaSuccess) return e;
-  return launch_kernel(kern, dim3(grid), dim3(kThreads), Cfg::kDynSmem, stream, L);
+  // Cooperative: the pass-2 epilogue of each CTA waits for every CTA's pass-1 flag, so all CTAs must be
+  // resident at once (the launch fails instead of starting if they cannot be).
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = Cfg::kDynSmem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, L);
 }
 
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
@@ -656,6 +792,8 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   L.g = g;
   L.n_layers = n_layers;
   L.part = part;
+  L.flags = reinterpret_cast<unsigned long long*>(reinterpret_cast<uint8_t*>(part) +
+                                                  score_partial_slots_bytes(n_layers, Hkv, Hq, W));
   L.out = rows_out;
   L.out_stride = out_stride;
   L.t_acc = t_acc;
@@ -670,22 +808,17 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   cudaError_t e = device_sm_count(&n_sm);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   const int grid_cap = std::max(1, std::min(n_sm, kMaxGrid));
-  // all (layer, KV head) pairs in one launch per pass
-  const int n_pairs = n_layers * Hkv;
-  const int ppg = n_pairs;
-  for (int p0 = 0; p0 < n_pairs; p0 += ppg) {
-    const int np = std::min(ppg, n_pairs - p0);
-    L.pair0 = p0;
-    L.zero_acc = (t_acc != nullptr && p0 == 0) ? 1 : 0;
-    L.n_units = np * g.n_rg;
-    const int U = L.n_units * g.n_tiles;
-    const int grid0 = std::min(grid_cap, U);
-    L.tpc = (U + grid0 - 1) / grid0;
-    const int grid = (U + L.tpc - 1) / L.tpc;
-    e = d == 128 ? launch_pass<1, 2>(L, grid, stream) : launch_pass<1, 1>(L, grid, stream);
-    if (e == cudaSuccess) e = d == 128 ? launch_pass<2, 2>(L, grid, stream) : launch_pass<2, 1>(L, grid, stream);
-    if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
-  }
+  // all (layer, KV head) pairs in one launch: every CTA gets a contiguous range of (unit, tile) items
+  L.pair0 = 0;
+  L.zero_acc = t_acc != nullptr ? 1 : 0;
+  L.n_units = n_layers * Hkv * g.n_rg;
+  const int U = L.n_units * g.n_tiles;
+  const int grid0 = std::min(grid_cap, U);
+  L.tpc = (U + grid0 - 1) / grid0;
+  const int grid = (U + L.tpc - 1) / L.tpc;
+  L.token = next_launch_token();
+  e = d == 128 ? launch_score<2>(L, grid, stream) : launch_score<1>(L, grid, stream);
+  if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   return STEPKV_OK;
 }
 

@@ -109,7 +109,7 @@ class DeviceTraj:
 def launches_per_pass(tr) -> int:
     """Kernel launches of one stepkv_compress call (mirrors the library's launch plan)."""
     s = tr.shape
-    return 2 + 1 + math.ceil(s.L / 96)  # score pass 1, pass 2, select, compaction
+    return 1 + 1 + math.ceil(s.L / 96)  # score (both passes, one cooperative launch), select, compaction
 
 
 def algorithmic_bytes(tr, n_kept):

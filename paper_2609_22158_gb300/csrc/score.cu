@@ -93,25 +93,31 @@ __host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
   return r;
 }
 
-// Shared memory of the kernel.  Pass 1 streams K through kStages1 stages; pass 2 through the first
-// kStages2 = kStages1 - 1 of them, and keeps its per-row tables in the last stage's bytes (free once the
-// last pass-1 MMA has completed).
+// Shared memory of the kernel.
 template <int NCH>
 struct ScoreCfg {
-  static constexpr int kStages1 = NCH == 2 ? 5 : 12;
-  static constexpr int kStages2 = kStages1 - 1;
+  // Pass 1 streams pairs of key tiles: a slot is two stages whose chunks sit side by side, so one
+  // N = 256 MMA reads 256 consecutive keys.  Pass 2 streams single tiles through kStages2 stages.
+  static constexpr int kSlots1 = NCH == 2 ? 2 : 5;
+  static constexpr int kStages2 = NCH == 2 ? 4 : 10;
+  static constexpr int kStages = 2 * kSlots1 > kStages2 ? 2 * kSlots1 : kStages2;
   static constexpr int kQBytes = NCH * kQChunkBytes;
   static constexpr int kStageBytes = NCH * kKChunkBytes;
-  static constexpr int kTabOff = kQBytes + kStages2 * kStageBytes;   // float negoff[2][256] | int pw[2][256]
+  static constexpr int kTabOff = kQBytes + kStages * kStageBytes;     // float negoff[2][256] | int pw[2][256]
   static constexpr int kCombOff = kTabOff + 2 * 2 * kMaxRows * 4;    // | float comb[2 grp][2 parity][128]
-  static constexpr int kBarOff = kQBytes + kStages1 * kStageBytes;
-  // k_full/k_empty per stage, q_full/q_empty, acc_full/acc_empty[2], epi[2], p1_mma_done, p1_flushed
-  static constexpr int kNumBars = 2 * kStages1 + 2 + 4 + 2 + 2;
+  static constexpr int kBarOff = kCombOff + 2 * 2 * 128 * 4;
+  // k_full/k_empty per stage, q_full/q_empty, acc_full/acc_empty[2], epi[2], p1_flushed
+  static constexpr int kNumBars = 2 * kStages + 2 + 4 + 2 + 1;
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;                 // tmem base, abort flag
   static constexpr int kBytes = kMiscOff + 16;
   static constexpr int kDynSmem = kBytes + 1024;                          // + alignment slack
   static_assert(kDynSmem <= 232448, "shared memory budget");
-  static_assert(kCombOff + 2 * 2 * 128 * 4 <= kBarOff, "pass-2 tables fit in the last stage");
+  static_assert(kStages % 2 == 0, "stages come in pairs");
+  // Byte offset (from the first stage) of chunk c of stage s: stages 2i and 2i+1 hold their chunk c
+  // back to back, 256 consecutive keys.
+  __host__ __device__ static constexpr int chunk_off(int s, int c) {
+    return (s >> 1) * 2 * kStageBytes + c * 2 * kKChunkBytes + (s & 1) * kKChunkBytes;
+  }
 };
 
 // Pass-1 partial (m, Z) slots: one per (unit, CTA), each with 4 entries per row (one per warp that
@@ -218,25 +224,30 @@ __device__ __forceinline__ float key_mass(const float (&v)[32], const float* neg
   return (s0 + s1) + (s2 + s3);
 }
 
-__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
   unsigned long long v;
-  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
+__device__ __forceinline__ void fence_acquire_gpu() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 __device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
   asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
 // Both passes in one launch.  A CTA owns a contiguous range of (unit, key tile) items; it streams them
-// forward for pass 1 and backward for pass 2, so the TMA ring, the MMA issuer and the Q staging run on
-// without a break at the change of pass (the first pass-2 tile is the last pass-1 tile, same Q).  Only
-// the pass-2 epilogue depends on other CTAs: it starts once every CTA has published its pass-1
-// partials (a flag per CTA set to this launch's token; the launch is cooperative, so all CTAs are
-// resident and the wait ends, else it gives up after the wait limit).
+// forward for pass 1 (in pairs of tiles: one N = 256 MMA per query half) and backward for pass 2, so
+// the TMA ring, the MMA issuer and the Q staging run on without a break at the change of pass (the
+// first pass-2 tile is the last pass-1 tile, same Q).  Only the pass-2 epilogue depends on other CTAs:
+// it starts once every CTA has published its pass-1 partials (a flag per CTA set to this launch's
+// token; the launch is cooperative, so all CTAs are resident and the wait ends, else it gives up after
+// the wait limit).
+//
+// Accumulator work is counted in "halves": a pass-1 pair item gives one half per 128-row query tile,
+// a pass-2 item one half.  Half h goes to TMEM buffer h & 1 and is drained by epilogue group h & 1.
 template <int NCH>
 __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constant__ ScoreLaunch p) {
   using Cfg = ScoreCfg<NCH>;
-  constexpr int S1 = Cfg::kStages1, S2 = Cfg::kStages2;
+  constexpr int S2 = Cfg::kStages2, P1 = Cfg::kSlots1;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = sm;
@@ -246,14 +257,13 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   float* sComb = reinterpret_cast<float*>(sm + Cfg::kCombOff);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::kBarOff);
   uint64_t* k_full = bars;
-  uint64_t* k_empty = bars + S1;
-  uint64_t* q_full = bars + 2 * S1;
+  uint64_t* k_empty = bars + Cfg::kStages;
+  uint64_t* q_full = bars + 2 * Cfg::kStages;
   uint64_t* q_empty = q_full + 1;
   uint64_t* acc_full = q_empty + 1;    // [2]
   uint64_t* acc_empty = acc_full + 2;  // [2]
   uint64_t* epi_bar = acc_empty + 2;   // [2], one per epilogue group
-  uint64_t* p1_mma_done = epi_bar + 2; // every pass-1 MMA has completed (the last stage is free)
-  uint64_t* p1_flushed = p1_mma_done + 1;  // every epilogue warp has written its pass-1 partials
+  uint64_t* p1_flushed = epi_bar + 2;  // every epilogue warp has written its pass-1 partials
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + Cfg::kMiscOff);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(sm + Cfg::kMiscOff + 4);
 
@@ -262,15 +272,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   const int U = p.n_units * g.n_tiles;
   const int t_lo = blockIdx.x * p.tpc;
   const int t_hi = min(U, t_lo + p.tpc);
-  const int n1 = max(0, t_hi - t_lo);  // pass-1 items; the same number of pass-2 items follows
-  const int n_seq = 2 * n1;
-  // Item k of the CTA's sequence: pass 1 forward, then pass 2 backward (the tiles pass 1 streamed last
-  // are still in L2).
-  auto tile_at = [&](int k) { return k < n1 ? t_lo + k : t_hi - 1 - (k - n1); };
-  auto stage_of = [&](int k) { return k < n1 ? k % S1 : (k - n1) % S2; };
+  const int n1 = max(0, t_hi - t_lo);  // tiles of the CTA (each is streamed once per pass)
+  // Pass-1 items: two consecutive tiles of one unit where possible, else one.
+  auto item_tiles = [&](int t) { return (t + 1 < t_hi && (t + 1) / g.n_tiles == t / g.n_tiles) ? 2 : 1; };
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < S1; ++i) {
+    for (int i = 0; i < Cfg::kStages; ++i) {
       mbar_init(&k_full[i], 1);
       mbar_init(&k_empty[i], 1);
     }
@@ -281,7 +288,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       mbar_init(&acc_empty[b], kGroupWarps);
       mbar_init(&epi_bar[b], kGroupWarps);
     }
-    mbar_init(p1_mma_done, 1);
     mbar_init(p1_flushed, kEpiWarps);
     *abort_flag = 0;
     mbar_fence_init();
@@ -316,14 +322,13 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       uint32_t qe_phase = 0, q_issued = 0;
       uint32_t par = 0, used = 0;  // per stage: parity of its next use / loaded at least once
       bool ok = true;
-      for (int k = 0; k < n_seq; ++k) {
-        const int gt = tile_at(k);
+      auto load_tile = [&](int gt, int st) -> bool {
         const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
         const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
         const int layer = pair / g.Hkv, h = pair - layer * g.Hkv;
         if (u != cur) {
           if (cur >= 0) {
-            if (!mbar_wait(q_empty, qe_phase, abort_flag)) { ok = false; break; }
+            if (!mbar_wait(q_empty, qe_phase, abort_flag)) return false;
             qe_phase ^= 1;
           }
           const RowGroup r = row_group(g, rg);
@@ -336,91 +341,131 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           ++q_issued;
           cur = u;
         }
-        const int st = stage_of(k);
         const uint32_t ph = (par >> st) & 1u;
-        if (!mbar_wait(&k_empty[st], ph ^ 1u, abort_flag)) { ok = false; break; }
+        if (!mbar_wait(&k_empty[st], ph ^ 1u, abort_flag)) return false;
         mbar_arrive_expect_tx(&k_full[st], (uint32_t)(NCH * kKChunkBytes));
         for (int c = 0; c < NCH; ++c)
-          tma_load_3d(sK + st * Cfg::kStageBytes + c * kKChunkBytes, &p.tmK[layer], c * 64, tile * kKeyTile, h,
-                      &k_full[st]);
+          tma_load_3d(sK + Cfg::chunk_off(st, c), &p.tmK[layer], c * 64, tile * kKeyTile, h, &k_full[st]);
         used |= 1u << st;
         par ^= 1u << st;
+        return true;
+      };
+      int slot = 0;
+      for (int t = t_lo; t < t_hi && ok;) {
+        const int nt = item_tiles(t);
+        for (int i = 0; i < nt && ok; ++i) ok = load_tile(t + i, 2 * slot + i);
+        t += nt;
+        if (++slot == P1) slot = 0;
       }
+      for (int k = 0; k < n1 && ok; ++k) ok = load_tile(t_hi - 1 - k, k % S2);
       if (!ok) {
         *abort_flag = 1;
         record_status(p.status, STEPKV_ETIMEOUT);
       }
       // Drain: every copy this thread issued has landed before the CTA may exit.
-      for (int i = 0; i < S1; ++i)
+      for (int i = 0; i < Cfg::kStages; ++i)
         if (used >> i & 1u) mbar_wait_drain(&k_full[i], ((par >> i) & 1u) ^ 1u);
       if (q_issued) mbar_wait_drain(q_full, (q_issued - 1) & 1u);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer (one thread)
     if (lane == 0) {
-      int buf = 0, cur = -1;
-      uint32_t par = 0, buf_phase = 0, q_phase = 0;
-      bool issued = false, ok = true;
-      int last_buf = 0;
-      uint32_t last_buf_parity = 0;
-      for (int k = 0; k < n_seq; ++k) {
-        const int u = tile_at(k) / g.n_tiles;
-        const RowGroup r = row_group(g, u % g.n_rg);
-        if (u != cur) {
-          if (cur >= 0) umma_commit(q_empty);  // Q may be overwritten once the previous unit's MMAs finish
-          if (!mbar_wait(q_full, q_phase, abort_flag)) { ok = false; break; }
-          q_phase ^= 1;
-          cur = u;
-        }
-        if (!mbar_wait(&acc_empty[buf], buf_phase ^ 1, abort_flag)) { ok = false; break; }
-        const int st = stage_of(k);
-        if (!mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag)) { ok = false; break; }
+      int cur = -1;
+      uint32_t par = 0, buf_par = 0, q_phase = 0;  // per stage / per accumulator buffer: use parity
+      uint32_t hh = 0;                              // halves issued so far
+      bool ok = true;
+      const uint32_t qst = smem_u32(sQ);
+      auto new_unit = [&](int u) -> bool {
+        if (u == cur) return true;
+        if (cur >= 0) umma_commit(q_empty);  // Q may be overwritten once the previous unit's MMAs finish
+        if (!mbar_wait(q_full, q_phase, abort_flag)) return false;
+        q_phase ^= 1;
+        cur = u;
+        return true;
+      };
+      auto take_buffer = [&](int& b) -> bool {
+        b = (int)(hh & 1u);
+        if (!mbar_wait(&acc_empty[b], ((buf_par >> b) & 1u) ^ 1u, abort_flag)) return false;
         tc_fence_after();
-        const uint32_t kst = smem_u32(sK + st * Cfg::kStageBytes);
-        const uint32_t qst = smem_u32(sQ);
-        const uint32_t dcol = tmem_base + (uint32_t)(buf * 256);
-        if (k < n1) {
-          // S = Q K^T: queries on M (one or two 128-row halves), the tile's 128 keys on N
-          const int n_mt = r.rows > 128 ? 2 : 1;
-          constexpr uint32_t idesc = umma_idesc_bf16(128, kKeyTile);
-          for (int mt = 0; mt < n_mt; ++mt)
-#pragma unroll
-            for (int kk = 0; kk < NCH * 4; ++kk) {
-              const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + mt * 128 * 128 + (kk & 3) * 32);
-              const uint32_t koff = (uint32_t)((kk >> 2) * kKChunkBytes + (kk & 3) * 32);
-              umma_bf16(dcol + (uint32_t)(mt * 128), umma_desc_sw128(qst + qoff), umma_desc_sw128(kst + koff), idesc,
-                        kk > 0 ? 1u : 0u);
-            }
-        } else {
-          // S^T = K Q^T: the tile's keys on M, the query rows on N
-          const int n_mma = (r.rows + 31) & ~31;  // every TMEM column the epilogue loads is written
-          const uint32_t idesc = umma_idesc_bf16(128, n_mma);
+        return true;
+      };
+      auto give_buffer = [&](int b) {
+        umma_commit(&acc_full[b]);
+        buf_par ^= 1u << b;
+        ++hh;
+      };
+      // pass 1: S = Q K^T, one half per 128-row query tile, N = the item's keys (256 or 128)
+      int slot = 0;
+      for (int t = t_lo; t < t_hi && ok;) {
+        const int nt = item_tiles(t);
+        const int u = t / g.n_tiles;
+        const RowGroup r = row_group(g, u % g.n_rg);
+        if (!(ok = new_unit(u))) break;
+        for (int i = 0; i < nt && ok; ++i) {
+          const int st = 2 * slot + i;
+          ok = mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag);
+        }
+        if (!ok) break;
+        tc_fence_after();
+        const int n_mt = r.rows > 128 ? 2 : 1;
+        const uint32_t idesc = umma_idesc_bf16(128, nt * kKeyTile);
+        for (int mt = 0; mt < n_mt && ok; ++mt) {
+          int b;
+          if (!(ok = take_buffer(b))) break;
+          const uint32_t dcol = tmem_base + (uint32_t)(b * 256);
 #pragma unroll
           for (int kk = 0; kk < NCH * 4; ++kk) {
-            const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + (kk & 3) * 32);
-            const uint32_t koff = (uint32_t)((kk >> 2) * kKChunkBytes + (kk & 3) * 32);
-            umma_bf16(dcol, umma_desc_sw128(kst + koff), umma_desc_sw128(qst + qoff), idesc, kk > 0 ? 1u : 0u);
+            const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + mt * 128 * 128 + (kk & 3) * 32);
+            const uint32_t koff = (uint32_t)(Cfg::chunk_off(2 * slot, kk >> 2) + (kk & 3) * 32);
+            umma_bf16(dcol, umma_desc_sw128(qst + qoff), umma_desc_sw128(smem_u32(sK) + koff), idesc, kk > 0 ? 1u : 0u);
           }
+          give_buffer(b);
+        }
+        if (!ok) break;
+        for (int i = 0; i < nt; ++i) {
+          const int st = 2 * slot + i;
+          umma_commit(&k_empty[st]);
+          par ^= 1u << st;
+        }
+        t += nt;
+        if (++slot == P1) slot = 0;
+      }
+      // pass 2: S^T = K Q^T, the tile's keys on M, the query rows on N
+      for (int k = 0; k < n1 && ok; ++k) {
+        const int u = (t_hi - 1 - k) / g.n_tiles;
+        const RowGroup r = row_group(g, u % g.n_rg);
+        if (!(ok = new_unit(u))) break;
+        int b;
+        if (!(ok = take_buffer(b))) break;
+        const int st = k % S2;
+        if (!(ok = mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag))) break;
+        tc_fence_after();
+        const uint32_t dcol = tmem_base + (uint32_t)(b * 256);
+        const int n_mma = (r.rows + 31) & ~31;  // every TMEM column the epilogue loads is written
+        const uint32_t idesc = umma_idesc_bf16(128, n_mma);
+#pragma unroll
+        for (int kk = 0; kk < NCH * 4; ++kk) {
+          const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + (kk & 3) * 32);
+          const uint32_t koff = (uint32_t)(Cfg::chunk_off(st, kk >> 2) + (kk & 3) * 32);
+          umma_bf16(dcol, umma_desc_sw128(smem_u32(sK) + koff), umma_desc_sw128(qst + qoff), idesc, kk > 0 ? 1u : 0u);
         }
         umma_commit(&k_empty[st]);
-        umma_commit(&acc_full[buf]);
-        if (k == n1 - 1) umma_commit(p1_mma_done);
-        issued = true;
-        last_buf = buf;
-        last_buf_parity = buf_phase;
         par ^= 1u << st;
-        if (++buf == 2) { buf = 0; buf_phase ^= 1; }
+        give_buffer(b);
       }
       if (!ok) {
         *abort_flag = 1;
         record_status(p.status, STEPKV_ETIMEOUT);
       }
       // Drain: the last MMA group has completed before TMEM is released.
-      if (issued) mbar_wait_drain(&acc_full[last_buf], last_buf_parity);
+      if (hh > 0) {
+        const int lb = (int)((hh - 1) & 1u);
+        mbar_wait_drain(&acc_full[lb], ((buf_par >> lb) & 1u) ^ 1u);
+      }
     }
   } else {
     // ------------------------------------------------------------ epilogue (16 warps, 4 per lane quarter)
-    // Two groups of 8 warps take alternate items (group g drains accumulator buffer g), so one group's
+    // Two groups of 8 warps drain alternate halves (group g drains accumulator buffer g), so one group's
     // TMEM round trips and barrier waits overlap the other group's exponentials.  Within a group, two
     // warps share each TMEM lane quarter.
     const int ew = warp - 2;
@@ -430,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     const int s2 = sub & 1;     // which of the group's two warps on this quarter
     const bool leader = (ew & 7) == 0;
     const float c = g.c;
-    uint32_t acc_phase = 0, eb_phase = 0;
+    uint32_t acc_phase = 0, eb_phase = 0, hh = 0;
     bool ok = true;
     const uint32_t lane_base = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(grp * 256);
     auto release_buffer = [&]() {
@@ -449,17 +494,22 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       auto flush_partial = [&](int u) {
         p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + my_e) * kMaxRows + my_row] = make_float2(m, Z);
       };
-      for (int k = 0; k < n1 && ok; ++k) {
-        const int gt = tile_at(k);
-        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+      for (int t = t_lo; t < t_hi && ok;) {
+        const int nt = item_tiles(t);
+        const int u = t / g.n_tiles, tile = t - u * g.n_tiles;
+        t += nt;
         if (u != cur) {
-          // Every group flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
+          // Every warp flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
           // so each of the unit's partial entries is written.
           if (cur >= 0) flush_partial(cur);
           const RowGroup r = row_group(g, u % g.n_rg);
           two = r.rows > 128;
-          my_row = (two ? s2 * 128 : 0) + q * 32 + lane;
-          my_e = two ? grp : grp * 2 + s2;
+          // Above 128 rows every item has two halves, query tile mt in buffer (h0 + mt) & 1 (h0 = halves
+          // before the item, of fixed parity within the unit), so group g drains tile (g + h0) & 1 of
+          // every item; otherwise the groups alternate items over the single query tile.
+          const int mt_g = two ? (int)((grp + hh) & 1u) : 0;
+          my_row = mt_g * 128 + q * 32 + lane;
+          my_e = two ? s2 : grp * 2 + s2;
           const int w = r.w0 + my_row % r.blk_rows;
           row_ok = my_row < r.rows && w < g.W;
           my_pw = g.T - g.W + w;
@@ -467,24 +517,27 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           Z = 0.f;
           cur = u;
         }
-        if ((k & 1) != grp) continue;
+        const int n_halves = two ? 2 : 1;
+        const bool mine = two || (hh & 1u) == (uint32_t)grp;
+        hh += n_halves;
+        if (!mine) continue;
         if (!(ok = mbar_wait(&acc_full[grp], acc_phase, abort_flag))) break;
         acc_phase ^= 1;
         tc_fence_after();
-        const int key0 = tile * kKeyTile;
-        const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
-        // Queries on the TMEM lanes.  Above 128 rows warp s2 takes M-tile s2 (128 columns = all 128 keys
-        // of the tile); otherwise the two warps split the 128 columns (keys) in halves.
-        const uint32_t col0 = two ? (uint32_t)(s2 * 128) : (uint32_t)(s2 * 64);
-        const int kofs = two ? 0 : s2 * 64;
-        const int n_pairs_ch = two ? 2 : 1;  // pairs of 32-column chunks
+        // Keys on the TMEM columns: warp s2 takes half of the item's nt*128 keys, in pairs of 32-column
+        // chunks (one TMEM round trip per pair); the buffer is released once the last pair is loaded.
+        const int half_keys = nt * 64;
+        const int key0 = tile * kKeyTile + s2 * half_keys;
+        const bool need_mask = key0 + half_keys - 1 > g.T - g.W;  // reaches into the causal window
+        const int n_pairs_ch = half_keys / 64;
 #pragma unroll 1
         for (int h2 = 0; h2 < n_pairs_ch; ++h2) {
           float va[32], vb[32];
-          tmem_ld32x2(lane_base + col0 + (uint32_t)(h2 * 64), lane_base + col0 + (uint32_t)(h2 * 64 + 32), va, vb);
+          const uint32_t col = (uint32_t)(s2 * half_keys + h2 * 64);
+          tmem_ld32x2(lane_base + col, lane_base + col + 32u, va, vb);
           if (h2 == n_pairs_ch - 1) release_buffer();
           if (row_ok) {
-            const int j0 = key0 + kofs + h2 * 64;
+            const int j0 = key0 + h2 * 64;
             if (need_mask) {
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
@@ -497,9 +550,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         }
       }
       // End of pass 1: every warp writes its last partial; then one thread publishes the CTA's flag.
+      // The partial stores are ordered before the flag by the mbarrier (release/acquire within the CTA)
+      // followed by the publisher's GPU-scope fence and release store.
       if (ok) {
         if (cur >= 0) flush_partial(cur);
-        __threadfence();
         __syncwarp();
         if (lane == 0) mbar_arrive(p1_flushed);
         if (ew == 0 && lane == 0) {
@@ -522,24 +576,25 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       float* negoff = sNegOff + grp * kMaxRows;  // this group's per-row offsets and causal limits
       int* pw_tab = sPw + grp * kMaxRows;
       float* combf = sComb + grp * (2 * 128);     // rows output: [2 parity][128]
-      for (int k = n1; k < n_seq && ok; ++k) {
-        if ((k & 1) != grp) continue;
-        const int gt = tile_at(k);
+      for (int k = 0; k < n1 && ok; ++k, ++hh) {
+        if ((hh & 1u) != (uint32_t)grp) continue;
+        const int gt = t_hi - 1 - k;
         const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
         if (u != cur) {
           if (!others_done) {
-            // Wait until every CTA has published its pass-1 partials (and zeroed its share of t_acc),
-            // and until this CTA's pass-1 MMAs no longer read the stage that holds the pass-2 tables.
+            // Wait until every CTA has published its pass-1 partials (and zeroed its share of t_acc).
             if (leader) {
+              // Relaxed polls (the lanes' loads overlap), then one acquire fence once all flags match.
               bool all = false;
               const uint64_t t0 = globaltimer_ns();
               for (uint32_t it = 0; !all; ++it) {
                 bool mine = true;
-                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_acquire_u64(&p.flags[b]) == p.token;
+#pragma unroll 4
+                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.token;
                 all = __all_sync(0xffffffffu, mine);
                 if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) break;
               }
-              if (all) all = mbar_wait(p1_mma_done, 0, abort_flag);
+              fence_acquire_gpu();
               if (!all) {
                 *abort_flag = 1;
                 if (lane == 0) record_status(p.status, STEPKV_ETIMEOUT);
@@ -566,20 +621,20 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             for (int i0 = 0; i0 < n_ent; i0 += 8) {
               float2 pz[8];
 #pragma unroll
-              for (int t = 0; t < 8; ++t) {
-                const int i = i0 + t;
+              for (int t8 = 0; t8 < 8; ++t8) {
+                const int i = i0 + t8;
                 const int ci = c0 + i / n_e, e = i - (i / n_e) * n_e;
-                pz[t] = i < n_ent ? __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row])
-                                  : make_float2(-INFINITY, 0.f);
+                pz[t8] = i < n_ent ? __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row])
+                                   : make_float2(-INFINITY, 0.f);
               }
 #pragma unroll
-              for (int t = 0; t < 8; ++t) {
-                if (pz[t].x == -INFINITY) continue;
-                if (pz[t].x > M) {
-                  Zs = Zs * ex2_approx((M - pz[t].x) * c) + pz[t].y;
-                  M = pz[t].x;
+              for (int t8 = 0; t8 < 8; ++t8) {
+                if (pz[t8].x == -INFINITY) continue;
+                if (pz[t8].x > M) {
+                  Zs = Zs * ex2_approx((M - pz[t8].x) * c) + pz[t8].y;
+                  M = pz[t8].x;
                 } else {
-                  Zs += pz[t].y * ex2_approx((pz[t].x - M) * c);
+                  Zs += pz[t8].y * ex2_approx((pz[t8].x - M) * c);
                 }
               }
             }

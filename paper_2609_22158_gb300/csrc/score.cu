@@ -306,10 +306,6 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   // Every thread waits for the earlier kernels on the stream before its first global access.
   pdl_wait();
   pdl_launch_dependents();
-  if (p.zero_acc) {
-    for (int i = blockIdx.x * kThreads + threadIdx.x; i < g.T; i += gridDim.x * kThreads) p.t_acc[i] = 0ull;
-    __threadfence();  // ordered before this CTA's pass-1 flag, hence before any pass-2 addition
-  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -484,6 +480,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       if (lane == 0) mbar_arrive(&acc_empty[grp]);
     };
 
+    // The epilogue warps zero this CTA's share of t_acc while the first tiles stream in.  The stores
+    // precede the warp's p1_flushed arrival, so the publisher's fence orders them before the CTA's flag,
+    // hence before any pass-2 addition by any CTA.
+    if (p.zero_acc) {
+      for (int i = blockIdx.x * (kEpiWarps * 32) + (threadIdx.x - 64); i < g.T; i += gridDim.x * (kEpiWarps * 32))
+        p.t_acc[i] = 0ull;
+    }
+
     // ---- pass 1: per-row running (m, Z) over the keys this warp sees
     {
       int cur = -1;
@@ -614,29 +618,30 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           const bool valid = row < r.rows && w < g.W;
           float off = INFINITY;
           if (valid) {
-            // Online log-sum-exp over the unit's entries, in a fixed order; loads are issued eight at a
-            // time so their latencies overlap.
+            // Log-sum-exp over the unit's entries in a fixed order.  Up to 16 entries (every unit spans
+            // at most 8 CTAs for tile ranges of 32 or more) are loaded at once, so one L2 round trip
+            // serves them all; longer lists continue in batches of 16.
             const int n_ent = (c1 - c0 + 1) * n_e;
             float M = -INFINITY, Zs = 0.f;
-            for (int i0 = 0; i0 < n_ent; i0 += 8) {
-              float2 pz[8];
+            for (int i0 = 0; i0 < n_ent; i0 += 16) {
+              float2 pz[16];
 #pragma unroll
-              for (int t8 = 0; t8 < 8; ++t8) {
+              for (int t8 = 0; t8 < 16; ++t8) {
                 const int i = i0 + t8;
                 const int ci = c0 + i / n_e, e = i - (i / n_e) * n_e;
                 pz[t8] = i < n_ent ? __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row])
                                    : make_float2(-INFINITY, 0.f);
               }
+              float Mb = M;
 #pragma unroll
-              for (int t8 = 0; t8 < 8; ++t8) {
-                if (pz[t8].x == -INFINITY) continue;
-                if (pz[t8].x > M) {
-                  Zs = Zs * ex2_approx((M - pz[t8].x) * c) + pz[t8].y;
-                  M = pz[t8].x;
-                } else {
-                  Zs += pz[t8].y * ex2_approx((pz[t8].x - M) * c);
-                }
-              }
+              for (int t8 = 0; t8 < 16; ++t8) Mb = fmaxf(Mb, pz[t8].x);
+              if (Mb == -INFINITY) continue;
+              float Zb = M == -INFINITY ? 0.f : Zs * ex2_approx((M - Mb) * c);
+#pragma unroll
+              for (int t8 = 0; t8 < 16; ++t8)
+                Zb += pz[t8].x == -INFINITY ? 0.f : pz[t8].y * ex2_approx((pz[t8].x - Mb) * c);
+              M = Mb;
+              Zs = Zb;
             }
             off = M * c + __log2f(Zs);
           }

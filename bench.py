@@ -459,8 +459,15 @@ def main():
     ap.add_argument("--ref-pairs", type=int, default=2)
     ap.add_argument("--ref-compact-sets", type=int, default=4)
     ap.add_argument("--compact-traffic", type=float, default=None,
-                    help="dram bytes (read+write) per compaction launch from an ncu capture of this workload")
+                    help="dram bytes (read+write) per compaction launch from an ncu capture of this workload "
+                         "(default: the capture of the current compaction kernel for the 32-layer 32K workload)")
     args = ap.parse_args()
+    if args.compact_traffic is None and args.T == 32768 and args.layers == 32:
+        # dram__bytes_read.sum + dram__bytes_write.sum of compact_kernel from one ncu capture of the
+        # 8-layer variant of this workload (109.78 MB read + 59.16 MB written), scaled by row sets (x4):
+        # the kernel does the same work per row set.  Writes below the algorithmic bytes are dirty lines
+        # still in L2 when the kernel ends.
+        args.compact_traffic = 4 * (109.782528e6 + 59.157760e6)
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -427,8 +427,20 @@ class Problem:
     step_id_out: object = None
     pos_out: object = None
     _keep: list = field(default_factory=list, repr=False)
+    _c: object = field(default=None, repr=False)
 
     def c(self) -> CProblem:
+        """The C struct, validated and built on first use and reused afterwards (building it checks
+        every per-layer tensor, which costs more host time than the pass itself takes on the GPU).
+        Call refresh() after replacing or reshaping any tensor of the problem."""
+        if self._c is None:
+            self._c = self._build()
+        return self._c
+
+    def refresh(self):
+        self._c = None
+
+    def _build(self) -> CProblem:
         torch = _torch()
         L = len(self.K)
         Ls = len(self.Q)

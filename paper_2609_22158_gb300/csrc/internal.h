@@ -20,11 +20,12 @@ void set_last_cuda_error(cudaError_t e);
 cudaError_t device_sm_count(int* n);
 cudaError_t ensure_smem_attr(const void* func, int bytes);
 
-// Kernel launch on `stream` (ordinary stream order).  Programmatic dependent launch is deliberately not
-// used: measured on GB300, the compaction kernel ran ~25% slower when launched with the programmatic
-// serialization attribute (178 us vs 140 us for the 32K workload) and the overlap gained elsewhere was
-// smaller than that loss.  The kernels still execute griddepcontrol.wait / launch_dependents, which
-// are no-ops for ordinary launches, so enabling the attribute stays a one-line change.
+// Kernel launch on `stream`.  Ordinary stream order unless `pdl` is set: then the launch carries the
+// programmatic-stream-serialization attribute, so the kernel may start while the preceding kernel
+// finishes and must execute griddepcontrol.wait (pdl_wait) before reading anything that kernel wrote.
+// Only the selection kernel uses it.  Measured on GB300 with the 32K workload, the compaction kernel
+// ran ~25% slower when launched with the attribute (178 us vs 140 us), so it is launched plainly.
+// Every kernel executes griddepcontrol.launch_dependents, a no-op when the next launch is ordinary.
 template <typename... KArgs, typename... Args>
 cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
                           Args&&... args) {
@@ -39,9 +40,9 @@ cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t 
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
-template <typename... KArgs, typename... Args>
-cudaError_t launch_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cluster_x, size_t smem,
-                           cudaStream_t stream, Args&&... args) {
+template <typename... KArgs, typename A0>
+cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream, A0&& a0,
+                          bool pdl) {
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
   cfg.gridDim = grid;
@@ -49,13 +50,32 @@ cudaError_t launch_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cl
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<A0>(a0));
+}
+
+template <typename... KArgs, typename A0>
+cudaError_t launch_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cluster_x, size_t smem,
+                           cudaStream_t stream, A0&& a0, bool pdl = false) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = cluster_x;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<A0>(a0));
 }
 
 // ---- score (score.cu)

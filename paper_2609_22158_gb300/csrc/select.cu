@@ -197,7 +197,9 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
   const int len = max(0, min(a.chunk, T - base));
   const bool s_in_smem = a.s_in_smem != 0;
 
-  pdl_wait();  // every global read below may depend on an earlier kernel on the stream
+  // Launched with programmatic dependent launch: everything up to pdl_wait() reads only the call's
+  // inputs (step signals, step ids, mask) and writes only this kernel's workspace and outputs, so it
+  // may overlap the tail of the kernel that produces the token saliency.
   pdl_launch_dependents();
 
   // ---- Phase 1+2 of Algorithm 1 (Eqs. 2-4).  With few steps every CTA keeps all S_k in shared memory
@@ -229,20 +231,44 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
     a.acc_kept[k] = 0;
   }
 
-  // ---- this CTA's tokens: step ids / protection flags and token saliency T_i (loads batched)
+  // ---- this CTA's tokens: step ids / protection flags (inputs), then, once the producing kernel has
+  // finished, token saliency T_i (loads batched)
   float lmax = -INFINITY;
   int lN = 0, lerr = 0;
   for (int i0 = 0; i0 < len; i0 += NT * UNROLL) {
-    float tv[UNROLL];
     uint8_t pv[UNROLL];
     int sv[UNROLL];
 #pragma unroll
     for (int u = 0; u < UNROLL; ++u) {
       const int i = i0 + u * NT + tid;
       if (i < len) {
+        pv[u] = __ldg(&a.prot[base + i]);
+        sv[u] = __ldg(&a.step_id[base + i]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      const int i = i0 + u * NT + tid;
+      if (i < len) {
+        if (!pv[u]) {
+          ++lN;
+          const bool bad = sv[u] < 0 || sv[u] >= n_steps;
+          if (bad) lerr = 1;
+          sSid[i] = bad ? 0 : (uint16_t)sv[u];
+        } else {
+          sSid[i] = 0xFFFFu;
+        }
+      }
+    }
+  }
+  pdl_wait();  // t_acc / T_in come from the preceding kernel
+  for (int i0 = 0; i0 < len; i0 += NT * UNROLL) {
+    float tv[UNROLL];
+#pragma unroll
+    for (int u = 0; u < UNROLL; ++u) {
+      const int i = i0 + u * NT + tid;
+      if (i < len) {
         const int gi = base + i;
-        pv[u] = __ldg(&a.prot[gi]);
-        sv[u] = __ldg(&a.step_id[gi]);
         tv[u] = a.t_acc ? __ull2float_rn(__ldcg(&a.t_acc[gi])) * a.acc_to_T : __ldcg(&a.T_in[gi]);
       }
     }
@@ -251,15 +277,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
       const int i = i0 + u * NT + tid;
       if (i < len) {
         sT[i] = tv[u];
-        if (!pv[u]) {
-          ++lN;
-          lmax = fmaxf(lmax, tv[u]);
-          const bool bad = sv[u] < 0 || sv[u] >= n_steps;
-          if (bad) lerr = 1;
-          sSid[i] = bad ? 0 : (uint16_t)sv[u];
-        } else {
-          sSid[i] = 0xFFFFu;
-        }
+        if (sSid[i] != 0xFFFFu) lmax = fmaxf(lmax, tv[u]);  // this thread wrote sSid[i] above
       }
     }
   }
@@ -615,12 +633,12 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
   if (nc == 1) {
     void (*kern)(SelectArgs) = select_kernel<1, 1024>;
     e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
-    if (e == cudaSuccess) e = launch_kernel(kern, dim3(1), dim3(1024), smem, stream, a);
+    if (e == cudaSuccess) e = launch_kernel(kern, dim3(1), dim3(1024), smem, stream, a, true);
   } else {
     void (*kern)(SelectArgs) = select_kernel<kSelClusterCtas, 512>;
     e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
     if (e == cudaSuccess)
-      e = launch_cluster(kern, dim3(kSelClusterCtas), dim3(512), kSelClusterCtas, smem, stream, a);
+      e = launch_cluster(kern, dim3(kSelClusterCtas), dim3(512), kSelClusterCtas, smem, stream, a, true);
   }
   if (e != cudaSuccess) {
     set_last_cuda_error(e);

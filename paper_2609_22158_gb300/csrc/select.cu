@@ -140,6 +140,37 @@ __device__ __forceinline__ void step_stat_add(bool act, int sid, unsigned long l
   }
 }
 
+// Warp-wide flush of per-lane step statistics (lane: `act`, its step `sid`, count, fixed-point sum,
+// max bits): one set of atomics per warp when every active lane holds the same step, else one per
+// lane.  Integer atomics only, so the totals do not depend on the order of arrival.
+__device__ __forceinline__ void step_stat_flush(bool act, int sid, int cnt_v, unsigned long long sum_v,
+                                                uint32_t max_v, int32_t* cnt, unsigned long long* sum,
+                                                uint32_t* mx) {
+  const unsigned am = __ballot_sync(0xffffffffu, act);
+  if (!am) return;
+  const int lane = threadIdx.x & 31;
+  const int sid0 = __shfl_sync(0xffffffffu, sid, __ffs(am) - 1);
+  if (__all_sync(0xffffffffu, !act || sid == sid0)) {
+    int c = act ? cnt_v : 0;
+    unsigned long long v = act ? sum_v : 0ull;
+    uint32_t m = act ? max_v : 0u;
+    for (int o = 16; o > 0; o >>= 1) {
+      c += __shfl_xor_sync(0xffffffffu, c, o);
+      if (sum) v += __shfl_xor_sync(0xffffffffu, v, o);
+      if (mx) m = max(m, __shfl_xor_sync(0xffffffffu, m, o));
+    }
+    if (lane == 0) {
+      atomicAdd(&cnt[sid0], c);
+      if (sum) atomicAdd(&sum[sid0], v);
+      if (mx) atomicMax(&mx[sid0], m);
+    }
+  } else if (act) {
+    atomicAdd(&cnt[sid], cnt_v);
+    if (sum) atomicAdd(&sum[sid], sum_v);
+    if (mx) atomicMax(&mx[sid], max_v);
+  }
+}
+
 __device__ __forceinline__ float step_utility(const SelectArgs& a, int k, int t_last, float* c_out) {
   const stepkv_params_t& p = a.prm;
   const float r = a.steps.valid[k] + a.steps.gain[k] - p.lambda * a.steps.red[k];  // Eq. 2
@@ -282,10 +313,29 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
     }
   }
   {
-    const float bm = block_reduce_max<NT>(lmax, reinterpret_cast<float*>(scratch));
-    const int bn = block_reduce_sum_int<NT>(lN, scratch);
-    const int be = block_reduce_sum_int<NT>(lerr, scratch);
+    // one block reduction for (max T, prunable count, error flag); the histogram area is free here
+    for (int o = 16; o > 0; o >>= 1) {
+      lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, o));
+      lN += __shfl_xor_sync(0xffffffffu, lN, o);
+      lerr |= __shfl_xor_sync(0xffffffffu, lerr, o);
+    }
+    float* red_max = reinterpret_cast<float*>(hist);
+    int* red_n = hist + NW;
+    int* red_e = hist + 2 * NW;
+    if (lane == 0) {
+      red_max[warp] = lmax;
+      red_n[warp] = lN;
+      red_e[warp] = lerr;
+    }
+    __syncthreads();
     if (tid == 0) {
+      float bm = -INFINITY;
+      int bn = 0, be = 0;
+      for (int w = 0; w < NW; ++w) {
+        bm = fmaxf(bm, red_max[w]);
+        bn += red_n[w];
+        be |= red_e[w];
+      }
       ex->loc_max = bm;
       ex->loc_N = bn;
       ex->loc_err = be;
@@ -341,29 +391,51 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
   const int fx_shift = min(62 - log2N - e_max, 126);  // every partial sum < 2^62
   const float* Sk = s_in_smem ? sS : a.S;
 
-  // ---- priorities (Eq. 5), ordered keys and per-step statistics.  The loop bound is uniform per warp
-  // (warp-aggregated atomics); T_hat is read before its shared-memory slot is overwritten by the key.
-  for (int i0 = 0; i0 < len; i0 += NT) {
-    const int i = i0 + tid;
-    const bool in = i < len;
-    const int gi = base + i;
-    const float th = in ? sT[i] * inv_max : 0.f;
-    const int sid = in ? sSid[i] : 0xFFFF;
-    const bool act = sid != 0xFFFF;
-    if (in) {
+  // Warp w owns the consecutive slots [w*seg, (w+1)*seg) of this CTA in the passes that need slot order
+  // or per-step runs (keys and statistics, counts, ordered write); lanes take consecutive slots.
+  const int seg = ((len + NW - 1) / NW + 31) & ~31;
+  const int s0 = min(len, warp * seg), s1 = min(len, s0 + seg);
+
+  // ---- priorities (Eq. 5), ordered keys and per-step statistics.  A lane accumulates its tokens'
+  // statistics while their step does not change (slots of a step are mostly contiguous) and flushes
+  // with integer atomics; T_hat is read before its shared-memory slot is overwritten by the key.
+  {
+    int run_sid = -1, run_c = 0;
+    unsigned long long run_s = 0ull;
+    uint32_t run_m = 0u;
+    for (int i0 = s0; i0 < s1; i0 += 32) {
+      const int i = i0 + lane;
+      if (i >= s1) break;
+      const int gi = base + i;
+      const float th = sT[i] * inv_max;
+      const int sid = sSid[i];
       uint32_t key = 0u;
-      if (act) {
+      if (sid != 0xFFFF) {
         const float P = fmaf(a.prm.alpha, th, a.prm.beta * Sk[sid]);
         key = float_to_ordered(P);
         if (a.out.priority) a.out.priority[gi] = P;
+        const float thc = fmaxf(th, 0.f);
+        if (sid != run_sid) {
+          if (run_c) {
+            atomicAdd(&a.acc_cnt[run_sid], run_c);
+            atomicAdd(&a.acc_sum[run_sid], run_s);
+            atomicMax(&a.acc_max[run_sid], run_m);
+          }
+          run_sid = sid;
+          run_c = 0;
+          run_s = 0ull;
+          run_m = 0u;
+        }
+        ++run_c;
+        run_s += to_fixed(thc, fx_shift);
+        run_m = max(run_m, __float_as_uint(thc));
       } else if (a.out.priority) {
         a.out.priority[gi] = -INFINITY;
       }
       if (a.out.token_sal) a.out.token_sal[gi] = th;
       sKey[i] = key;
     }
-    const float thc = fmaxf(th, 0.f);
-    step_stat_add(act, sid, to_fixed(thc, fx_shift), __float_as_uint(thc), a.acc_cnt, a.acc_sum, a.acc_max);
+    step_stat_flush(run_c > 0, run_sid, run_c, run_s, run_m, a.acc_cnt, a.acc_sum, a.acc_max);
   }
   __syncthreads();
 
@@ -453,20 +525,38 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
   }
   // B == N: kth = 0 keeps every prunable token (all prunable keys are > 0)
 
-  // ---- per-CTA counts: protected + strictly greater, ties at the threshold
-  {
-    int kb = 0, eq = 0;
-    for (int i = tid; i < len; i += NT) {
-      if (sSid[i] == 0xFFFF) ++kb;
-      else if (sKey[i] > kth) ++kb;
-      else if (sKey[i] == kth) ++eq;
+  // ---- counts per warp segment: kept for sure (protected or strictly above the threshold) and ties
+  int strict_w = 0, eq_w = 0;  // warp-uniform
+  for (int i0 = s0; i0 < s1; i0 += 32) {
+    const int i = i0 + lane;
+    const bool in = i < s1;
+    const uint32_t k = in ? sKey[i] : 0u;
+    const bool pr = in && sSid[i] == 0xFFFF;
+    strict_w += __popc(__ballot_sync(0xffffffffu, in && (pr || k > kth)));
+    eq_w += __popc(__ballot_sync(0xffffffffu, in && !pr && k == kth));
+  }
+  // [NW] each, in the second radix pass's histogram buffer (hist + 2048): peers may still be reading the
+  // last pass's buffer (hist[0..]) through DSMEM until barrier (B), but every CTA is done with this one
+  int* seg_strict = hist + 2048;
+  int* seg_eq = hist + 2048 + NW;
+  if (lane == 0) {
+    seg_strict[warp] = strict_w;
+    seg_eq[warp] = eq_w;
+  }
+  __syncthreads();
+  int strict_before = 0, eq_before = 0, strict_cta = 0, eq_cta = 0;  // exclusive prefixes over warps
+  for (int w = 0; w < NW; ++w) {
+    const int sw = seg_strict[w], ew = seg_eq[w];
+    if (w < warp) {
+      strict_before += sw;
+      eq_before += ew;
     }
-    const int bkb = block_reduce_sum_int<NT>(kb, scratch);
-    const int beq = block_reduce_sum_int<NT>(eq, scratch);
-    if (tid == 0) {
-      ex->loc_keep_base = bkb;
-      ex->loc_eq = beq;
-    }
+    strict_cta += sw;
+    eq_cta += ew;
+  }
+  if (tid == 0) {
+    ex->loc_keep_base = strict_cta;
+    ex->loc_eq = eq_cta;
   }
   cl.sync();  // (B)
   if (tid < NC) {
@@ -478,7 +568,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
   __syncthreads();
   // offsets: CTA r keeps its protected + strictly-greater tokens and the ties that fall within the
   // first need_eq ties in slot order
-  int out_off = 0, total_kept = 0, ties_before = 0, eq_cum = 0;
+  int out_off = 0, total_kept = 0, ties_before = 0, eq_cum = 0, granted_cta = 0;
   for (int r = 0; r < NC; ++r) {
     const int granted = max(0, min(need_eq - eq_cum, all[r].loc_eq));
     const int kept_r = all[r].loc_keep_base + granted;
@@ -486,6 +576,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
       out_off += kept_r;
       ties_before += all[r].loc_eq;
     }
+    if (r == rank) granted_cta = granted;
     total_kept += kept_r;
     eq_cum += all[r].loc_eq;
   }
@@ -496,49 +587,36 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
     if (overflow) record_status(a.status, STEPKV_ENOSPACE);
   }
 
-  // ---- ordered write of the retained slots.  Token i of round r = i / NT is handled by thread i % NT;
-  // each warp records per-round tie and keep counts, block-wide prefix passes order them.
+  // ---- ordered write of the retained slots: a warp walks its segment in slot order with running
+  // counts (ballot + popc), starting from its segment's prefix within the CTA and the cluster.
   if (!overflow) {
-    const int n_rounds = (len + NT - 1) / NT;
-    int* cnt_eq = hist;                           // [rounds][warps] (the histograms are no longer read)
-    int* cnt_keep = cnt_eq + n_rounds * NW;       // [rounds][warps]
-    for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * NT + tid;
-      const bool is_eq = i < len && sSid[i] != 0xFFFF && sKey[i] == kth;
-      const unsigned m = __ballot_sync(0xffffffffu, is_eq);
-      if (lane == 0) cnt_eq[r * NW + warp] = __popc(m);
-    }
-    __syncthreads();
-    block_scan_array<NT>(cnt_eq, n_rounds * NW, ties_before, scratch);
-    for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * NT + tid;
-      const bool in = i < len;
-      const uint32_t k = in ? sKey[i] : 0u;
-      const bool pr = in && sSid[i] == 0xFFFF;
-      const bool is_eq = in && !pr && k == kth;
-      const unsigned em = __ballot_sync(0xffffffffu, is_eq);
-      const int eq_rank = cnt_eq[r * NW + warp] + __popc(em & ((1u << lane) - 1u));
-      const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
-      const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (lane == 0) cnt_keep[r * NW + warp] = __popc(km);
-    }
-    __syncthreads();
-    block_scan_array<NT>(cnt_keep, n_rounds * NW, out_off, scratch);
-    for (int r = 0; r < n_rounds; ++r) {
-      const int i = r * NT + tid;
-      const bool in = i < len;
+    int tie_rank = ties_before + eq_before;                                 // cluster-wide tie rank
+    int out_pos = out_off + strict_before + min(granted_cta, eq_before);   // next output slot
+    int run_sid = -1, run_c = 0;
+    for (int i0 = s0; i0 < s1; i0 += 32) {
+      const int i = i0 + lane;
+      const bool in = i < s1;
       const uint32_t k = in ? sKey[i] : 0u;
       const int sid = in ? sSid[i] : 0xFFFF;
       const bool pr = in && sid == 0xFFFF;
       const bool is_eq = in && !pr && k == kth;
+      const unsigned lt = (1u << lane) - 1u;
       const unsigned em = __ballot_sync(0xffffffffu, is_eq);
-      const int eq_rank = cnt_eq[r * NW + warp] + __popc(em & ((1u << lane) - 1u));
-      const bool keep = in && (pr || k > kth || (is_eq && eq_rank < need_eq));
+      const bool keep = in && (pr || k > kth || (is_eq && tie_rank + __popc(em & lt) < need_eq));
       const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (keep) a.out.kept_idx[cnt_keep[r * NW + warp] + __popc(km & ((1u << lane) - 1u))] = base + i;
-      const bool kept_prunable = keep && !pr;
-      step_stat_add(kept_prunable, sid, 0ull, 0u, a.acc_kept, nullptr, nullptr);
+      if (keep) a.out.kept_idx[out_pos + __popc(km & lt)] = base + i;
+      out_pos += __popc(km);
+      tie_rank += __popc(em);
+      if (keep && !pr) {
+        if (sid != run_sid) {
+          if (run_c) atomicAdd(&a.acc_kept[run_sid], run_c);
+          run_sid = sid;
+          run_c = 0;
+        }
+        ++run_c;
+      }
     }
+    step_stat_flush(run_c > 0, run_sid, run_c, 0ull, 0u, a.acc_kept, nullptr, nullptr);
   }
   cl.sync();  // (C) all step accumulators final
 

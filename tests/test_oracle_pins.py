@@ -296,6 +296,100 @@ def test_priority_range_and_sharing():
     assert abs((P[i] - P[j]) - p.alpha * (T_hat[i] - T_hat[j])) < 1e-12
 
 
+# ------------------------------------------------------------------ decode attention (S6)
+def check_decode_single_key(O):
+    # one cached key: the softmax weight is 1 and the output is that key's value row, exactly
+    rng = np.random.default_rng(7)
+    q = _bits(rng.standard_normal((4, 16)))
+    K = _bits(rng.standard_normal((2, 1, 16)))
+    V = _bits(rng.standard_normal((2, 1, 16)))
+    out = O.decode_attention(q, K, V)
+    Vf = O.bf16_to_f64(V)
+    for g in range(4):
+        assert np.array_equal(out[g], Vf[g // 2, 0])
+
+
+def check_decode_identical_keys(O):
+    # equal keys: uniform weights, the output is the mean of the value rows
+    rng = np.random.default_rng(8)
+    k = rng.standard_normal(32)
+    K = _bits(np.tile(k, (1, 9, 1)))
+    V = _bits(rng.standard_normal((1, 9, 32)))
+    q = _bits(rng.standard_normal((3, 32)))
+    out = O.decode_attention(q, K, V)
+    mean = O.bf16_to_f64(V)[0].mean(axis=0)
+    assert np.allclose(out, np.tile(mean, (3, 1)), rtol=0, atol=1e-12)
+
+
+def check_decode_two_key_analytic(O):
+    # two keys: the first weight is the logistic function of the scaled logit difference
+    d = 16
+    q = np.zeros((1, d), np.float32)
+    q[0, 0] = 2.0
+    K = np.zeros((1, 2, d), np.float32)
+    K[0, 0, 0] = 1.5
+    K[0, 1, 0] = -0.5
+    V = np.zeros((1, 2, d), np.float32)
+    V[0, 0, 3] = 1.0
+    V[0, 1, 5] = 1.0
+    out = O.decode_attention(_bits(q), _bits(K), _bits(V))
+    w0 = expit((2.0 * 1.5 - 2.0 * -0.5) / math.sqrt(d))
+    assert abs(out[0, 3] - w0) < 1e-12 and abs(out[0, 5] - (1 - w0)) < 1e-12
+    assert abs(out[0].sum() - 1.0) < 1e-12
+
+
+def check_decode_gqa(O):
+    # query head g reads KV head g // G: value rows are constant per KV head
+    d, n = 8, 5
+    rng = np.random.default_rng(9)
+    q = _bits(rng.standard_normal((6, d)))
+    K = _bits(rng.standard_normal((3, n, d)))
+    V = np.stack([np.full((n, d), 1.0 + h, np.float32) for h in range(3)])
+    out = O.decode_attention(q, K, _bits(V))
+    for g in range(6):
+        assert np.allclose(out[g], 1.0 + g // 2, rtol=0, atol=1e-12)
+
+
+def check_decode_bruteforce(O):
+    # element-by-element restatement with math.exp on a tiny case
+    rng = np.random.default_rng(10)
+    Hq, Hkv, n, d = 4, 2, 6, 4
+    q = _bits(rng.standard_normal((Hq, d)))
+    K = _bits(rng.standard_normal((Hkv, n, d)))
+    V = _bits(rng.standard_normal((Hkv, n, d)))
+    qf, Kf, Vf = (O.bf16_to_f64(x) for x in (q, K, V))
+    out = O.decode_attention(q, K, V)
+    for g in range(Hq):
+        h = g * Hkv // Hq
+        logits = [sum(qf[g][t] * Kf[h][j][t] for t in range(d)) / math.sqrt(d) for j in range(n)]
+        mx = max(logits)
+        w = [math.exp(x - mx) for x in logits]
+        z = sum(w)
+        for t in range(d):
+            ref = sum(w[j] / z * Vf[h][j][t] for j in range(n))
+            assert abs(out[g][t] - ref) < 1e-12
+
+
+def test_decode_single_key():
+    check_decode_single_key(REAL)
+
+
+def test_decode_identical_keys():
+    check_decode_identical_keys(REAL)
+
+
+def test_decode_two_key_analytic():
+    check_decode_two_key_analytic(REAL)
+
+
+def test_decode_gqa():
+    check_decode_gqa(REAL)
+
+
+def test_decode_bruteforce():
+    check_decode_bruteforce(REAL)
+
+
 # ------------------------------------------------------------------ end-to-end invariants
 def test_boundary_invariants_tiny():
     tr = wl.tiny(0)
@@ -416,6 +510,37 @@ def _budget_no_floor_one(N, mode, num=1, den=1, count=0):
     return min((num * N) // den if mode == "ratio" else count, N)
 
 
+def _decode_interleaved(q, K, V):
+    # wrong GQA convention: q head g reads KV head g % Hkv
+    Hkv = K.shape[0]
+    Hq = q.shape[0]
+    G = Hq // Hkv
+    inv = np.array([(g % Hkv) * G + g // Hkv for g in range(Hq)])
+    out = REAL.decode_attention(q[np.argsort(inv)], K, V)
+    return out[inv]
+
+
+def _decode_no_scale(q, K, V):
+    qf, Kf, Vf = REAL.bf16_to_f64(q), REAL.bf16_to_f64(K), REAL.bf16_to_f64(V)
+    Hq, d = qf.shape
+    G = Hq // Kf.shape[0]
+    out = np.zeros((Hq, d))
+    for g in range(Hq):
+        out[g] = softmax(Kf[g // G] @ qf[g]) @ Vf[g // G]
+    return out
+
+
+def _decode_unnormalised(q, K, V):
+    qf, Kf, Vf = REAL.bf16_to_f64(q), REAL.bf16_to_f64(K), REAL.bf16_to_f64(V)
+    Hq, d = qf.shape
+    G = Hq // Kf.shape[0]
+    out = np.zeros((Hq, d))
+    for g in range(Hq):
+        s = Kf[g // G] @ qf[g] / math.sqrt(d)
+        out[g] = np.exp(s - s.max()) @ Vf[g // G]
+    return out
+
+
 @pytest.mark.parametrize("check, mutant", [
     (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
     (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
@@ -427,6 +552,10 @@ def _budget_no_floor_one(N, mode, num=1, den=1, count=0):
     (check_step_utility_table, _mutant(completion_score=_completion_wrong_sign)),
     (check_select_bruteforce, _mutant(select_top=_select_newer_wins)),
     (check_budget, _mutant(budget_tokens=_budget_no_floor_one)),
+    (check_decode_gqa, _mutant(decode_attention=_decode_interleaved)),
+    (check_decode_two_key_analytic, _mutant(decode_attention=_decode_no_scale)),
+    (check_decode_identical_keys, _mutant(decode_attention=_decode_unnormalised)),
+    (check_decode_bruteforce, _mutant(decode_attention=_decode_no_scale)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

@@ -258,6 +258,32 @@ STEPKV_API stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K
                                int32_t* dev_status, void* stream);
 
 /* ---------------------------------------------------------------------------------------------
+ * Decode attention over a compacted cache: the reads an agent makes after a boundary, each new
+ * token attending to the retained rows C_hat = C_prot || C_traj[K] (Eq. 1).  One query token per
+ * layer; GQA as above (query head g reads KV head g / G).
+ *
+ * For every layer l < n_layers and query head g < Hq:
+ *   out[l][g][:] = sum_{j < n} softmax_j( q[l][g] . K[l][g/G][j] / sqrt(d) ) V[l][g/G][j][:]
+ *  q[l]     host array of device pointers, [Hq][d] bf16.
+ *  K[l], V[l] host arrays of device pointers, [Hkv][rows >= n_cap][d] bf16, head stride
+ *           kv_head_stride elements (% 8 == 0); bases 16-byte aligned.
+ *  n        keys per head: *n_dev when n_dev is not NULL (read on the device, e.g. the n_kept of a
+ *           compaction), else n_host.  A device value above n_cap sets STEPKV_ENOSPACE and n_cap rows
+ *           are used; a value below 1 sets STEPKV_EDATA and the output is zero.
+ *  out[l]   host array of device pointers, [Hq][d] fp32.
+ *  ws       scratch of stepkv_decode_workspace_size bytes (256-byte aligned): per-split partials.
+ *  Supported: d in {64, 128}; G = Hq / Hkv in {1, 2, 4, 5, 8}; 1 <= n_cap; n_host <= n_cap.
+ *  Work: split-K over 512-key chunks (one chunk of one (layer, KV head) per CTA, all G heads of the
+ *  group per key-row load), then a merge of the chunks in order (deterministic).
+ */
+STEPKV_API size_t stepkv_decode_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t d, int32_t n_cap);
+STEPKV_API stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q, const void* const* K,
+                              const void* const* V, int64_t kv_head_stride, int32_t Hkv, int32_t Hq,
+                              int32_t d, const int32_t* n_dev, int32_t n_host, int32_t n_cap,
+                              float* const* out, void* ws, size_t ws_bytes, int32_t* dev_status,
+                              void* stream);
+
+/* ---------------------------------------------------------------------------------------------
  * The fused pass (score -> reduce/fuse -> select -> compact) for n_traj independent trajectories
  * (one pruning boundary each, Algorithm 1).  probs is a host array; all trajectories run on
  * `stream` in order, sharing `ws` (size from stepkv_compress_workspace_size over the same array).

@@ -6,5 +6,5 @@ library; the first call does, and raises if the library has not been built.
 """
 from .binding import (  # noqa: F401
     StepKVError, Params, default_params, load_library, stepkv_score, stepkv_select, stepkv_compact,
-    stepkv_compress, stepkv_workspace_size, status_string, stepkv_select_static_scratch,
+    stepkv_compress, stepkv_workspace_size, status_string, stepkv_select_static_scratch, stepkv_decode,
 )

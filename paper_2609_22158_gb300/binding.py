@@ -82,6 +82,9 @@ SIGNATURES = {
                                             ctypes.POINTER(CSelOut), _VP, _VP]),
     "stepkv_compact": (_I32, [_I32, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _VP, _I32, _VP, _VP, _I64, _VP, _VP,
                               _VP, _VP, _VP, _VP]),
+    "stepkv_decode_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
+    "stepkv_decode": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _SZ, _VP,
+                             _VP]),
     "stepkv_compress_workspace_size": (_SZ, [ctypes.POINTER(CProblem), _I32]),
     "stepkv_compress": (_I32, [ctypes.POINTER(CProblem), _I32, ctypes.POINTER(CParams), _VP, _SZ, _VP, _VP]),
 }
@@ -343,6 +346,47 @@ def stepkv_select(sal, step_id, prot, steps: StepSignals, params: Params, budget
                              ctypes.byref(cp), ctypes.byref(budget), ctypes.byref(co), wp, wn, status.data_ptr(),
                              _stream_handle(stream))
     _check(code, "stepkv_select")
+    return out
+
+
+# ----------------------------------------------------------------------------- decode attention
+def stepkv_decode(q: Sequence, K: Sequence, V: Sequence, n, out: Optional[Sequence] = None, ws=None, status=None,
+                  stream=None):
+    """One query token per layer over a (compacted) cache: out[l][g] = softmax(q[l][g] K^T / sqrt(d)) V.
+
+    q[l]: [Hq, d] bf16; K[l], V[l]: [Hkv, rows, d] bf16 (rows >= n); n: an int, or a device int32 tensor
+    (e.g. the n_kept of a compaction) read on the device.  Returns the list of [Hq, d] fp32 outputs."""
+    torch = _torch()
+    lib = load_library()
+    L = len(q)
+    if L < 1 or len(K) != L or len(V) != L:
+        raise ValueError("q, K and V need one tensor per layer")
+    hs = _rows_layout(list(K) + list(V), "K/V")
+    Hkv, rows, d = K[0].shape
+    for i, t in enumerate(q):
+        _need(t, torch.bfloat16, f"q[{i}]", 2)
+        if not t.is_contiguous():
+            raise ValueError(f"q[{i}] must be contiguous")
+    Hq = q[0].shape[0]
+    dev = q[0].device
+    if out is None:
+        out = [torch.empty((Hq, d), dtype=torch.float32, device=dev) for _ in range(L)]
+    for i, t in enumerate(out):
+        _need(t, torch.float32, f"out[{i}]", 2)
+    if isinstance(n, int):
+        n_dev, n_host = None, n
+    else:
+        _need(n, torch.int32, "n")
+        n_dev, n_host = n, 0
+    need = lib.stepkv_decode_workspace_size(L, Hkv, Hq, d, rows)
+    ws = _workspace(need + 256, ws, dev)
+    wp, wn = _aligned_ws(ws)
+    status = status if status is not None else new_status(dev)
+    arrs = [_ptr_array(q), _ptr_array(K), _ptr_array(V), _ptr_array(out)]
+    cv = lambda a: ctypes.cast(a, ctypes.c_void_p)
+    code = lib.stepkv_decode(L, cv(arrs[0]), cv(arrs[1]), cv(arrs[2]), hs, Hkv, Hq, d, _ptr(n_dev), n_host, rows,
+                             cv(arrs[3]), wp, wn, status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_decode")
     return out
 
 

@@ -1,0 +1,296 @@
+// Decode attention over the compacted cache: after a compression boundary the agent keeps decoding,
+// and every new token attends to the retained rows C_hat = C_prot || C_traj[K] (Eq. 1).  For each
+// layer and query head g (KV head g / G):
+//   out[g][:] = sum_{j < n} softmax_j( q[g] . K[g/G][j] / sqrt(d) ) V[g/G][j][:]
+//
+// GB300 design: HBM-bound (the K and V rows are read once per token, 1.08 GB for 32 layers x 8 heads x
+// 8272 rows), so the kernel is built around coalesced 16-byte loads and enough bytes in flight; the
+// contraction is 2 x G x d flop per key row and stays on the FP32 pipe.  Split-K: a CTA owns 512 keys of
+// one (layer, KV head) pair and all G query heads of its group, so every key row is loaded once for the
+// whole group.  d/8 lanes share a key row (8 bf16 each); a warp covers 32/(d/8) keys per step, four steps
+// per block, and keeps a running (max, sum, weighted values) per head, rescaled once per block.  A
+// second kernel merges the per-split partials of each (pair, head) in split order (deterministic).
+// The number of keys may be read on the device (n_kept of a compaction), so no host sync is needed.
+#include <math.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace stepkv {
+
+constexpr int kDecThreads = 128;
+constexpr int kDecWarps = kDecThreads / 32;
+constexpr int kDecSplitKeys = 512;
+constexpr int kDecBlockSteps = 4;
+
+struct DecodeArgs {
+  const uint16_t* q[kMaxDecodeLayers];
+  const uint16_t* K[kMaxDecodeLayers];
+  const uint16_t* V[kMaxDecodeLayers];
+  float* out[kMaxDecodeLayers];
+  int64_t head_stride;  // elements
+  int Hkv;
+  int n_splits;
+  const int32_t* n_dev;
+  int n_host;
+  int n_cap;
+  float c;              // log2(e) / sqrt(d)
+  float* part;          // [pairs][n_splits][G][d + 4]: m, l, -, -, acc[d]
+  int32_t* status;
+};
+
+__device__ __forceinline__ int decode_n(const DecodeArgs& a) {
+  const int n = a.n_dev ? *a.n_dev : a.n_host;
+  return n;
+}
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& r, float (&f)[8]) {
+  const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+  }
+}
+
+// Merge the state (m2, l2, acc2) into (m, l, acc); -inf marks an empty state.
+template <int E>
+__device__ __forceinline__ void merge_state(float& m, float& l, float (&acc)[E], float m2, float l2,
+                                            const float (&acc2)[E]) {
+  const float mn = fmaxf(m, m2);
+  if (mn == -INFINITY) return;
+  const float a = ex2_approx(m - mn), b = ex2_approx(m2 - mn);
+  l = l * a + l2 * b;
+#pragma unroll
+  for (int e = 0; e < E; ++e) acc[e] = acc[e] * a + acc2[e] * b;
+  m = mn;
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __grid_constant__ DecodeArgs a) {
+  constexpr int LPK = D / 8;          // lanes per key row
+  constexpr int KPS = 32 / LPK;       // keys per warp step
+  constexpr int BLK = KPS * kDecBlockSteps;
+  __shared__ float s_m[kDecWarps][G], s_l[kDecWarps][G];
+  __shared__ float s_acc[kDecWarps][G][D];
+
+  pdl_wait();
+  pdl_launch_dependents();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int pair = blockIdx.x / a.n_splits, split = blockIdx.x - pair * a.n_splits;
+  const int layer = pair / a.Hkv, h = pair - layer * a.Hkv;
+  int n = decode_n(a);
+  if (n > a.n_cap) {
+    if (threadIdx.x == 0 && blockIdx.x == 0) record_status(a.status, STEPKV_ENOSPACE);
+    n = a.n_cap;
+  }
+  if (n < 1 && threadIdx.x == 0 && blockIdx.x == 0) record_status(a.status, STEPKV_EDATA);
+  const int k_begin = split * kDecSplitKeys;
+  const int k_end = min(n, k_begin + kDecSplitKeys);
+  const int kslot = lane / LPK, hl = lane - kslot * LPK;
+
+  // this lane's 8 elements of every query head of the group, pre-scaled for exp2
+  float q[G][8];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    const uint4 r = __ldg(reinterpret_cast<const uint4*>(a.q[layer] + (size_t)(h * G + g) * D) + hl);
+    bf16x8_to_f32(r, q[g]);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) q[g][e] *= a.c;
+  }
+  float m[G], l[G], acc[G][8];
+#pragma unroll
+  for (int g = 0; g < G; ++g) {
+    m[g] = -INFINITY;
+    l[g] = 0.f;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[g][e] = 0.f;
+  }
+
+  const uint16_t* Kh = a.K[layer] + (size_t)h * a.head_stride;
+  const uint16_t* Vh = a.V[layer] + (size_t)h * a.head_stride;
+  // warp w takes blocks w, w + 4, ... of BLK consecutive keys
+  for (int kb = k_begin + warp * BLK; kb < k_end; kb += kDecWarps * BLK) {
+    uint4 kr[kDecBlockSteps], vr[kDecBlockSteps];
+    bool ok[kDecBlockSteps];
+#pragma unroll
+    for (int t = 0; t < kDecBlockSteps; ++t) {
+      const int j = kb + t * KPS + kslot;
+      ok[t] = j < k_end;
+      kr[t] = ok[t] ? __ldcs(reinterpret_cast<const uint4*>(Kh + (size_t)j * D) + hl) : make_uint4(0, 0, 0, 0);
+      vr[t] = ok[t] ? __ldcs(reinterpret_cast<const uint4*>(Vh + (size_t)j * D) + hl) : make_uint4(0, 0, 0, 0);
+    }
+    float s[kDecBlockSteps][G];
+#pragma unroll
+    for (int t = 0; t < kDecBlockSteps; ++t) {
+      float kf[8];
+      bf16x8_to_f32(kr[t], kf);
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        float x = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) x = fmaf(q[g][e], kf[e], x);
+#pragma unroll
+        for (int o = LPK / 2; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        s[t][g] = ok[t] ? x : -INFINITY;
+      }
+    }
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      float mb = m[g];
+#pragma unroll
+      for (int t = 0; t < kDecBlockSteps; ++t) mb = fmaxf(mb, s[t][g]);
+      if (mb == -INFINITY) continue;
+      const float sc = ex2_approx(m[g] - mb);
+      l[g] *= sc;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[g][e] *= sc;
+#pragma unroll
+      for (int t = 0; t < kDecBlockSteps; ++t) {
+        const float p = ex2_approx(s[t][g] - mb);
+        float vf[8];
+        bf16x8_to_f32(vr[t], vf);
+        l[g] += p;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
+      }
+      m[g] = mb;
+    }
+  }
+  // merge the key slots of the warp (lanes with the same hl), then the warps through shared memory
+#pragma unroll
+  for (int o = LPK; o < 32; o <<= 1) {
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m[g], o);
+      const float l2 = __shfl_xor_sync(0xffffffffu, l[g], o);
+      float acc2[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc2[e] = __shfl_xor_sync(0xffffffffu, acc[g][e], o);
+      merge_state<8>(m[g], l[g], acc[g], m2, l2, acc2);
+    }
+  }
+  if (kslot == 0) {
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (hl == 0) {
+        s_m[warp][g] = m[g];
+        s_l[warp][g] = l[g];
+      }
+#pragma unroll
+      for (int e = 0; e < 8; ++e) s_acc[warp][g][hl * 8 + e] = acc[g][e];
+    }
+  }
+  __syncthreads();
+  // thread t < G*D/4: head g = t / (D/4), elements 4*(t % (D/4)) .. +4 -> merge the warps in order
+  constexpr int PER = 4;
+  for (int t = threadIdx.x; t < G * (D / PER); t += kDecThreads) {
+    const int g = t / (D / PER), e0 = (t - g * (D / PER)) * PER;
+    float mm = -INFINITY, ll = 0.f, aa[PER] = {0.f, 0.f, 0.f, 0.f};
+    for (int w = 0; w < kDecWarps; ++w) {
+      float a2[PER];
+#pragma unroll
+      for (int e = 0; e < PER; ++e) a2[e] = s_acc[w][g][e0 + e];
+      merge_state<PER>(mm, ll, aa, s_m[w][g], s_l[w][g], a2);
+    }
+    float* dst = a.part + ((size_t)(pair * a.n_splits + split) * G + g) * (D + 4);
+    if (e0 == 0) {
+      dst[0] = mm;
+      dst[1] = ll;
+    }
+    *reinterpret_cast<float4*>(dst + 4 + e0) = make_float4(aa[0], aa[1], aa[2], aa[3]);
+  }
+}
+
+// One warp per (pair, head): merge the splits in order and write out = acc / l.
+template <int D, int G>
+__global__ void __launch_bounds__(128) decode_merge_kernel(const __grid_constant__ DecodeArgs a, int n_items) {
+  constexpr int PER = D / 32;
+  pdl_wait();
+  pdl_launch_dependents();
+  const int item = blockIdx.x * 4 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (item >= n_items) return;
+  const int pair = item / G, g = item - pair * G;
+  const int layer = pair / a.Hkv, h = pair - layer * a.Hkv;
+  int n = min(decode_n(a), a.n_cap);
+  const int used = max(0, min(a.n_splits, (n + kDecSplitKeys - 1) / kDecSplitKeys));
+  float mm = -INFINITY, ll = 0.f, aa[PER];
+#pragma unroll
+  for (int e = 0; e < PER; ++e) aa[e] = 0.f;
+  for (int sp = 0; sp < used; ++sp) {
+    const float* src = a.part + ((size_t)(pair * a.n_splits + sp) * G + g) * (D + 4);
+    float a2[PER];
+#pragma unroll
+    for (int e = 0; e < PER; ++e) a2[e] = __ldcg(src + 4 + lane * PER + e);
+    merge_state<PER>(mm, ll, aa, __ldcg(src), __ldcg(src + 1), a2);
+  }
+  const float inv = ll > 0.f ? 1.f / ll : 0.f;
+  float* o = a.out[layer] + (size_t)(h * G + g) * D + lane * PER;
+#pragma unroll
+  for (int e = 0; e < PER; ++e) o[e] = aa[e] * inv;
+}
+
+size_t decode_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap) {
+  const int n_splits = std::max(1, (n_cap + kDecSplitKeys - 1) / kDecSplitKeys);
+  return (size_t)n_layers * Hq * n_splits * (d + 4) * sizeof(float);
+}
+
+template <int D, int G>
+static cudaError_t decode_launch(const DecodeArgs& a, int pairs, cudaStream_t stream) {
+  cudaError_t e = launch_kernel(decode_partial_kernel<D, G>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
+                                stream, a);
+  if (e != cudaSuccess) return e;
+  const int items = pairs * G;
+  return launch_kernel(decode_merge_kernel<D, G>, dim3((items + 3) / 4), dim3(128), 0, stream, a, items);
+}
+
+template <int D>
+static cudaError_t decode_dispatch_g(const DecodeArgs& a, int G, int pairs, cudaStream_t stream) {
+  switch (G) {
+    case 1: return decode_launch<D, 1>(a, pairs, stream);
+    case 2: return decode_launch<D, 2>(a, pairs, stream);
+    case 4: return decode_launch<D, 4>(a, pairs, stream);
+    case 5: return decode_launch<D, 5>(a, pairs, stream);
+    case 8: return decode_launch<D, 8>(a, pairs, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const* K, const void* const* V,
+                           int64_t head_stride, int Hkv, int Hq, int d, const int32_t* n_dev, int n_host, int n_cap,
+                           float* const* out, void* ws, int32_t* status, cudaStream_t stream) {
+  const int G = Hq / Hkv;
+  const int n_splits = std::max(1, (n_cap + kDecSplitKeys - 1) / kDecSplitKeys);
+  float* part = static_cast<float*>(ws);
+  for (int l0 = 0; l0 < n_layers; l0 += kMaxDecodeLayers) {
+    const int nl = std::min(kMaxDecodeLayers, n_layers - l0);
+    DecodeArgs a;
+    memset(&a, 0, sizeof(a));
+    for (int l = 0; l < nl; ++l) {
+      a.q[l] = static_cast<const uint16_t*>(q[l0 + l]);
+      a.K[l] = static_cast<const uint16_t*>(K[l0 + l]);
+      a.V[l] = static_cast<const uint16_t*>(V[l0 + l]);
+      a.out[l] = out[l0 + l];
+    }
+    a.head_stride = head_stride;
+    a.Hkv = Hkv;
+    a.n_splits = n_splits;
+    a.n_dev = n_dev;
+    a.n_host = n_host;
+    a.n_cap = n_cap;
+    a.c = (float)(1.4426950408889634 / sqrt((double)d));
+    a.part = part;
+    a.status = status;
+    const cudaError_t e = d == 128 ? decode_dispatch_g<128>(a, G, nl * Hkv, stream)
+                                   : decode_dispatch_g<64>(a, G, nl * Hkv, stream);
+    if (e != cudaSuccess) {
+      set_last_cuda_error(e);
+      return STEPKV_ECUDA;
+    }
+  }
+  return STEPKV_OK;
+}
+
+}  // namespace stepkv

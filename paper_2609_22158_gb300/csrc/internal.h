@@ -78,6 +78,13 @@ cudaError_t launch_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cl
   return cudaLaunchKernelEx(&cfg, kern, std::forward<A0>(a0));
 }
 
+// ---- decode attention (decode.cu)
+constexpr int kMaxDecodeLayers = 64;  // layers per launch (pointer arrays travel in the kernel parameters)
+size_t decode_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap);
+stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const* K, const void* const* V,
+                           int64_t head_stride, int Hkv, int Hq, int d, const int32_t* n_dev, int n_host, int n_cap,
+                           float* const* out, void* ws, int32_t* status, cudaStream_t stream);
+
 // ---- score (score.cu)
 int score_row_groups(int Hkv, int Hq, int W);
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W);

@@ -110,6 +110,23 @@ def test_compact_rejects_bad_arguments_on_host(lib):
                               None, None, None, None, None, None) == B.STEPKV_EINVAL
 
 
+def test_decode_rejects_bad_arguments_on_host(lib):
+    from paper_2609_22158_gb300 import binding as B
+    p = ctypes.cast((ctypes.c_void_p * 1)(256), ctypes.c_void_p)
+    ws = ctypes.c_void_p(1 << 20)
+    call = lambda Hkv, Hq, d, stride, n, cap, w=ws: lib.stepkv_decode(1, p, p, p, stride, Hkv, Hq, d, None, n, cap,
+                                                                       p, w, 1 << 30, None, None)
+    assert call(2, 8, 96, 96 * 100, 50, 100) == B.STEPKV_EUNSUPPORTED    # d
+    assert call(2, 6, 128, 128 * 100, 50, 100) == B.STEPKV_EUNSUPPORTED   # G = 3
+    assert call(3, 8, 128, 128 * 100, 50, 100) == B.STEPKV_EINVAL         # Hq % Hkv
+    assert call(2, 8, 128, 128 * 99, 50, 100) == B.STEPKV_EINVAL          # head stride below capacity
+    assert call(2, 8, 128, 128 * 100, 101, 100) == B.STEPKV_EINVAL        # host n above capacity
+    assert call(2, 8, 128, 128 * 100, 0, 100) == B.STEPKV_EINVAL          # no keys
+    assert call(2, 8, 128, 128 * 100, 50, 100, ctypes.c_void_p(1 << 20 | 8)) == B.STEPKV_EINVAL  # ws alignment
+    assert lib.stepkv_decode_workspace_size(32, 8, 32, 128, 8272) > 0
+    assert lib.stepkv_decode_workspace_size(32, 8, 32, 96, 8272) == 0
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2609_22158_gb300 import binding
     with pytest.raises(binding.StepKVError):

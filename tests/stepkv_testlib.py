@@ -101,7 +101,7 @@ class GpuTraj:
         from paper_2609_22158_gb300 import binding as B
         return B.StepSignals(self.valid, self.gain, self.red, self.reuse_in, self.obs_sim, self.reuse_out)
 
-    def problem(self):
+    def problem(self, budget=None):
         t = torch()
         from paper_2609_22158_gb300 import binding as B
         s = self.tr.shape
@@ -111,7 +111,8 @@ class GpuTraj:
         self.out = B.SelectOutputs.allocate(s.T, self.tr.n_steps, cap, "cuda")
         self.step_id_out = t.full((cap,), -7, dtype=t.int32, device="cuda")
         self.pos_out = t.full((cap,), -7, dtype=t.int32, device="cuda")
-        return B.Problem(self.K, self.V, self.Q, s.T, self.step_id, self.prot, self.steps(), self.budget(),
+        return B.Problem(self.K, self.V, self.Q, s.T, self.step_id, self.prot, self.steps(),
+                         budget if budget is not None else self.budget(),
                          self.K_out, self.V_out, self.out, pos_in=self.pos, step_id_out=self.step_id_out,
                          pos_out=self.pos_out)
 

@@ -240,9 +240,8 @@ def run_ours(args):
     import torch
     from paper_2609_22158_gb300 import binding as B
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2609_22158_gb300 import multirank as MR
+    world, rank, local = MR.rank_env()
     dist = None
     if world > 1:
         import torch.distributed as dist
@@ -256,7 +255,7 @@ def run_ours(args):
 
     tr = make_traj(args)
     s = tr.shape
-    dt = DeviceTraj(tr, dev, seed=1234 + rank)
+    dt = DeviceTraj(tr, dev, seed=MR.rank_seed(1234, rank))
     params = B.Params()
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
@@ -293,14 +292,11 @@ def run_ours(args):
     if dist:
         dist.barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
-    ms = sum(step_ms) / len(step_ms)
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = MR.max_over_ranks(sum(step_ms) / len(step_ms), dist, dev)
     if int(dt.status.item()) != 0:
         raise RuntimeError(f"device status {int(dt.status.item())} in the timed region")
-    value = world * s.T / (ms * 1e-3)
+    tokens = MR.gather_tokens(s.T, dist, dev)
+    value = MR.job_throughput(tokens, ms * 1e-3)
 
     # per-stage timing (same shapes, separate entry points, same stream) for the roofline
     stage = {}
@@ -372,13 +368,9 @@ def run_ours(args):
             e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = e0.elapsed_time(e1) / k2
-        if dist:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
+        e2e_ms = MR.max_over_ranks(e0.elapsed_time(e1) / k2, dist, dev)
         assert int(host_idx[dt.cap].item()) == dt.n_kept_expected
-        e2e = {"value": world * s.T / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+        e2e = {"value": MR.job_throughput(tokens, e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": k2}
 
     # decode attention over a compacted cache (timed separately, not part of the metric): the incremental
@@ -461,8 +453,8 @@ def run_ours(args):
 # ---------------------------------------------------------------------------------- reference arm
 def run_reference(args):
     """The oracle as it stands on the host cores, same workload/metric; each step a bounded sample."""
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
+    from paper_2609_22158_gb300 import multirank as MR
+    world, rank, _ = MR.rank_env()
     if rank != 0:
         return
     tr = make_traj(args)

@@ -285,8 +285,11 @@ STEPKV_API stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q,
 
 /* ---------------------------------------------------------------------------------------------
  * The fused pass (score -> reduce/fuse -> select -> compact) for n_traj independent trajectories
- * (one pruning boundary each, Algorithm 1).  probs is a host array; all trajectories run on
- * `stream` in order, sharing `ws` (size from stepkv_compress_workspace_size over the same array).
+ * (one pruning boundary each, Algorithm 1).  probs is a host array; everything runs on `stream`:
+ * the saliency of each trajectory (one launch each), then the selections of all trajectories in one
+ * launch (one 8-CTA cluster per trajectory, up to 16 per launch), then each compaction.  `ws` (size
+ * from stepkv_compress_workspace_size over the same array) holds one shared region for the saliency
+ * partials and a private region per trajectory.
  */
 STEPKV_API size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj);
 STEPKV_API stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj,

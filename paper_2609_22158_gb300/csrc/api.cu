@@ -7,6 +7,7 @@
 #include <mutex>
 #include <map>
 #include <utility>
+#include <vector>
 
 #include "common.cuh"
 #include "internal.h"
@@ -297,24 +298,28 @@ stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q, const void
                     static_cast<cudaStream_t>(stream));
 }
 
-static size_t compress_ws_one(const stepkv_problem_t& p) {
+// Workspace of the fused pass: one region of pass-1 partials (the score launches run one after another
+// and reuse it), then per trajectory its fixed-point token saliency T_acc and its selection scratch
+// (all selections run in one batched launch, so these are private).
+static size_t compress_part_bytes(const stepkv_problem_t& p) {
   const int Ls = std::min(p.n_sal_layers, p.L);
-  size_t b = align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
-  b += align256((size_t)p.T * sizeof(unsigned long long));
-  b += align256(select_ws_bytes(p.T, p.steps.n_steps));
-  return b;
+  return align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
+}
+static size_t compress_traj_bytes(const stepkv_problem_t& p) {
+  return align256((size_t)p.T * sizeof(unsigned long long)) + align256(select_ws_bytes(p.T, p.steps.n_steps));
 }
 
 size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj) {
   if (!probs || n_traj < 1) return 0;
-  size_t m = 0;
+  size_t part = 0, per = 0;
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     if (p.L < 1 || p.Hkv < 1 || p.Hq < p.Hkv || p.T < 1 || p.W < 1 || p.n_sal_layers < 1 || p.steps.n_steps < 1)
       return 0;
-    m = std::max(m, compress_ws_one(p));
+    part = std::max(part, compress_part_bytes(p));
+    per += compress_traj_bytes(p);
   }
-  return m;
+  return part + per;
 }
 
 stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, const stepkv_params_t* params,
@@ -336,26 +341,35 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
                             p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride);
     if (st != STEPKV_OK) return st;
-    if (ws_bytes < compress_ws_one(p)) return STEPKV_ENOSPACE;
   }
+  if (ws_bytes < stepkv_compress_workspace_size(probs, n_traj)) return STEPKV_ENOSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  size_t part_bytes = 0;
+  for (int i = 0; i < n_traj; ++i) part_bytes = std::max(part_bytes, compress_part_bytes(probs[i]));
+  float2* part = reinterpret_cast<float2*>(ws);
+  uint8_t* w = static_cast<uint8_t*>(ws) + part_bytes;
+  std::vector<SelectSpec> specs((size_t)n_traj);
+  // stage 1 for every trajectory (one cooperative launch each)
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     const int Ls = std::min(p.n_sal_layers, p.L);
-    uint8_t* w = static_cast<uint8_t*>(ws);
-    float2* part = reinterpret_cast<float2*>(w);
-    w += align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
     unsigned long long* t_acc = reinterpret_cast<unsigned long long*>(w);
-    w += align256((size_t)p.T * sizeof(unsigned long long));
-    void* sel_ws = w;
+    void* sel_ws = w + align256((size_t)p.T * sizeof(unsigned long long));
+    w += compress_traj_bytes(p);
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
     stepkv_status_t st = score_run(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
                                    p.T, p.W, nullptr, 0, t_acc, shift, part, dev_status, s);
     if (st != STEPKV_OK) return st;
-    st = select_run(nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps, *params,
-                    p.budget, p.sel, sel_ws, dev_status, s);
-    if (st != STEPKV_OK) return st;
+    specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
+                          *params, p.budget, p.sel, sel_ws, dev_status};
+  }
+  // stages 2-4 for all trajectories in one launch (one cluster per trajectory)
+  stepkv_status_t st = select_run_batch(specs.data(), n_traj, s);
+  if (st != STEPKV_OK) return st;
+  // stage 5
+  for (int i = 0; i < n_traj; ++i) {
+    const stepkv_problem_t& p = probs[i];
     st = compact_run(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap,
                      p.K_out, p.V_out, p.out_head_stride, p.step_id, p.pos_in, p.step_id_out, p.pos_out, dev_status,
                      s);

@@ -101,6 +101,22 @@ stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, i
 // ---- select (select.cu)
 size_t select_ws_bytes(int T, int n_steps);
 // Token saliency comes either as floats T_in[T] or as fixed-point sums t_acc[T] with T_i = t_acc * acc_to_T.
+struct SelectSpec {
+  const float* T_in;
+  const unsigned long long* t_acc;
+  double acc_to_T;
+  int T;
+  const int32_t* step_id;
+  const uint8_t* prot;
+  stepkv_steps_t steps;
+  stepkv_params_t params;
+  stepkv_budget_t budget;
+  stepkv_select_out_t out;
+  void* ws;          // select_ws_bytes(T, n_steps), 256-byte aligned, private to this trajectory
+  int32_t* status;
+};
+// Independent trajectories in as few launches as possible (one cluster each).
+stepkv_status_t select_run_batch(const SelectSpec* specs, int n, cudaStream_t stream);
 stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, double acc_to_T, int T,
                            const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
                            const stepkv_params_t& params, const stepkv_budget_t& budget,

@@ -63,6 +63,14 @@ struct SelShared {
   int pad[3];
 };
 
+// Several independent trajectories in one launch: cluster (or CTA) c selects for trajectory c, so the
+// latency-bound passes of different trajectories run side by side on different SMs.
+constexpr int kMaxSelBatch = 16;
+struct SelectBatch {
+  SelectArgs t[kMaxSelBatch];
+};
+static_assert(sizeof(SelectBatch) <= 32000, "kernel parameter space");
+
 template <int NT>
 __device__ __forceinline__ int block_reduce_sum_int(int v, int* scratch) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -202,7 +210,8 @@ struct ClusterOps<1> {
 };
 
 template <int NC, int NT>
-__global__ void __launch_bounds__(NT, 1) select_kernel(const SelectArgs a) {
+__global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ SelectBatch batch) {
+  const SelectArgs& a = batch.t[blockIdx.x / NC];
   constexpr int NW = NT / 32;
   constexpr int UNROLL = NT >= 1024 ? 4 : 8;
   ClusterOps<NC> cl;
@@ -673,24 +682,21 @@ size_t select_ws_bytes(int T, int n_steps) {
   return align256(n * 4) + align256(n * 4) + align256(n * 8) + align256(n * 4) + align256(n * 4);
 }
 
-stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, double acc_to_T, int T,
-                           const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
-                           const stepkv_params_t& params, const stepkv_budget_t& budget,
-                           const stepkv_select_out_t& out, void* ws, int32_t* status, cudaStream_t stream) {
+static SelectArgs make_select_args(const SelectSpec& sp) {
   SelectArgs a;
   memset(&a, 0, sizeof(a));
-  a.T_in = T_in;
-  a.t_acc = t_acc;
-  a.acc_to_T = (float)acc_to_T;
-  a.T = T;
-  a.step_id = step_id;
-  a.prot = prot;
-  a.steps = steps;
-  a.prm = params;
-  a.budget = budget;
-  a.out = out;
-  const size_t n = (size_t)std::max(steps.n_steps, 1);
-  uint8_t* w = static_cast<uint8_t*>(ws);
+  a.T_in = sp.T_in;
+  a.t_acc = sp.t_acc;
+  a.acc_to_T = (float)sp.acc_to_T;
+  a.T = sp.T;
+  a.step_id = sp.step_id;
+  a.prot = sp.prot;
+  a.steps = sp.steps;
+  a.prm = sp.params;
+  a.budget = sp.budget;
+  a.out = sp.out;
+  const size_t n = (size_t)std::max(sp.steps.n_steps, 1);
+  uint8_t* w = static_cast<uint8_t*>(sp.ws);
   a.S = reinterpret_cast<float*>(w);
   w += align256(n * 4);
   a.acc_cnt = reinterpret_cast<int32_t*>(w);
@@ -700,29 +706,59 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
   a.acc_max = reinterpret_cast<uint32_t*>(w);
   w += align256(n * 4);
   a.acc_kept = reinterpret_cast<int32_t*>(w);
-  a.status = status;
-  const int nc = T <= kSelSingleMaxT ? 1 : kSelClusterCtas;
-  a.chunk = ((T + nc - 1) / nc + 15) & ~15;
-  const size_t fixed = (((size_t)a.chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) + 64 * 4;
+  a.status = sp.status;
+  return a;
+}
+
+// Shared memory of one trajectory's CTA: keys + step ids of its chunk, histograms, exchange blocks,
+// scratch, and S_k when it fits.
+static size_t select_smem(int chunk, int nc, int n_steps, int* s_in_smem) {
+  const size_t fixed = (((size_t)chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) + 64 * 4;
   const size_t budget_smem = 232448 - 1024;
-  a.s_in_smem = fixed + (size_t)steps.n_steps * 4 <= budget_smem ? 1 : 0;
-  const size_t smem = fixed + (a.s_in_smem ? (size_t)steps.n_steps * 4 : 0);
-  cudaError_t e;
-  if (nc == 1) {
-    void (*kern)(SelectArgs) = select_kernel<1, 1024>;
-    e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
-    if (e == cudaSuccess) e = launch_kernel(kern, dim3(1), dim3(1024), smem, stream, a, true);
-  } else {
-    void (*kern)(SelectArgs) = select_kernel<kSelClusterCtas, 512>;
-    e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
-    if (e == cudaSuccess)
-      e = launch_cluster(kern, dim3(kSelClusterCtas), dim3(512), kSelClusterCtas, smem, stream, a, true);
-  }
-  if (e != cudaSuccess) {
-    set_last_cuda_error(e);
-    return STEPKV_ECUDA;
+  *s_in_smem = fixed + (size_t)n_steps * 4 <= budget_smem ? 1 : 0;
+  return fixed + (*s_in_smem ? (size_t)n_steps * 4 : 0);
+}
+
+stepkv_status_t select_run_batch(const SelectSpec* specs, int n, cudaStream_t stream) {
+  for (int b0 = 0; b0 < n; b0 += kMaxSelBatch) {
+    const int nb = std::min(kMaxSelBatch, n - b0);
+    int T_max = 0;
+    for (int i = 0; i < nb; ++i) T_max = std::max(T_max, specs[b0 + i].T);
+    const int nc = T_max <= kSelSingleMaxT ? 1 : kSelClusterCtas;
+    SelectBatch batch;
+    memset(&batch, 0, sizeof(batch));
+    size_t smem = 0;
+    for (int i = 0; i < nb; ++i) {
+      SelectArgs a = make_select_args(specs[b0 + i]);
+      a.chunk = ((a.T + nc - 1) / nc + 15) & ~15;
+      smem = std::max(smem, select_smem(a.chunk, nc, a.steps.n_steps, &a.s_in_smem));
+      batch.t[i] = a;
+    }
+    cudaError_t e;
+    if (nc == 1) {
+      void (*kern)(SelectBatch) = select_kernel<1, 1024>;
+      e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
+      if (e == cudaSuccess) e = launch_kernel(kern, dim3(nb), dim3(1024), smem, stream, batch, true);
+    } else {
+      void (*kern)(SelectBatch) = select_kernel<kSelClusterCtas, 512>;
+      e = ensure_smem_attr(reinterpret_cast<const void*>(kern), (int)smem);
+      if (e == cudaSuccess)
+        e = launch_cluster(kern, dim3(kSelClusterCtas * nb), dim3(512), kSelClusterCtas, smem, stream, batch, true);
+    }
+    if (e != cudaSuccess) {
+      set_last_cuda_error(e);
+      return STEPKV_ECUDA;
+    }
   }
   return STEPKV_OK;
+}
+
+stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, double acc_to_T, int T,
+                           const int32_t* step_id, const uint8_t* prot, const stepkv_steps_t& steps,
+                           const stepkv_params_t& params, const stepkv_budget_t& budget,
+                           const stepkv_select_out_t& out, void* ws, int32_t* status, cudaStream_t stream) {
+  const SelectSpec sp{T_in, t_acc, acc_to_T, T, step_id, prot, steps, params, budget, out, ws, status};
+  return select_run_batch(&sp, 1, stream);
 }
 
 }  // namespace stepkv

@@ -407,6 +407,13 @@ def run_ours(args):
             raise RuntimeError(f"device status {int(dt.status.item())} after decode")
         del Kd, Vd
 
+    # the incremental agent loop (timed separately, not part of the metric): Llama-3-8B heads, a 4096-token
+    # start, one new step per boundary, the compacted cache plus the new step compressed under a fixed
+    # 8192-token budget, then 64 single-token decode reads over the compacted cache
+    incremental = None
+    if rank == 0 and not args.no_incremental:
+        incremental = run_incremental(args, s, dev, stream, hbm)
+
     clocks = sampler.stop() if sampler else None
     if dist:
         dist.barrier()
@@ -438,7 +445,7 @@ def run_ours(args):
         "pass_hbm": {"algorithmic_bytes": ab["total"], "achieved_gbs": round(pass_gbs, 1),
                      "frac_of_measured": round(pass_gbs / hbm, 4), "frac_of_nominal_8tbs": round(pass_gbs / 8000, 4)},
         "stages_us": {k: round(v, 2) for k, v in stage.items()} if stage else None,
-        "cpu_baseline": cpu, "e2e": e2e, "decode": decode,
+        "cpu_baseline": cpu, "e2e": e2e, "decode": decode, "incremental": incremental,
         "gpu_launches": launches_per_pass(tr) * args.steps,
         "clocks": clocks,
         "wall_s_timed_region": round(wall1 - wall0, 4),
@@ -448,6 +455,91 @@ def run_ours(args):
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
+
+
+def run_incremental(args, s, dev, stream, hbm):
+    """Boundaries of the incremental loop on device-random K/V/Q (layout and signals from the seeded
+    generator); events time each compression and each group of 64 decode reads."""
+    import numpy as np
+    import torch
+    from paper_2609_22158_gb300 import binding as B, workload as wl
+    budget, t0, n_dec = 8192, 4096, 64
+    lp = wl.IncrementalLoop(5, L=s.L, Hq=s.Hq, Hkv=s.Hkv, d=s.d, W=s.W, t0=t0, budget_count=budget)
+    gen = torch.Generator(device=dev).manual_seed(55)
+    rnd = lambda n: torch.randn((s.Hkv, n, s.d), generator=gen, device=dev, dtype=torch.bfloat16)
+    step_id, n_steps = lp.initial_layout()
+    pos = np.arange(t0, dtype=np.int32)
+    next_pos = t0
+    K = [rnd(t0) for _ in range(s.L)]
+    V = [rnd(t0) for _ in range(s.L)]
+    reuse = np.zeros(n_steps, np.float32)
+    params = B.Params()
+    status = B.new_status(dev)
+    comp_us, dec_us, rows = [], [], []
+    for b in range(args.inc_boundaries):
+        if b > 0:
+            n_new = lp.step_length(b)
+            n_steps += 1
+            K = [torch.cat([k, rnd(n_new)], dim=1) for k in K]
+            V = [torch.cat([v, rnd(n_new)], dim=1) for v in V]
+            step_id = np.concatenate([step_id, np.full(n_new, n_steps - 1, np.int32)])
+            pos = np.concatenate([pos, np.arange(next_pos, next_pos + n_new, dtype=np.int32)])
+            next_pos += n_new
+            reuse = np.concatenate([reuse, np.float32([0.0])])
+        T = int(step_id.shape[0])
+        prot = lp.protected(step_id)
+        valid, gain, red, obs_sim = lp.signals(b, n_steps)
+        t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+        reuse_out = torch.empty(n_steps, dtype=torch.float32, device=dev)
+        steps = B.StepSignals(t(valid), t(gain), t(red), t(reuse), t(obs_sim), reuse_out)
+        cap = min(T, budget + int(prot.sum()))
+        out = B.SelectOutputs.allocate(T, n_steps, cap, dev, full=False)
+        K_out = [torch.empty((s.Hkv, cap, s.d), dtype=torch.bfloat16, device=dev) for _ in range(s.L)]
+        V_out = [torch.empty((s.Hkv, cap, s.d), dtype=torch.bfloat16, device=dev) for _ in range(s.L)]
+        sid_out = torch.empty(cap, dtype=torch.int32, device=dev)
+        pos_out = torch.empty(cap, dtype=torch.int32, device=dev)
+        Q = [torch.randn((s.Hq, s.W, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.Ls)]
+        prob = B.Problem(K, V, Q, T, t(step_id), t(prot), steps, B.budget_count(budget), K_out, V_out, out,
+                         pos_in=t(pos), step_id_out=sid_out, pos_out=pos_out)
+        ws = torch.empty(B.stepkv_workspace_size([prob]) + 512, dtype=torch.uint8, device=dev)
+        qd = [torch.randn((s.Hq, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
+        outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
+        ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, cap) + 512,
+                           dtype=torch.uint8, device=dev)
+        torch.cuda.synchronize()
+        torch.cuda._sleep(300_000)  # the device stays busy while the host prepares the call
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e[0].record(stream)
+        B.stepkv_compress([prob], params, ws=ws, status=status, stream=stream)
+        e[1].record(stream)
+        for _ in range(n_dec):
+            B.stepkv_decode(qd, K_out, V_out, out.n_kept, out=outd, ws=ws_d, status=status, stream=stream)
+        e[2].record(stream)
+        torch.cuda.synchronize()
+        if int(status.item()) != 0:
+            raise RuntimeError(f"device status {int(status.item())} at boundary {b}")
+        n = int(out.n_kept.item())
+        rows.append(T)
+        comp_us.append(e[0].elapsed_time(e[1]) * 1e3)
+        dec_us.append(e[1].elapsed_time(e[2]) * 1e3 / n_dec)
+        kept = out.kept_idx[:n].long()
+        K = [k[:, :n].clone() for k in K_out]
+        V = [v[:, :n].clone() for v in V_out]
+        step_id = sid_out[:n].cpu().numpy()
+        pos = pos_out[:n].cpu().numpy()
+        reuse = reuse_out.cpu().numpy()
+        del kept
+    steady = [i for i in range(len(rows)) if rows[i] > budget + 2 * s.W]  # the budget binds
+    pick = steady or list(range(len(rows)))
+    return {"workload": f"incremental loop: {args.inc_boundaries} boundaries from a {t0}-token start, one new "
+                        f"step each, fixed {budget}-token budget, {n_dec} decode reads after each compression; "
+                        f"{s.L} layers, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, W={s.W}",
+            "boundaries_with_budget_binding": len(steady),
+            "cache_rows_mean": round(float(np.mean([rows[i] for i in pick])), 1),
+            "compress_us_mean": round(float(np.mean([comp_us[i] for i in pick])), 2),
+            "decode_us_per_token_mean": round(float(np.mean([dec_us[i] for i in pick])), 2),
+            "compress_tokens_per_s": round(float(np.mean([rows[i] for i in pick])) /
+                                           (float(np.mean([comp_us[i] for i in pick])) * 1e-6))}
 
 
 # ---------------------------------------------------------------------------------- reference arm
@@ -492,6 +584,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-stages", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-incremental", action="store_true")
+    ap.add_argument("--inc-boundaries", type=int, default=24)
     ap.add_argument("--oracle-pairs", type=int, default=24)
     ap.add_argument("--oracle-compact-sets", type=int, default=16)
     ap.add_argument("--ref-pairs", type=int, default=2)

@@ -326,6 +326,82 @@ def custom(seed: int, L: int, Hq: int, Hkv: int, d: int, T: int, W: int, n_steps
                      outlier_scale=8.0, outlier_channels=outlier_channels, kv_std=kv_std)
 
 
+class IncrementalLoop:
+    """The incremental agent loop: a trajectory that grows by one step per boundary.  After every step,
+    the already-compacted cache plus the new step is compressed again under a fixed budget, and the
+    agent then decodes over the compacted cache.
+
+    This class draws only the new material of each boundary: the rows of the new step (K/V per layer,
+    step id, original positions), the window queries, and the per-step signals.  The compacted state
+    (retained rows, their step ids and positions, the reuse accumulators) is carried by the caller from
+    one boundary to the next.  The first boundary compresses an initial trajectory of ``t0`` tokens
+    (prompt + steps); every later boundary adds one step with the config-2 field ranges, the Observation
+    at least W + 1 tokens long so that the window lies inside the new step.
+    """
+
+    def __init__(self, seed: int, L: int, Hq: int, Hkv: int, d: int, W: int, t0: int, budget_count: int,
+                 n_prompt: int = 16, n_steps0: int = 8, n_sal_layers: int = 3):
+        self.seed = int(seed)
+        self.shape = Shape(L=L, Hq=Hq, Hkv=Hkv, d=d, T=t0, W=W, n_sal_layers=n_sal_layers)
+        self.t0 = int(t0)
+        self.n_prompt = int(n_prompt)
+        self.budget = Budget.fixed(budget_count)
+        g = _rng(seed, _K_LAYOUT, 50_000)
+        self.init_fields = _cycle_steps(g, n_steps0, (50, 300), (10, 50), (200, 2000), t0 - n_prompt, W)
+
+    # ---- layout
+    def step_length(self, b: int) -> int:
+        """Tokens of the step added at boundary b >= 1 (Thought + Action + Observation)."""
+        g = _rng(self.seed, _K_LAYOUT, 60_000 + b)
+        th, act = int(g.integers(50, 301)), int(g.integers(10, 51))
+        obs = max(int(g.integers(200, 2001)), self.shape.W + 1)
+        return th + act + obs
+
+    def initial_layout(self):
+        """(step_id [t0], n_steps) of the first boundary's trajectory."""
+        step_id = np.full(self.t0, -1, dtype=np.int32)
+        pos = self.n_prompt
+        for k, row in enumerate(self.init_fields):
+            ln = int(row.sum())
+            step_id[pos:pos + ln] = k
+            pos += ln
+        return step_id, int(self.init_fields.shape[0])
+
+    # ---- rows (bf16 bits)
+    def rows(self, b: int, layer: int, which: int, n: int) -> np.ndarray:
+        """New rows of boundary b for one layer: [Hkv, n, d]; which = _K_KEYS or _K_VALUES.  Boundary 0's
+        rows are the initial trajectory."""
+        s = self.shape
+        g = _rng(self.seed, which, layer, 70_000 + b)
+        return f32_to_bf16_bits(g.standard_normal((s.Hkv, n, s.d), dtype=np.float32))
+
+    def queries(self, b: int, layer: int) -> np.ndarray:
+        """Window queries of boundary b, [Hq, W, d]."""
+        s = self.shape
+        g = _rng(self.seed, _K_QUERIES, layer, 80_000 + b)
+        return f32_to_bf16_bits(g.standard_normal((s.Hq, s.W, s.d), dtype=np.float32))
+
+    # ---- signals
+    def signals(self, b: int, n_steps: int):
+        """valid/gain/red of steps 0..n_steps-1 (fixed once drawn per step) and this boundary's obs_sim."""
+        valid = np.empty(n_steps, np.float32)
+        gain = np.empty(n_steps, np.float32)
+        red = np.empty(n_steps, np.float32)
+        for k in range(n_steps):
+            g = _rng(self.seed, _K_SIGNALS, 90_000 + k)
+            valid[k] = np.float32(g.random() >= 0.2)
+            gain[k] = np.float32(g.random())
+            red[k] = np.float32(g.random())
+        obs_sim = _rng(self.seed, _K_SIGNALS, 95_000 + b).random(n_steps).astype(np.float32)
+        return valid, gain, red, obs_sim
+
+    def protected(self, step_id: np.ndarray) -> np.ndarray:
+        """Prompt rows (step id -1) and the last W rows (the window of the newest step)."""
+        prot = (step_id < 0).astype(np.uint8)
+        prot[-self.shape.W:] = 1
+        return prot
+
+
 def decode_queries(seed: int, n_layers: int, Hq: int, d: int, n: int) -> np.ndarray:
     """Single-token decode queries [n, n_layers, Hq, d] bf16 bits."""
     g = _rng(seed, _K_QUERIES, 77_777)

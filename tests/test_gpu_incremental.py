@@ -1,0 +1,100 @@
+"""The incremental agent loop through the C ABI: compress at a boundary, decode over the compacted cache,
+append the next step to the retained rows, compress again.  Every boundary is checked against the
+oracle on the same inputs (the GPU's carried cache, step ids, positions and reuse accumulators), so the
+carrying of state across boundaries is exercised without letting a tolerated swap at one boundary
+change what the next boundary is compared on.
+"""
+import types
+
+import numpy as np
+import pytest
+
+from oracle import stepkv_oracle as O
+from paper_2609_22158_gb300 import workload as wl
+import stepkv_testlib as TL
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def B():
+    import torch
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    from paper_2609_22158_gb300 import binding, build
+    build.build_library()
+    binding.load_library()
+    return binding
+
+
+def _heads_close(g, o):
+    for h in range(o.shape[0]):
+        assert np.abs(g[h] - o[h]).max() <= 2e-3 * np.abs(o[h]).max()
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_incremental_loop_four_boundaries(B, d):
+    import torch
+    L, Hq, Hkv, W, t0, budget = 3, 8, 2, 16, 1200, 300
+    lp = wl.IncrementalLoop(7 + d, L=L, Hq=Hq, Hkv=Hkv, d=d, W=W, t0=t0, budget_count=budget)
+    step_id, n_steps = lp.initial_layout()
+    pos = np.arange(t0, dtype=np.int32)
+    next_pos = t0
+    K = [lp.rows(0, l, wl._K_KEYS, t0) for l in range(L)]
+    V = [lp.rows(0, l, wl._K_VALUES, t0) for l in range(L)]
+    reuse = np.zeros(n_steps, np.float32)
+    p = B.Params()
+    sal_ids = list(range(L - min(3, L), L))
+    for b in range(4):
+        if b > 0:
+            n_new = lp.step_length(b)
+            n_steps += 1
+            K = [np.concatenate([k, lp.rows(b, l, wl._K_KEYS, n_new)], axis=1) for l, k in enumerate(K)]
+            V = [np.concatenate([v, lp.rows(b, l, wl._K_VALUES, n_new)], axis=1) for l, v in enumerate(V)]
+            step_id = np.concatenate([step_id, np.full(n_new, n_steps - 1, np.int32)])
+            pos = np.concatenate([pos, np.arange(next_pos, next_pos + n_new, dtype=np.int32)])
+            next_pos += n_new
+            reuse = np.concatenate([reuse, np.float32([0.5])])  # stale: Algorithm 1 resets c_t
+        T = step_id.shape[0]
+        prot = lp.protected(step_id)
+        valid, gain, red, obs_sim = lp.signals(b, n_steps)
+        Q = [lp.queries(b, l) for l in sal_ids]
+        dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+        Kd = [TL.bf16_dev(k) for k in K]
+        Vd = [TL.bf16_dev(v) for v in V]
+        reuse_out = torch.empty(n_steps, dtype=torch.float32, device="cuda")
+        steps = B.StepSignals(dev(valid), dev(gain), dev(red), dev(reuse), dev(obs_sim), reuse_out)
+        cap = T
+        out = B.SelectOutputs.allocate(T, n_steps, cap, "cuda")
+        K_out = [torch.empty((Hkv, cap, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+        V_out = [torch.empty((Hkv, cap, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+        sid_out = torch.empty(cap, dtype=torch.int32, device="cuda")
+        pos_out = torch.empty(cap, dtype=torch.int32, device="cuda")
+        prob = B.Problem(Kd, Vd, [TL.bf16_dev(q) for q in Q], T, dev(step_id), dev(prot), steps,
+                         B.budget_count(budget), K_out, V_out, out, pos_in=dev(pos), step_id_out=sid_out,
+                         pos_out=pos_out)
+        st = B.stepkv_compress([prob], p)
+        # decode over the compacted cache right away, n read on the device
+        qdec = [wl.decode_queries(100 + b, L, Hq, d, 1)[0, l] for l in range(L)]
+        dec = B.stepkv_decode([TL.bf16_dev(q) for q in qdec], K_out, V_out, out.n_kept, status=st)
+        torch.cuda.synchronize()
+        assert st.item() == 0, b
+        ref = O.compress([K[l] for l in sal_ids], Q, step_id, prot, valid, gain, red, obs_sim, reuse,
+                         TL.oracle_params(p), "count", count=budget)
+        g = types.SimpleNamespace(out=out, tr=types.SimpleNamespace(prot=prot), reuse_out=reuse_out)
+        TL.check_select_outputs(g, ref)
+        n = int(out.n_kept.item())
+        assert n == int(prot.sum()) + min(budget, T - int(prot.sum()))
+        kept = out.kept_idx[:n].cpu().numpy().astype(np.int64)
+        kt = torch.from_numpy(kept).cuda()
+        for l in range(L):
+            assert torch.equal(K_out[l][:, :n], Kd[l].index_select(1, kt))
+            assert torch.equal(V_out[l][:, :n], Vd[l].index_select(1, kt))
+            _heads_close(dec[l].cpu().numpy(), O.decode_attention(qdec[l], K[l][:, kept], V[l][:, kept]))
+        assert np.array_equal(sid_out[:n].cpu().numpy(), step_id[kept])
+        assert np.array_equal(pos_out[:n].cpu().numpy(), pos[kept])
+        # carry the compacted state to the next boundary
+        K = [k[:, kept] for k in K]
+        V = [v[:, kept] for v in V]
+        step_id = step_id[kept]
+        pos = pos[kept]
+        reuse = reuse_out.cpu().numpy()

@@ -459,29 +459,39 @@ def run_ours(args):
 
 def run_incremental(args, s, dev, stream, hbm):
     """Boundaries of the incremental loop on device-random K/V/Q (layout and signals from the seeded
-    generator); events time each compression and each group of 64 decode reads."""
+    generator).  The cache lives in one capacity buffer per layer and is compacted in place (hole
+    filling); each new step is appended after the retained rows.  Events time each compression and each
+    group of 64 decode reads."""
     import numpy as np
     import torch
     from paper_2609_22158_gb300 import binding as B, workload as wl
     budget, t0, n_dec = 8192, 4096, 64
     lp = wl.IncrementalLoop(5, L=s.L, Hq=s.Hq, Hkv=s.Hkv, d=s.d, W=s.W, t0=t0, budget_count=budget)
     gen = torch.Generator(device=dev).manual_seed(55)
-    rnd = lambda n: torch.randn((s.Hkv, n, s.d), generator=gen, device=dev, dtype=torch.bfloat16)
+    cap = budget + 16 + 4 * s.W + 2400  # retained rows + the largest new step
+    Kbuf = [torch.randn((s.Hkv, cap, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
+    Vbuf = [torch.randn((s.Hkv, cap, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
     step_id, n_steps = lp.initial_layout()
     pos = np.arange(t0, dtype=np.int32)
     next_pos = t0
-    K = [rnd(t0) for _ in range(s.L)]
-    V = [rnd(t0) for _ in range(s.L)]
     reuse = np.zeros(n_steps, np.float32)
     params = B.Params()
     status = B.new_status(dev)
-    comp_us, dec_us, rows = [], [], []
+    comp_us, dec_us, rows, moved = [], [], [], []
+    ws = torch.empty(64 << 20, dtype=torch.uint8, device=dev)
+    ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, cap) + 512,
+                       dtype=torch.uint8, device=dev)
+    outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
     for b in range(args.inc_boundaries):
         if b > 0:
             n_new = lp.step_length(b)
             n_steps += 1
-            K = [torch.cat([k, rnd(n_new)], dim=1) for k in K]
-            V = [torch.cat([v, rnd(n_new)], dim=1) for v in V]
+            T0 = int(step_id.shape[0])
+            if T0 + n_new > cap:
+                raise RuntimeError("capacity buffer too small")
+            for k, v in zip(Kbuf, Vbuf):  # the new step's rows, after the retained ones
+                k[:, T0:T0 + n_new].normal_(generator=gen)
+                v[:, T0:T0 + n_new].normal_(generator=gen)
             step_id = np.concatenate([step_id, np.full(n_new, n_steps - 1, np.int32)])
             pos = np.concatenate([pos, np.arange(next_pos, next_pos + n_new, dtype=np.int32)])
             next_pos += n_new
@@ -492,20 +502,18 @@ def run_incremental(args, s, dev, stream, hbm):
         t = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
         reuse_out = torch.empty(n_steps, dtype=torch.float32, device=dev)
         steps = B.StepSignals(t(valid), t(gain), t(red), t(reuse), t(obs_sim), reuse_out)
-        cap = min(T, budget + int(prot.sum()))
-        out = B.SelectOutputs.allocate(T, n_steps, cap, dev, full=False)
-        K_out = [torch.empty((s.Hkv, cap, s.d), dtype=torch.bfloat16, device=dev) for _ in range(s.L)]
-        V_out = [torch.empty((s.Hkv, cap, s.d), dtype=torch.bfloat16, device=dev) for _ in range(s.L)]
-        sid_out = torch.empty(cap, dtype=torch.int32, device=dev)
-        pos_out = torch.empty(cap, dtype=torch.int32, device=dev)
+        kcap = min(T, budget + int(prot.sum()))
+        out = B.SelectOutputs.allocate(T, n_steps, kcap, dev, full=False)
+        sid_out = torch.empty(kcap, dtype=torch.int32, device=dev)
+        pos_out = torch.empty(kcap, dtype=torch.int32, device=dev)
         Q = [torch.randn((s.Hq, s.W, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.Ls)]
-        prob = B.Problem(K, V, Q, T, t(step_id), t(prot), steps, B.budget_count(budget), K_out, V_out, out,
-                         pos_in=t(pos), step_id_out=sid_out, pos_out=pos_out)
-        ws = torch.empty(B.stepkv_workspace_size([prob]) + 512, dtype=torch.uint8, device=dev)
+        live_K = [k[:, :T] for k in Kbuf]
+        live_V = [v[:, :T] for v in Vbuf]
+        prob = B.Problem(live_K, live_V, Q, T, t(step_id), t(prot), steps, B.budget_count(budget), live_K, live_V,
+                         out, pos_in=t(pos), step_id_out=sid_out, pos_out=pos_out)
+        need = B.stepkv_workspace_size([prob])
+        assert need <= ws.numel() - 512
         qd = [torch.randn((s.Hq, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
-        outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
-        ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, cap) + 512,
-                           dtype=torch.uint8, device=dev)
         torch.cuda.synchronize()
         torch.cuda._sleep(300_000)  # the device stays busy while the host prepares the call
         e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
@@ -513,33 +521,32 @@ def run_incremental(args, s, dev, stream, hbm):
         B.stepkv_compress([prob], params, ws=ws, status=status, stream=stream)
         e[1].record(stream)
         for _ in range(n_dec):
-            B.stepkv_decode(qd, K_out, V_out, out.n_kept, out=outd, ws=ws_d, status=status, stream=stream)
+            B.stepkv_decode(qd, live_K, live_V, out.n_kept, out=outd, ws=ws_d, status=status, stream=stream)
         e[2].record(stream)
         torch.cuda.synchronize()
         if int(status.item()) != 0:
             raise RuntimeError(f"device status {int(status.item())} at boundary {b}")
         n = int(out.n_kept.item())
+        kept = out.kept_idx[:n].cpu().numpy()
         rows.append(T)
+        moved.append(int((kept >= n).sum()))
         comp_us.append(e[0].elapsed_time(e[1]) * 1e3)
         dec_us.append(e[1].elapsed_time(e[2]) * 1e3 / n_dec)
-        kept = out.kept_idx[:n].long()
-        K = [k[:, :n].clone() for k in K_out]
-        V = [v[:, :n].clone() for v in V_out]
         step_id = sid_out[:n].cpu().numpy()
         pos = pos_out[:n].cpu().numpy()
         reuse = reuse_out.cpu().numpy()
-        del kept
     steady = [i for i in range(len(rows)) if rows[i] > budget + 2 * s.W]  # the budget binds
     pick = steady or list(range(len(rows)))
+    mean = lambda xs: float(np.mean([xs[i] for i in pick]))
     return {"workload": f"incremental loop: {args.inc_boundaries} boundaries from a {t0}-token start, one new "
-                        f"step each, fixed {budget}-token budget, {n_dec} decode reads after each compression; "
-                        f"{s.L} layers, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, W={s.W}",
+                        f"step each, fixed {budget}-token budget, cache compacted in place (hole filling), "
+                        f"{n_dec} decode reads after each compression; {s.L} layers, Hq={s.Hq}, Hkv={s.Hkv}, "
+                        f"d={s.d}, W={s.W}",
             "boundaries_with_budget_binding": len(steady),
-            "cache_rows_mean": round(float(np.mean([rows[i] for i in pick])), 1),
-            "compress_us_mean": round(float(np.mean([comp_us[i] for i in pick])), 2),
-            "decode_us_per_token_mean": round(float(np.mean([dec_us[i] for i in pick])), 2),
-            "compress_tokens_per_s": round(float(np.mean([rows[i] for i in pick])) /
-                                           (float(np.mean([comp_us[i] for i in pick])) * 1e-6))}
+            "cache_rows_mean": round(mean(rows), 1), "rows_moved_mean": round(mean(moved), 1),
+            "compress_us_mean": round(mean(comp_us), 2),
+            "decode_us_per_token_mean": round(mean(dec_us), 2),
+            "compress_tokens_per_s": round(mean(rows) / (mean(comp_us) * 1e-6))}
 
 
 # ---------------------------------------------------------------------------------- reference arm

@@ -138,7 +138,14 @@ typedef struct {
   const int32_t* pos_in;           /* [T] or NULL: original position of each slot */
   stepkv_steps_t steps;
   stepkv_budget_t budget;
-  void* const* K_out;              /* host [L]: compacted K, [Hkv][rows >= kept_cap][d] */
+  void* const* K_out;              /* host [L]: compacted K, [Hkv][rows >= kept_cap][d].  When every
+                                      K_out[l] is K[l] and every V_out[l] is V[l] (one head stride), the
+                                      compaction runs in place by hole filling: rows [0, n_kept) end up
+                                      holding the retained set, each retained slot below n_kept staying
+                                      where it is and each hole receiving a retained row from a slot at or
+                                      above n_kept, so the rows are no longer in slot order; step_id_out
+                                      and pos_out give each row's step and original position.  Attention
+                                      over the rows does not depend on their order. */
   void* const* V_out;              /* host [L] */
   int64_t out_head_stride;         /* elements (>= kept_cap*d, multiple of 8) */
   int32_t* step_id_out;            /* [kept_cap] or NULL: step_id of each retained slot */
@@ -247,7 +254,8 @@ STEPKV_API stepkv_status_t stepkv_select_static_scratch(const float* sal, int32_
  *  outside [0, T) sets STEPKV_ENOSPACE / STEPKV_EDATA and skips the bad rows.
  *  V_in/V_out may be NULL (keys only); step/pos pointers may be NULL.
  *  Rows are d bf16 values; d*2 bytes must be a multiple of 16 and d <= 256; bases 16-byte aligned;
- *  in/out head strides % 8 == 0.  In-place compaction (K_out == K_in) is not supported.
+ *  in/out head strides % 8 == 0.  In-place compaction (K_out == K_in) is not supported here; the fused
+ *  pass (stepkv_compress) offers it by hole filling.
  */
 STEPKV_API stepkv_status_t stepkv_compact(int32_t n_layers, const void* const* K_in, const void* const* V_in,
                                int64_t in_head_stride, int32_t Hkv, int32_t d, int32_t T,

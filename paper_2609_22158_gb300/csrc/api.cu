@@ -83,10 +83,13 @@ static stepkv_status_t check_select_args(int n_sal, int T, const int32_t* step_i
   return STEPKV_OK;
 }
 
+// In place (every K_out[l] == K_in[l] and V_out[l] == V_in[l], one head stride) is accepted only where
+// `inplace` is non-null (the fused pass); it is then reported there.
 static stepkv_status_t check_compact_args(int n_layers, const void* const* K_in, const void* const* V_in,
                                           int64_t in_head_stride, int Hkv, int d, int T, const int32_t* kept_idx,
                                           const int32_t* n_kept, int kept_cap, void* const* K_out,
-                                          void* const* V_out, int64_t out_head_stride) {
+                                          void* const* V_out, int64_t out_head_stride, bool* inplace = nullptr) {
+  if (inplace) *inplace = false;
   if (n_layers < 0 || Hkv < 1 || d < 8 || T < 1 || kept_cap < 0) return STEPKV_EINVAL;
   if (!kept_idx || !n_kept) return STEPKV_EINVAL;
   if ((d * 2) % 16 || d > 256) return STEPKV_EUNSUPPORTED;
@@ -95,15 +98,22 @@ static stepkv_status_t check_compact_args(int n_layers, const void* const* K_in,
     if ((V_in == nullptr) != (V_out == nullptr)) return STEPKV_EINVAL;
     if (in_head_stride < (int64_t)T * d || out_head_stride < (int64_t)kept_cap * d) return STEPKV_EINVAL;
     if (in_head_stride % 8 || out_head_stride % 8) return STEPKV_EUNSUPPORTED;
+    int same = 0, tensors = 0;
     for (int l = 0; l < n_layers; ++l) {
       if (!K_in[l] || !K_out[l]) return STEPKV_EINVAL;
       if (!aligned16(K_in[l]) || !aligned16(K_out[l])) return STEPKV_EUNSUPPORTED;
-      if (K_in[l] == K_out[l]) return STEPKV_EUNSUPPORTED;
+      same += K_in[l] == K_out[l];
+      ++tensors;
       if (V_in) {
         if (!V_in[l] || !V_out[l]) return STEPKV_EINVAL;
         if (!aligned16(V_in[l]) || !aligned16(V_out[l])) return STEPKV_EUNSUPPORTED;
-        if (V_in[l] == V_out[l]) return STEPKV_EUNSUPPORTED;
+        same += V_in[l] == V_out[l];
+        ++tensors;
       }
+    }
+    if (same != 0) {
+      if (!inplace || same != tensors || in_head_stride != out_head_stride) return STEPKV_EUNSUPPORTED;
+      *inplace = true;
     }
   }
   return STEPKV_OK;
@@ -306,7 +316,8 @@ static size_t compress_part_bytes(const stepkv_problem_t& p) {
   return align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
 }
 static size_t compress_traj_bytes(const stepkv_problem_t& p) {
-  return align256((size_t)p.T * sizeof(unsigned long long)) + align256(select_ws_bytes(p.T, p.steps.n_steps));
+  return align256((size_t)p.T * sizeof(unsigned long long)) + align256(select_ws_bytes(p.T, p.steps.n_steps)) +
+         align256(compact_inplace_ws_bytes(p.T));
 }
 
 size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj) {
@@ -338,8 +349,9 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     if (st != STEPKV_OK) return st;
     st = check_select_args(Ls * p.Hkv, p.T, p.step_id, p.prot, &p.steps, params, &p.budget, &p.sel);
     if (st != STEPKV_OK) return st;
+    bool inplace = false;
     st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
-                            p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride);
+                            p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
     if (st != STEPKV_OK) return st;
   }
   if (ws_bytes < stepkv_compress_workspace_size(probs, n_traj)) return STEPKV_ENOSPACE;
@@ -349,12 +361,14 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   float2* part = reinterpret_cast<float2*>(ws);
   uint8_t* w = static_cast<uint8_t*>(ws) + part_bytes;
   std::vector<SelectSpec> specs((size_t)n_traj);
+  std::vector<void*> plan_ws((size_t)n_traj);
   // stage 1 for every trajectory (one cooperative launch each)
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     const int Ls = std::min(p.n_sal_layers, p.L);
     unsigned long long* t_acc = reinterpret_cast<unsigned long long*>(w);
     void* sel_ws = w + align256((size_t)p.T * sizeof(unsigned long long));
+    plan_ws[i] = static_cast<uint8_t*>(sel_ws) + align256(select_ws_bytes(p.T, p.steps.n_steps));
     w += compress_traj_bytes(p);
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
@@ -367,9 +381,19 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   // stages 2-4 for all trajectories in one launch (one cluster per trajectory)
   stepkv_status_t st = select_run_batch(specs.data(), n_traj, s);
   if (st != STEPKV_OK) return st;
-  // stage 5
+  // stage 5 (out of place, or in place by hole filling when the outputs are the inputs)
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
+    bool inplace = false;
+    check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
+                       p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
+    if (inplace) {
+      st = compact_inplace_run(p.L, p.K_out, p.V_out, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
+                               p.sel.kept_cap, p.step_id, p.pos_in, p.step_id_out, p.pos_out, plan_ws[i], dev_status,
+                               s);
+      if (st != STEPKV_OK) return st;
+      continue;
+    }
     st = compact_run(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap,
                      p.K_out, p.V_out, p.out_head_stride, p.step_id, p.pos_in, p.step_id_out, p.pos_out, dev_status,
                      s);

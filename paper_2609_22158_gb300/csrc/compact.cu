@@ -100,6 +100,144 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
   }
 }
 
+// -------------------------------------------------------------------------------------------------
+// In-place compaction by hole filling.  With the retained slots kept_idx ascending and n = n_kept, the
+// slots below n that are retained stay where they are; every slot below n that is not retained (a hole)
+// receives one retained row from a slot at or above n (a mover), the j-th hole the j-th mover.  Sources
+// (>= n) and destinations (< n) never overlap, so all moves run in parallel.  Rows [0, n) then hold the
+// retained set, no longer in slot order; step_id_out / pos_out record each row's step and original
+// position.  Only the movers are read and written, instead of every retained row.
+
+__device__ __forceinline__ int lower_bound_i32(const int32_t* a, int n, int x) {
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (__ldg(&a[mid]) < x) lo = mid + 1; else hi = mid;
+  }
+  return lo;
+}
+
+// Plan: plan[0] = number of moves; hole[j], mover[j]; and the step/position metadata of rows [0, n).
+__global__ void __launch_bounds__(kCompactThreads) compact_plan_kernel(
+    const int32_t* kept_idx, const int32_t* n_kept_p, int kept_cap, int T, const int32_t* step_id_in,
+    const int32_t* pos_in, int32_t* step_id_out, int32_t* pos_out, int32_t* plan, int32_t* status) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int n = *n_kept_p;
+  if (n > kept_cap || n < 0 || n > T) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+      record_status(status, STEPKV_ENOSPACE);
+      plan[0] = 0;
+    }
+    return;
+  }
+  const int m0 = lower_bound_i32(kept_idx, n, n);  // retained slots below n: kept_idx[0..m0)
+  if (blockIdx.x == 0 && threadIdx.x == 0) plan[0] = n - m0;
+  int32_t* hole = plan + 1;
+  int32_t* mover = plan + 1 + T;
+  for (int r = blockIdx.x * kCompactThreads + threadIdx.x; r < n; r += gridDim.x * kCompactThreads) {
+    const int c = lower_bound_i32(kept_idx, m0, r);  // retained slots below r
+    int src;
+    if (c < m0 && __ldg(&kept_idx[c]) == r) {
+      src = r;
+    } else {
+      const int j = r - c;  // holes below r
+      src = __ldg(&kept_idx[m0 + j]);
+      if (src < n || src >= T) {
+        record_status(status, STEPKV_EDATA);
+        src = r;
+      }
+      hole[j] = r;
+      mover[j] = src;
+    }
+    if (step_id_out) step_id_out[r] = step_id_in ? step_id_in[src] : -1;
+    if (pos_out) pos_out[r] = pos_in ? pos_in[src] : src;
+  }
+}
+
+__global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __grid_constant__ CompactArgs a,
+                                                                       const int32_t* plan) {
+  pdl_wait();
+  pdl_launch_dependents();
+  const int n_moves = *plan;
+  const int32_t* hole = plan + 1;
+  const int32_t* mover = plan + 1 + a.T;
+  const int64_t total = (int64_t)a.n_sets * n_moves;
+  const int64_t per_cta = (total + gridDim.x - 1) / gridDim.x;
+  const int64_t lo = blockIdx.x * per_cta;
+  const int64_t hi = min(total, lo + per_cta);
+  const int vpr = a.row_bytes >> 4;
+  const int rpw = 32 / vpr;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int sub_row = lane / vpr, col = lane - sub_row * vpr;
+  const bool lane_active = sub_row < rpw;
+  const int64_t step = (int64_t)(kCompactThreads / 32) * rpw * kCompactUnroll;
+  for (int64_t base = lo + (int64_t)warp * rpw * kCompactUnroll; base < hi; base += step) {
+    uint4 buf[kCompactUnroll];
+    uint4* dptr[kCompactUnroll];
+#pragma unroll
+    for (int u = 0; u < kCompactUnroll; ++u) {
+      const int64_t ri = base + u * rpw + sub_row;
+      dptr[u] = nullptr;
+      if (lane_active && ri < hi) {
+        const int set = (int)(ri / n_moves);
+        const int j = (int)(ri - (int64_t)set * n_moves);
+        const int src_row = __ldg(&mover[j]), dst_row = __ldg(&hole[j]);
+        const int lt = set / a.Hkv, h = set - lt * a.Hkv;
+        uint8_t* head = a.dst[lt] + (int64_t)h * a.out_head_bytes;
+        buf[u] = ld_stream(reinterpret_cast<const uint4*>(head + (int64_t)src_row * a.row_bytes) + col);
+        dptr[u] = reinterpret_cast<uint4*>(head + (int64_t)dst_row * a.row_bytes) + col;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kCompactUnroll; ++u)
+      if (dptr[u]) st_stream(dptr[u], buf[u]);
+  }
+}
+
+size_t compact_inplace_ws_bytes(int T) { return (size_t)(1 + 2 * (size_t)T) * sizeof(int32_t); }
+
+stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V, int64_t head_stride, int Hkv, int d,
+                                    int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
+                                    const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
+                                    int32_t* pos_out, void* ws, int32_t* status, cudaStream_t stream) {
+  int32_t* plan = static_cast<int32_t*>(ws);
+  int n_sm = 0;
+  cudaError_t e = device_sm_count(&n_sm);
+  if (e == cudaSuccess) {
+    const int blocks = std::max(1, std::min((std::max(kept_cap, 1) + kCompactThreads - 1) / kCompactThreads, n_sm * 4));
+    e = launch_kernel(compact_plan_kernel, dim3(blocks), dim3(kCompactThreads), 0, stream, kept_idx, n_kept, kept_cap,
+                      T, step_id_in, pos_in, step_id_out, pos_out, plan, status);
+  }
+  const int n_tensors = V ? 2 : 1;
+  for (int l0 = 0; e == cudaSuccess && l0 < std::max(n_layers, 1); l0 += kCompactLayersPerLaunch) {
+    const int nl = std::min(kCompactLayersPerLaunch, n_layers - l0);
+    if (nl <= 0) break;
+    CompactArgs a;
+    memset(&a, 0, sizeof(a));
+    for (int l = 0; l < nl; ++l) {
+      a.dst[l * n_tensors] = static_cast<uint8_t*>(K[l0 + l]);
+      if (n_tensors == 2) a.dst[l * 2 + 1] = static_cast<uint8_t*>(V[l0 + l]);
+    }
+    a.n_sets = nl * n_tensors * Hkv;
+    a.Hkv = Hkv;
+    a.row_bytes = d * 2;
+    a.out_head_bytes = head_stride * 2;
+    a.T = T;
+    a.status = status;
+    const int64_t rows_max = (int64_t)a.n_sets * std::max(std::min(kept_cap, T - 1), 1);
+    const int64_t want = (rows_max + 31) / 32;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * kCompactCtasPerSm, want));
+    e = launch_kernel(compact_move_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a,
+                      static_cast<const int32_t*>(plan));
+  }
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return STEPKV_ECUDA;
+  }
+  return STEPKV_OK;
+}
+
 stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* const* V_in, int64_t in_head_stride,
                             int Hkv, int d, int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
                             void* const* K_out, void* const* V_out, int64_t out_head_stride,

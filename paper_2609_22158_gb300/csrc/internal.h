@@ -132,4 +132,11 @@ stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* c
                             const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
                             int32_t* pos_out, int32_t* status, cudaStream_t stream);
 
+// In place (K_out == K): hole filling; ws holds the move plan (compact_inplace_ws_bytes(T)).
+size_t compact_inplace_ws_bytes(int T);
+stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V, int64_t head_stride, int Hkv, int d,
+                                    int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
+                                    const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
+                                    int32_t* pos_out, void* ws, int32_t* status, cudaStream_t stream);
+
 }  // namespace stepkv

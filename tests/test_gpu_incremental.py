@@ -98,3 +98,81 @@ def test_incremental_loop_four_boundaries(B, d):
         step_id = step_id[kept]
         pos = pos[kept]
         reuse = reuse_out.cpu().numpy()
+
+
+def test_incremental_loop_in_place(B):
+    """The same loop with the cache compacted in place (hole filling) inside one capacity buffer per
+    layer: each boundary's rows are checked as a set against the oracle's retained rows, through the
+    original positions the pass reports, and the next step is appended after the retained rows."""
+    import torch
+    L, Hq, Hkv, d, W, t0, budget = 3, 8, 2, 64, 16, 1200, 300
+    lp = wl.IncrementalLoop(11, L=L, Hq=Hq, Hkv=Hkv, d=d, W=W, t0=t0, budget_count=budget)
+    n_b = 4
+    cap_total = t0 + sum(lp.step_length(b) for b in range(1, n_b))
+    Kbuf = [torch.zeros((Hkv, cap_total, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+    Vbuf = [torch.zeros((Hkv, cap_total, d), dtype=torch.bfloat16, device="cuda") for _ in range(L)]
+    step_id, n_steps = lp.initial_layout()
+    pos = np.arange(t0, dtype=np.int32)
+    next_pos = t0
+    K = [lp.rows(0, l, wl._K_KEYS, t0) for l in range(L)]  # host mirror of the live rows, same order
+    V = [lp.rows(0, l, wl._K_VALUES, t0) for l in range(L)]
+    for l in range(L):
+        Kbuf[l][:, :t0] = TL.bf16_dev(K[l])
+        Vbuf[l][:, :t0] = TL.bf16_dev(V[l])
+    reuse = np.zeros(n_steps, np.float32)
+    p = B.Params()
+    for b in range(n_b):
+        if b > 0:
+            n_new = lp.step_length(b)
+            n_steps += 1
+            T0 = step_id.shape[0]
+            for l in range(L):
+                kn, vn = lp.rows(b, l, wl._K_KEYS, n_new), lp.rows(b, l, wl._K_VALUES, n_new)
+                Kbuf[l][:, T0:T0 + n_new] = TL.bf16_dev(kn)
+                Vbuf[l][:, T0:T0 + n_new] = TL.bf16_dev(vn)
+                K[l] = np.concatenate([K[l], kn], axis=1)
+                V[l] = np.concatenate([V[l], vn], axis=1)
+            step_id = np.concatenate([step_id, np.full(n_new, n_steps - 1, np.int32)])
+            pos = np.concatenate([pos, np.arange(next_pos, next_pos + n_new, dtype=np.int32)])
+            next_pos += n_new
+            reuse = np.concatenate([reuse, np.float32([0.5])])
+        T = step_id.shape[0]
+        prot = lp.protected(step_id)
+        valid, gain, red, obs_sim = lp.signals(b, n_steps)
+        Q = [lp.queries(b, l) for l in range(L)]
+        dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+        live_K = [k[:, :T] for k in Kbuf]
+        live_V = [v[:, :T] for v in Vbuf]
+        reuse_out = torch.empty(n_steps, dtype=torch.float32, device="cuda")
+        steps = B.StepSignals(dev(valid), dev(gain), dev(red), dev(reuse), dev(obs_sim), reuse_out)
+        out = B.SelectOutputs.allocate(T, n_steps, T, "cuda")
+        sid_out = torch.empty(T, dtype=torch.int32, device="cuda")
+        pos_out = torch.empty(T, dtype=torch.int32, device="cuda")
+        prob = B.Problem(live_K, live_V, [TL.bf16_dev(q) for q in Q], T, dev(step_id), dev(prot), steps,
+                         B.budget_count(budget), live_K, live_V, out, pos_in=dev(pos), step_id_out=sid_out,
+                         pos_out=pos_out)
+        st = B.stepkv_compress([prob], p)
+        torch.cuda.synchronize()
+        assert st.item() == 0, b
+        ref = O.compress(K, Q, step_id, prot, valid, gain, red, obs_sim, reuse, TL.oracle_params(p), "count",
+                         count=budget)
+        g = types.SimpleNamespace(out=out, tr=types.SimpleNamespace(prot=prot), reuse_out=reuse_out)
+        TL.check_select_outputs(g, ref)
+        n = int(out.n_kept.item())
+        kept = out.kept_idx[:n].cpu().numpy().astype(np.int64)
+        # rows [0, n) hold the retained set: slot r came from slot src[r] (r itself when retained below n)
+        pos_of_slot = {int(pp): i for i, pp in enumerate(pos)}
+        po = pos_out[:n].cpu().numpy()
+        src = np.array([pos_of_slot[int(x)] for x in po])
+        assert np.array_equal(np.sort(src), kept)
+        below = kept[kept < n]
+        assert np.array_equal(src[below], below)  # retained rows below n did not move
+        assert np.array_equal(sid_out[:n].cpu().numpy(), step_id[src])
+        for l in range(L):
+            assert np.array_equal(TL.bits_of(Kbuf[l][:, :n]), K[l][:, src])
+            assert np.array_equal(TL.bits_of(Vbuf[l][:, :n]), V[l][:, src])
+        K = [k[:, src] for k in K]
+        V = [v[:, src] for v in V]
+        step_id = step_id[src]
+        pos = pos[src]
+        reuse = reuse_out.cpu().numpy()

@@ -127,14 +127,37 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
     for (int t = 0; t < kDecBlockSteps; ++t) {
       float kf[8];
       bf16x8_to_f32(kr[t], kf);
+      float x[G];
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        float x = 0.f;
+        x[g] = 0.f;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) x = fmaf(q[g][e], kf[e], x);
+        for (int e = 0; e < 8; ++e) x[g] = fmaf(q[g][e], kf[e], x[g]);
+      }
+      if constexpr (G == 4) {
+        // reduce-scatter over the LPK lanes of the row (each lane ends with one head's full sum), then
+        // broadcast the four sums: 9 shuffles instead of 4 x log2(LPK)
+        constexpr int A = LPK / 2, Bx = LPK / 4;
+        const bool ba = (hl & A) != 0, bb = (hl & Bx) != 0;
+        const float y0 = (ba ? x[2] : x[0]) + __shfl_xor_sync(0xffffffffu, ba ? x[0] : x[2], A);
+        const float y1 = (ba ? x[3] : x[1]) + __shfl_xor_sync(0xffffffffu, ba ? x[1] : x[3], A);
+        float z = (bb ? y1 : y0) + __shfl_xor_sync(0xffffffffu, bb ? y0 : y1, Bx);
 #pragma unroll
-        for (int o = LPK / 2; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-        s[t][g] = ok[t] ? x : -INFINITY;
+        for (int o = Bx / 2; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+        const int base_lane = lane & ~(LPK - 1);
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          const float v = __shfl_sync(0xffffffffu, z, base_lane | (((g >> 1) ? A : 0) | ((g & 1) ? Bx : 0)));
+          s[t][g] = ok[t] ? v : -INFINITY;
+        }
+      } else {
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+          float v = x[g];
+#pragma unroll
+          for (int o = LPK / 2; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+          s[t][g] = ok[t] ? v : -INFINITY;
+        }
       }
     }
 #pragma unroll

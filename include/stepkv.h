@@ -151,7 +151,21 @@ typedef struct {
   int32_t* step_id_out;            /* [kept_cap] or NULL: step_id of each retained slot */
   int32_t* pos_out;                /* [kept_cap] or NULL: pos_in (or the slot index) of each retained slot */
   stepkv_select_out_t sel;
+  /* Where the caches live.  STEPKV_MEM_DEVICE (0, the default of a zeroed struct): K/V and
+     K_out/V_out are device memory.  STEPKV_MEM_HOST: page-locked host memory (cudaHostAlloc or
+     cudaHostRegister; checked with cudaPointerGetAttributes, else STEPKV_EINVAL) that the compaction
+     reads or writes across the CPU-GPU link, moving only the retained rows: a cache offloaded to host
+     memory is compressed straight into HBM (out_location DEVICE) or back into host memory.  With
+     kv_location HOST the saliency stage reads K_sal instead of K. */
+  int32_t kv_location;
+  int32_t out_location;
+  const void* const* K_sal;        /* host [n_sal_layers] of device pointers, required when kv_location is
+                                      HOST: layer L-n_sal_layers+i's K in device memory, same layout and
+                                      head stride as K; ignored otherwise */
 } stepkv_problem_t;
+
+#define STEPKV_MEM_DEVICE 0
+#define STEPKV_MEM_HOST 1
 
 /* Table H defaults (appendix "Implementation Details"): lambda=0.3, w_r=0.85, w_c=0.15, r_min=-1,
  * r_max=2, S_max=8, eta=1.5, alpha=0.2, beta=0.8, max-normalised saliency. */
@@ -297,7 +311,9 @@ STEPKV_API stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q,
  * the saliency of each trajectory (one launch each), then the selections of all trajectories in one
  * launch (one 8-CTA cluster per trajectory, up to 16 per launch), then each compaction.  `ws` (size
  * from stepkv_compress_workspace_size over the same array) holds one shared region for the saliency
- * partials and a private region per trajectory.
+ * partials and a private region per trajectory.  Caches in host memory (kv_location / out_location
+ * STEPKV_MEM_HOST) are read and written in place over the CPU-GPU link by the compaction kernels;
+ * their pointers are checked on the host before anything is enqueued.
  */
 STEPKV_API size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj);
 STEPKV_API stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj,

@@ -60,7 +60,12 @@ class CProblem(ctypes.Structure):
                 ("step_id", ctypes.c_void_p), ("prot", ctypes.c_void_p), ("pos_in", ctypes.c_void_p),
                 ("steps", CSteps), ("budget", CBudget),
                 ("K_out", ctypes.c_void_p), ("V_out", ctypes.c_void_p), ("out_head_stride", ctypes.c_int64),
-                ("step_id_out", ctypes.c_void_p), ("pos_out", ctypes.c_void_p), ("sel", CSelOut)]
+                ("step_id_out", ctypes.c_void_p), ("pos_out", ctypes.c_void_p), ("sel", CSelOut),
+                ("kv_location", ctypes.c_int32), ("out_location", ctypes.c_int32), ("K_sal", ctypes.c_void_p)]
+
+
+STEPKV_MEM_DEVICE = 0
+STEPKV_MEM_HOST = 1
 
 
 _lib = None
@@ -165,25 +170,28 @@ def _check(code: int, where: str):
         raise StepKVError(code, where, detail)
 
 
-def _need(t, dtype, name, ndim=None):
+def _need(t, dtype, name, ndim=None, host=False):
     torch = _torch()
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
     if t.dtype != dtype:
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
-    if not t.is_cuda:
+    if host:
+        if t.is_cuda or not t.is_pinned():
+            raise ValueError(f"{name} must be in page-locked host memory (pin_memory())")
+    elif not t.is_cuda:
         raise ValueError(f"{name} must be on a CUDA device")
     if ndim is not None and t.dim() != ndim:
         raise ValueError(f"{name} must have {ndim} dims")
     return t
 
 
-def _rows_layout(ts: Sequence, name: str):
+def _rows_layout(ts: Sequence, name: str, host=False):
     """[H, rows, d] bf16 tensors with unit stride in d and dense rows; returns (head_stride, rows)."""
     torch = _torch()
     hs = None
     for i, t in enumerate(ts):
-        _need(t, torch.bfloat16, f"{name}[{i}]", 3)
+        _need(t, torch.bfloat16, f"{name}[{i}]", 3, host=host)
         H, R, d = t.shape
         if t.stride(2) != 1 or (R > 1 and t.stride(1) != d):
             raise ValueError(f"{name}[{i}] rows must be dense (stride(1) == d, stride(2) == 1)")
@@ -470,6 +478,12 @@ class Problem:
     pos_in: object = None
     step_id_out: object = None
     pos_out: object = None
+    # STEPKV_MEM_HOST: K/V (or K_out/V_out) are pinned host tensors that the compaction reads (writes)
+    # over the CPU-GPU link; the saliency stage then reads K_sal (device copies of the last
+    # n_sal_layers layers' K)
+    kv_location: int = STEPKV_MEM_DEVICE
+    out_location: int = STEPKV_MEM_DEVICE
+    K_sal: Optional[List] = None
     _keep: list = field(default_factory=list, repr=False)
     _c: object = field(default=None, repr=False)
 
@@ -488,20 +502,28 @@ class Problem:
         torch = _torch()
         L = len(self.K)
         Ls = len(self.Q)
-        ks = _rows_layout(list(self.K) + list(self.V), "K/V")
+        kv_host = self.kv_location == STEPKV_MEM_HOST
+        ks = _rows_layout(list(self.K) + list(self.V), "K/V", host=kv_host)
         qs = _rows_layout(self.Q, "Q")
-        outs = _rows_layout(list(self.K_out) + list(self.V_out), "K_out/V_out")
+        outs = _rows_layout(list(self.K_out) + list(self.V_out), "K_out/V_out",
+                            host=self.out_location == STEPKV_MEM_HOST)
+        if kv_host:
+            if self.K_sal is None or len(self.K_sal) != Ls:
+                raise ValueError("a host-resident cache needs K_sal: device copies of the saliency layers' K")
+            if _rows_layout(self.K_sal, "K_sal") != ks:
+                raise ValueError("K_sal must share the head stride of K")
         Hkv, _, d = self.K[0].shape
         Hq, W, _ = self.Q[0].shape
         _need(self.step_id, torch.int32, "step_id", 1)
         _need(self.prot, torch.uint8, "prot", 1)
         arrs = [_ptr_array(self.K), _ptr_array(self.V), _ptr_array(self.Q), _ptr_array(self.K_out),
-                _ptr_array(self.V_out)]
+                _ptr_array(self.V_out), _ptr_array(self.K_sal or [])]
         self._keep = arrs
         cv = lambda a: ctypes.cast(a, ctypes.c_void_p)
         return CProblem(L, Hkv, Hq, d, self.T, W, Ls, cv(arrs[0]), cv(arrs[1]), ks, cv(arrs[2]), qs,
                         _ptr(self.step_id), _ptr(self.prot), _ptr(self.pos_in), self.steps.c(), self.budget,
-                        cv(arrs[3]), cv(arrs[4]), outs, _ptr(self.step_id_out), _ptr(self.pos_out), self.out.c())
+                        cv(arrs[3]), cv(arrs[4]), outs, _ptr(self.step_id_out), _ptr(self.pos_out), self.out.c(),
+                        self.kv_location, self.out_location, cv(arrs[5]) if kv_host else None)
 
 
 def stepkv_workspace_size(problems: Sequence[Problem]) -> int:

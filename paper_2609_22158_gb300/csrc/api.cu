@@ -44,6 +44,55 @@ cudaError_t ensure_smem_attr(const void* func, int bytes) {
   return e;
 }
 
+// Device-visible address of page-locked host memory (cudaHostAlloc / cudaHostRegister); false for any
+// other kind of pointer (device, managed, pageable).
+static bool host_pinned_device_ptr(const void* p, void** dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  if (a.type != cudaMemoryTypeHost || !a.devicePointer) return false;
+  *dev = a.devicePointer;
+  return true;
+}
+
+// A problem's cache pointers as the kernels see them: host-resident caches translated to their
+// device-visible addresses.
+struct CachePtrs {
+  std::vector<const void*> K, V;
+  std::vector<void*> K_out, V_out;
+};
+
+static stepkv_status_t resolve_cache_ptrs(const stepkv_problem_t& p, CachePtrs* c) {
+  if ((p.kv_location != STEPKV_MEM_DEVICE && p.kv_location != STEPKV_MEM_HOST) ||
+      (p.out_location != STEPKV_MEM_DEVICE && p.out_location != STEPKV_MEM_HOST))
+    return STEPKV_EINVAL;
+  c->K.assign(p.K, p.K + p.L);
+  c->V.assign(p.V, p.V + p.L);
+  c->K_out.assign(p.K_out, p.K_out + p.L);
+  c->V_out.assign(p.V_out, p.V_out + p.L);
+  auto tr_in = [](std::vector<const void*>& v) {
+    for (auto& x : v) {
+      void* d = nullptr;
+      if (!host_pinned_device_ptr(x, &d)) return false;
+      x = d;
+    }
+    return true;
+  };
+  auto tr_out = [](std::vector<void*>& v) {
+    for (auto& x : v) {
+      void* d = nullptr;
+      if (!host_pinned_device_ptr(x, &d)) return false;
+      x = d;
+    }
+    return true;
+  };
+  if (p.kv_location == STEPKV_MEM_HOST && !(tr_in(c->K) && tr_in(c->V))) return STEPKV_EINVAL;
+  if (p.out_location == STEPKV_MEM_HOST && !(tr_out(c->K_out) && tr_out(c->V_out))) return STEPKV_EINVAL;
+  return STEPKV_OK;
+}
+
 static size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -308,6 +357,12 @@ stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q, const void
                     static_cast<cudaStream_t>(stream));
 }
 
+// K of the saliency layers as the score stage reads it (device memory in either cache location).
+static const void* const* sal_keys(const stepkv_problem_t& p) {
+  const int Ls = std::min(p.n_sal_layers, p.L);
+  return p.kv_location == STEPKV_MEM_HOST ? p.K_sal : p.K + (p.L - Ls);
+}
+
 // Workspace of the fused pass: one region of pass-1 partials (the score launches run one after another
 // and reuse it), then per trajectory its fixed-point token saliency T_acc and its selection scratch
 // (all selections run in one batched launch, so these are private).
@@ -344,7 +399,8 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     const int Ls = std::min(p.n_sal_layers, p.L);
     if (Ls > kMaxSalLayers) return STEPKV_EUNSUPPORTED;
     if (!p.K || !p.Q) return STEPKV_EINVAL;
-    stepkv_status_t st = check_score_args(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq,
+    if (p.kv_location == STEPKV_MEM_HOST && !p.K_sal) return STEPKV_EINVAL;
+    stepkv_status_t st = check_score_args(Ls, sal_keys(p), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq,
                                           p.d, p.T, p.W);
     if (st != STEPKV_OK) return st;
     st = check_select_args(Ls * p.Hkv, p.T, p.step_id, p.prot, &p.steps, params, &p.budget, &p.sel);
@@ -352,6 +408,13 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     bool inplace = false;
     st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
                             p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
+    if (st != STEPKV_OK) return st;
+    if (inplace && p.kv_location != p.out_location) return STEPKV_EINVAL;
+  }
+  // cache pointers as the kernels see them (host-resident caches: checked and translated here)
+  std::vector<CachePtrs> caches((size_t)n_traj);
+  for (int i = 0; i < n_traj; ++i) {
+    stepkv_status_t st = resolve_cache_ptrs(probs[i], &caches[i]);
     if (st != STEPKV_OK) return st;
   }
   if (ws_bytes < stepkv_compress_workspace_size(probs, n_traj)) return STEPKV_ENOSPACE;
@@ -372,7 +435,7 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     w += compress_traj_bytes(p);
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
-    stepkv_status_t st = score_run(Ls, p.K + (p.L - Ls), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
+    stepkv_status_t st = score_run(Ls, sal_keys(p), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
                                    p.T, p.W, nullptr, 0, t_acc, shift, part, dev_status, s);
     if (st != STEPKV_OK) return st;
     specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
@@ -387,16 +450,17 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     bool inplace = false;
     check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
                        p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
+    const CachePtrs& c = caches[i];
     if (inplace) {
-      st = compact_inplace_run(p.L, p.K_out, p.V_out, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
-                               p.sel.kept_cap, p.step_id, p.pos_in, p.step_id_out, p.pos_out, plan_ws[i], dev_status,
-                               s);
+      st = compact_inplace_run(p.L, c.K_out.data(), c.V_out.data(), p.kv_head_stride, p.Hkv, p.d, p.T,
+                               p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap, p.step_id, p.pos_in, p.step_id_out,
+                               p.pos_out, plan_ws[i], dev_status, s);
       if (st != STEPKV_OK) return st;
       continue;
     }
-    st = compact_run(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap,
-                     p.K_out, p.V_out, p.out_head_stride, p.step_id, p.pos_in, p.step_id_out, p.pos_out, dev_status,
-                     s);
+    st = compact_run(p.L, c.K.data(), c.V.data(), p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
+                     p.sel.kept_cap, c.K_out.data(), c.V_out.data(), p.out_head_stride, p.step_id, p.pos_in,
+                     p.step_id_out, p.pos_out, dev_status, s);
     if (st != STEPKV_OK) return st;
   }
   return STEPKV_OK;

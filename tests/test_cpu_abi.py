@@ -131,3 +131,36 @@ def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2609_22158_gb300 import binding
     with pytest.raises(binding.StepKVError):
         binding.load_library(str(tmp_path / "missing.so"))
+
+
+def test_ctypes_structs_mirror_the_header(tmp_path):
+    """The binding's ctypes structs have the size and field offsets of the C structs in include/stepkv.h
+    (compiled here with the system C compiler), so a struct passed through the ABI is read as written."""
+    import shutil
+    import subprocess
+    from paper_2609_22158_gb300 import binding as B
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    mirrors = {"stepkv_params_t": B.CParams, "stepkv_budget_t": B.CBudget, "stepkv_steps_t": B.CSteps,
+               "stepkv_select_out_t": B.CSelOut, "stepkv_problem_t": B.CProblem}
+    c_names = {"lambda_": "lambda"}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "stepkv.h"', 'int main(void) {']
+    for cname, py in mirrors.items():
+        lines.append(f'  printf("{cname} size %zu\\n", sizeof({cname}));')
+        for f, _ in py._fields_:
+            lines.append(f'  printf("{cname} {f} %zu\\n", offsetof({cname}, {c_names.get(f, f)}));')
+    lines += ['  return 0;', '}']
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    subprocess.run([cc, "-std=c99", "-I", inc, str(src), "-o", str(exe)], check=True)
+    got = {}
+    for ln in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.splitlines():
+        name, field, val = ln.split()
+        got[(name, field)] = int(val)
+    for cname, py in mirrors.items():
+        assert got[(cname, "size")] == ctypes.sizeof(py), cname
+        for f, _ in py._fields_:
+            assert got[(cname, f)] == getattr(py, f).offset, (cname, f)

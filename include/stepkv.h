@@ -305,6 +305,20 @@ STEPKV_API stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q,
                               float* const* out, void* ws, size_t ws_bytes, int32_t* dev_status,
                               void* stream);
 
+/* Failure-detection self-test (no counterpart in the paper).  Runs the saliency kernel of stepkv_score
+ * on the same arguments, except that the wait of its second pass (for every CTA's first-pass flag)
+ * looks for a value no CTA ever publishes, so every CTA's wait runs out after wait_limit_ns
+ * (1 us .. 1 s).  The kernel then records STEPKV_ETIMEOUT in *dev_status (caller-zeroed), drains its
+ * own TMA copies and tensor-core operations, frees its tensor memory and returns: the CUDA context
+ * stays usable and later calls on the stream run normally.  sal is left undefined.  Supported when
+ * G * W <= 256 (one row group); else STEPKV_EUNSUPPORTED.  ws as for stepkv_score.
+ */
+STEPKV_API stepkv_status_t stepkv_selftest_score_timeout(int32_t n_layers, const void* const* K,
+                                              int64_t k_head_stride, const void* const* Q,
+                                              int64_t q_head_stride, int32_t Hkv, int32_t Hq, int32_t d,
+                                              int32_t T, int32_t W, float* sal, void* ws, size_t ws_bytes,
+                                              uint64_t wait_limit_ns, int32_t* dev_status, void* stream);
+
 /* ---------------------------------------------------------------------------------------------
  * The fused pass (score -> reduce/fuse -> select -> compact) for n_traj independent trajectories
  * (one pruning boundary each, Algorithm 1).  probs is a host array; everything runs on `stream`:

@@ -79,6 +79,8 @@ SIGNATURES = {
     "stepkv_last_cuda_error": (ctypes.c_char_p, []),
     "stepkv_score_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
     "stepkv_score": (_I32, [_I32, _VP, _I64, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ, _VP, _VP]),
+    "stepkv_selftest_score_timeout": (_I32, [_I32, _VP, _I64, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ,
+                                             ctypes.c_uint64, _VP, _VP]),
     "stepkv_select_workspace_size": (_SZ, [_I32, _I32, _I32]),
     "stepkv_select": (_I32, [_VP, _I32, _I32, _VP, _VP, ctypes.POINTER(CSteps), ctypes.POINTER(CParams),
                              ctypes.POINTER(CBudget), ctypes.POINTER(CSelOut), _VP, _SZ, _VP, _VP]),
@@ -259,6 +261,30 @@ def stepkv_score(K: Sequence, Q: Sequence, T: int, W: Optional[int] = None, sal=
                             T, W, sal.data_ptr(), wp, wn, status.data_ptr(), _stream_handle(stream))
     _check(code, "stepkv_score")
     return sal
+
+
+def stepkv_selftest_score_timeout(K: Sequence, Q: Sequence, T: int, wait_limit_ns: int, status, W=None,
+                                  stream=None):
+    """Failure-path self-test: the saliency kernel with a second-pass wait that runs out after
+    wait_limit_ns; STEPKV_ETIMEOUT lands in `status` (caller-zeroed device int32) and the kernel returns."""
+    torch = _torch()
+    lib = load_library()
+    n = len(K)
+    ks = _rows_layout(K, "K")
+    qs = _rows_layout(Q, "Q")
+    Hkv, _, d = K[0].shape
+    Hq, Wq, _ = Q[0].shape
+    W = Wq if W is None else W
+    dev = K[0].device
+    sal = torch.empty((n, Hkv, T), dtype=torch.float32, device=dev)
+    ws = _workspace(lib.stepkv_score_workspace_size(n, Hkv, Hq, T, W) + 256, None, dev)
+    wp, wn = _aligned_ws(ws)
+    kp, qp = _ptr_array(K), _ptr_array(Q)
+    code = lib.stepkv_selftest_score_timeout(n, ctypes.cast(kp, ctypes.c_void_p), ks, ctypes.cast(qp, ctypes.c_void_p),
+                                             qs, Hkv, Hq, d, T, W, sal.data_ptr(), wp, wn, int(wait_limit_ns),
+                                             status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_selftest_score_timeout")
+    return ws
 
 
 # ----------------------------------------------------------------------------- stages 2-4

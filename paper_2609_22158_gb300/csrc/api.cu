@@ -239,6 +239,21 @@ stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_h
   return st;
 }
 
+stepkv_status_t stepkv_selftest_score_timeout(int32_t n_layers, const void* const* K, int64_t k_head_stride,
+                                              const void* const* Q, int64_t q_head_stride, int32_t Hkv, int32_t Hq,
+                                              int32_t d, int32_t T, int32_t W, float* sal, void* ws, size_t ws_bytes,
+                                              uint64_t wait_limit_ns, int32_t* dev_status, void* stream) {
+  stepkv_status_t st = check_score_args(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W);
+  if (st != STEPKV_OK) return st;
+  if (!sal || !ws || !dev_status) return STEPKV_EINVAL;
+  if (wait_limit_ns < 1000 || wait_limit_ns > kWaitLimitNs) return STEPKV_EINVAL;
+  if (ws_bytes < score_ws(n_layers, Hkv, Hq, T, W, false)) return STEPKV_ENOSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
+  if (score_row_groups(Hkv, Hq, W) != 1) return STEPKV_EUNSUPPORTED;  // G*W <= 256: rows straight into sal
+  return score_run(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W, sal, T, nullptr, 0,
+                   static_cast<float2*>(ws), dev_status, static_cast<cudaStream_t>(stream), wait_limit_ns);
+}
+
 size_t stepkv_select_workspace_size(int32_t n_sal, int32_t T, int32_t n_steps) {
   (void)n_sal;
   if (T < 1 || n_steps < 1) return 0;

@@ -95,7 +95,7 @@ int score_acc_shift(int n_pairs, int W);
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
                           int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
-                          cudaStream_t stream);
+                          cudaStream_t stream, unsigned long long selftest_wait_ns = 0);
 stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal, cudaStream_t stream);
 
 // ---- select (select.cu)

@@ -65,6 +65,8 @@ struct ScoreLaunch {
   int zero_acc;       // zero t_acc[0..T) before any contribution is added
   unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores `token` once its partials are written
   unsigned long long token;   // unique per launch, so flags left by earlier launches never match
+  unsigned long long wait_token;     // the value the pass-2 wait looks for (token, except in the self-test)
+  unsigned long long wait_limit_ns;  // the pass-2 wait gives up (STEPKV_ETIMEOUT) after this long
   int32_t* status;
 };
 
@@ -594,9 +596,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
               for (uint32_t it = 0; !all; ++it) {
                 bool mine = true;
 #pragma unroll 4
-                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.token;
+                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.wait_token;
                 all = __all_sync(0xffffffffu, mine);
-                if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > kWaitLimitNs)) break;
+                if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > p.wait_limit_ns)) break;
               }
               fence_acquire_gpu();
               if (!all) {
@@ -845,7 +847,7 @@ static cudaError_t launch_score(const ScoreLaunch& L, int grid, cudaStream_t str
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
                           int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, unsigned long long selftest_wait_ns) {
   const ScoreGeom g = make_geom(Hkv, Hq, d, T, W);
   ScoreLaunch L;
   memset(&L, 0, sizeof(L));
@@ -877,6 +879,10 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   L.tpc = (U + grid0 - 1) / grid0;
   const int grid = (U + L.tpc - 1) / L.tpc;
   L.token = next_launch_token();
+  // Self-test of the failure path: the pass-2 wait looks for a value no CTA ever publishes, so every
+  // CTA's wait runs out after selftest_wait_ns and the kernel takes its abort path.
+  L.wait_token = selftest_wait_ns ? ~L.token : L.token;
+  L.wait_limit_ns = selftest_wait_ns ? selftest_wait_ns : kWaitLimitNs;
   e = d == 128 ? launch_score<2>(L, grid, stream) : launch_score<1>(L, grid, stream);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   return STEPKV_OK;

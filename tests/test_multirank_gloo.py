@@ -74,3 +74,38 @@ def test_single_process_defaults(monkeypatch):
     assert MR.gather_tokens(123) == [123]
     with pytest.raises(ValueError):
         MR.job_throughput([1], 0.0)
+
+
+def _failing_worker(rank, world, port, q):
+    import datetime
+    import torch.distributed as dist
+    os.environ.update({"WORLD_SIZE": str(world), "RANK": str(rank), "LOCAL_RANK": str(rank),
+                       "MASTER_ADDR": "127.0.0.1", "MASTER_PORT": str(port)})
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world,
+                            timeout=datetime.timedelta(seconds=10))
+    if rank == 1:
+        # this rank fails between steps, before the timing exchange: it never joins the collective
+        q.put((rank, "raised"))
+        raise SystemExit(3)
+    try:
+        MR.max_over_ranks(1.0, dist)
+        q.put((rank, "no error"))
+    except Exception as e:  # the surviving rank learns of it from its next collective
+        q.put((rank, "detected: " + type(e).__name__))
+
+
+def test_a_failed_rank_is_detected_by_the_next_collective():
+    """A rank that leaves between steps (an exception on the host, no GPU involved) makes the other
+    rank's next timing exchange fail with an error instead of hanging."""
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_failing_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = dict(q.get(timeout=120) for _ in range(2))
+    for p in procs:
+        p.join(timeout=60)
+    assert res[1] == "raised" and procs[1].exitcode == 3
+    assert res[0].startswith("detected"), res[0]

@@ -378,12 +378,47 @@ static const void* const* sal_keys(const stepkv_problem_t& p) {
   return p.kv_location == STEPKV_MEM_HOST ? p.K_sal : p.K + (p.L - Ls);
 }
 
-// Workspace of the fused pass: one region of pass-1 partials (the score launches run one after another
-// and reuse it), then per trajectory its fixed-point token saliency T_acc and its selection scratch
-// (all selections run in one batched launch, so these are private).
-static size_t compress_part_bytes(const stepkv_problem_t& p) {
+// Saliency batches of the fused pass: runs of consecutive trajectories with one head shape (lengths and
+// strides may differ), up to kMaxScoreBatch trajectories and kMaxScoreMaps tensor maps each, share one
+// launch -- as long as the batch's saliency keys fit in half of L2.  The second pass walks each CTA's
+// tiles backwards and finds the ones the first pass read last still in L2; a trajectory whose keys fit
+// in L2 gets all of them there when it runs alone, and a batch only pays if that still holds, so short
+// trajectories (where the launch's fixed costs dominate) are batched and long ones run one per launch.
+constexpr size_t kSalBatchBytes = 64ull << 20;
+struct SalBatch {
+  int first, n;
+};
+static size_t sal_key_bytes(const stepkv_problem_t& p) {
+  return (size_t)std::min(p.n_sal_layers, p.L) * p.Hkv * p.T * p.d * 2;
+}
+static std::vector<SalBatch> saliency_batches(const stepkv_problem_t* probs, int n_traj) {
+  std::vector<SalBatch> out;
+  auto same = [](const stepkv_problem_t& a, const stepkv_problem_t& b) {
+    return std::min(a.n_sal_layers, a.L) == std::min(b.n_sal_layers, b.L) && a.Hkv == b.Hkv && a.Hq == b.Hq &&
+           a.d == b.d && a.W == b.W;
+  };
+  for (int i = 0; i < n_traj;) {
+    const int Ls = std::max(1, std::min(probs[i].n_sal_layers, probs[i].L));
+    int n = 1;
+    size_t bytes = sal_key_bytes(probs[i]);
+    while (i + n < n_traj && n < kMaxScoreBatch && (n + 1) * Ls <= kMaxScoreMaps && same(probs[i], probs[i + n]) &&
+           bytes + sal_key_bytes(probs[i + n]) <= kSalBatchBytes) {
+      bytes += sal_key_bytes(probs[i + n]);
+      ++n;
+    }
+    out.push_back(SalBatch{i, n});
+    i += n;
+  }
+  return out;
+}
+
+// Workspace of the fused pass: one region of pass-1 partials (the saliency launches run one after
+// another and reuse it; sized for the largest batch), then per trajectory its fixed-point token
+// saliency T_acc and its selection scratch (all selections run in one batched launch, so these are
+// private).
+static size_t compress_part_bytes(const stepkv_problem_t& p, int n_batch) {
   const int Ls = std::min(p.n_sal_layers, p.L);
-  return align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W));
+  return align256(score_partial_bytes(Ls, p.Hkv, p.Hq, p.W, n_batch));
 }
 static size_t compress_traj_bytes(const stepkv_problem_t& p) {
   return align256((size_t)p.T * sizeof(unsigned long long)) + align256(select_ws_bytes(p.T, p.steps.n_steps)) +
@@ -397,9 +432,10 @@ size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_t
     const stepkv_problem_t& p = probs[i];
     if (p.L < 1 || p.Hkv < 1 || p.Hq < p.Hkv || p.T < 1 || p.W < 1 || p.n_sal_layers < 1 || p.steps.n_steps < 1)
       return 0;
-    part = std::max(part, compress_part_bytes(p));
     per += compress_traj_bytes(p);
   }
+  for (const SalBatch& b : saliency_batches(probs, n_traj))
+    part = std::max(part, compress_part_bytes(probs[b.first], b.n));
   return part + per;
 }
 
@@ -434,13 +470,14 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   }
   if (ws_bytes < stepkv_compress_workspace_size(probs, n_traj)) return STEPKV_ENOSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const std::vector<SalBatch> batches = saliency_batches(probs, n_traj);
   size_t part_bytes = 0;
-  for (int i = 0; i < n_traj; ++i) part_bytes = std::max(part_bytes, compress_part_bytes(probs[i]));
+  for (const SalBatch& b : batches) part_bytes = std::max(part_bytes, compress_part_bytes(probs[b.first], b.n));
   float2* part = reinterpret_cast<float2*>(ws);
   uint8_t* w = static_cast<uint8_t*>(ws) + part_bytes;
   std::vector<SelectSpec> specs((size_t)n_traj);
   std::vector<void*> plan_ws((size_t)n_traj);
-  // stage 1 for every trajectory (one cooperative launch each)
+  std::vector<ScoreTrajSpec> sal((size_t)n_traj);
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     const int Ls = std::min(p.n_sal_layers, p.L);
@@ -450,11 +487,17 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     w += compress_traj_bytes(p);
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
-    stepkv_status_t st = score_run(Ls, sal_keys(p), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d,
-                                   p.T, p.W, nullptr, 0, t_acc, shift, part, dev_status, s);
-    if (st != STEPKV_OK) return st;
+    sal[i] = ScoreTrajSpec{sal_keys(p), p.Q, p.T, t_acc, p.kv_head_stride, p.q_head_stride};
     specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
                           *params, p.budget, p.sel, sel_ws, dev_status};
+  }
+  // stage 1: one cooperative launch per saliency batch
+  for (const SalBatch& b : batches) {
+    const stepkv_problem_t& p = probs[b.first];
+    const int Ls = std::min(p.n_sal_layers, p.L);
+    stepkv_status_t st = score_run_batch(Ls, &sal[b.first], b.n, p.Hkv, p.Hq, p.d, p.W, nullptr, 0,
+                                         score_acc_shift(Ls * p.Hkv, p.W), part, dev_status, s);
+    if (st != STEPKV_OK) return st;
   }
   // stages 2-4 for all trajectories in one launch (one cluster per trajectory)
   stepkv_status_t st = select_run_batch(specs.data(), n_traj, s);

@@ -13,6 +13,8 @@
 namespace stepkv {
 
 constexpr int kMaxSalLayers = 8;        // saliency layers per score launch (tensor maps in kernel params)
+constexpr int kMaxScoreBatch = 16;      // trajectories per saliency launch
+constexpr int kMaxScoreMaps = 48;       // trajectories x saliency layers per saliency launch
 constexpr int kMaxGrid = 1024;          // upper bound on the persistent score grid (partial-slot sizing)
 constexpr int kMaxCompactLayers = 256;  // layers per compaction launch (pointer tables in kernel params)
 
@@ -87,11 +89,25 @@ stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const
 
 // ---- score (score.cu)
 int score_row_groups(int Hkv, int Hq, int W);
-size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W);
+size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W, int n_traj = 1);
 int score_acc_shift(int n_pairs, int W);
 // Pass 2 either writes rows (row pair*n_rg + rg of rows_out, stride out_stride, pair = layer*Hkv + h) or,
 // when t_acc is non-null, adds every contribution to the per-token fixed-point sum t_acc[T] (scale
 // 2^acc_shift; the first launch zeroes it).
+// One trajectory of a batched saliency launch (per-layer device pointers, tokens, accumulator).
+struct ScoreTrajSpec {
+  const void* const* K;
+  const void* const* Q;
+  int T;
+  unsigned long long* t_acc;
+  int64_t k_head_stride, q_head_stride;
+};
+// Saliency of n_traj trajectories of one head shape in one cooperative launch (n_traj <= kMaxScoreBatch,
+// n_traj * n_layers <= kMaxScoreMaps); rows output only for n_traj == 1.
+stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_traj, int Hkv, int Hq, int d,
+                                int W, float* rows_out,
+                                int64_t out_stride, int acc_shift, float2* part, int32_t* status, cudaStream_t stream,
+                                unsigned long long selftest_wait_ns = 0);
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
                           int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,

@@ -49,20 +49,30 @@ struct ScoreGeom {
   float inv_G;
 };
 
+// One trajectory of a batched launch: its items are [item_off, item_off + units_per * n_tiles).
+struct ScoreTraj {
+  int T;
+  int n_tiles;                 // ceil(T / 128)
+  int item_off;
+  unsigned long long* t_acc;   // pass 2: per-token fixed-point sum (when the launch accumulates)
+};
+
 struct ScoreLaunch {
-  CUtensorMap tmK[kMaxSalLayers];
-  CUtensorMap tmQ[kMaxSalLayers];
-  ScoreGeom g;
+  CUtensorMap tmK[kMaxScoreMaps];  // [traj * n_layers + layer]
+  CUtensorMap tmQ[kMaxScoreMaps];
+  ScoreTraj traj[kMaxScoreBatch];
+  ScoreGeom g;                     // shared head geometry (T, n_tiles: see traj)
+  int n_traj;
   int n_layers;
-  int pair0;          // first (layer*Hkv + head) pair of this launch
-  int n_units;        // units = pairs of this launch x n_rg
+  int pair0;          // first (layer*Hkv + head) pair of this launch (rows output)
+  int units_per;      // units per trajectory = n_layers x Hkv x n_rg
+  int n_items;        // items of all trajectories
   int tpc;            // tiles per CTA (contiguous range)
   float2* part;       // pass-1 partials: slot (unit + cta) x 256 rows
-  float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when t_acc == nullptr)
+  float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when not accumulating)
   int64_t out_stride;
-  unsigned long long* t_acc;  // pass 2: per-token fixed-point sum over all (pair, row group) (when non-null)
+  int accumulate;     // 1: pass 2 adds into each trajectory's t_acc (zeroed first) instead of writing rows
   int acc_shift;      // k: fixed-point scale 2^k of t_acc
-  int zero_acc;       // zero t_acc[0..T) before any contribution is added
   unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores `token` once its partials are written
   unsigned long long token;   // unique per launch, so flags left by earlier launches never match
   unsigned long long wait_token;     // the value the pass-2 wait looks for (token, except in the self-test)
@@ -93,6 +103,29 @@ __host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
   }
   r.rows = r.n_blk * r.blk_rows;
   return r;
+}
+
+// Where global item t of a launch sits: trajectory b, local unit ul (global unit b * units_per + ul),
+// key tile of the unit.
+struct ItemLoc {
+  int b, ul, u, tile;
+};
+__device__ __forceinline__ ItemLoc locate(const ScoreLaunch& p, int t) {
+  int b = 0;
+  while (b + 1 < p.n_traj && p.traj[b + 1].item_off <= t) ++b;
+  const int local = t - p.traj[b].item_off;
+  const int nt = p.traj[b].n_tiles;
+  ItemLoc r;
+  r.b = b;
+  r.ul = local / nt;
+  r.tile = local - r.ul * nt;
+  r.u = b * p.units_per + r.ul;
+  return r;
+}
+// First item of global unit u.
+__device__ __forceinline__ int unit_first_item(const ScoreLaunch& p, int u) {
+  const int b = u / p.units_per, ul = u - b * p.units_per;
+  return p.traj[b].item_off + ul * p.traj[b].n_tiles;
 }
 
 // Shared memory of the kernel.
@@ -271,12 +304,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 
   const ScoreGeom& g = p.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int U = p.n_units * g.n_tiles;
+  const int U = p.n_items;
   const int t_lo = blockIdx.x * p.tpc;
   const int t_hi = min(U, t_lo + p.tpc);
   const int n1 = max(0, t_hi - t_lo);  // tiles of the CTA (each is streamed once per pass)
   // Pass-1 items: two consecutive tiles of one unit where possible, else one.
-  auto item_tiles = [&](int t) { return (t + 1 < t_hi && (t + 1) / g.n_tiles == t / g.n_tiles) ? 2 : 1; };
+  auto item_tiles = [&](const ItemLoc& l, int t) {
+    return (t + 1 < t_hi && l.tile + 1 < p.traj[l.b].n_tiles) ? 2 : 1;
+  };
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < Cfg::kStages; ++i) {
@@ -295,7 +330,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     mbar_fence_init();
   }
   if (warp == 0 && lane == 0) {
-    for (int l = 0; l < p.n_layers; ++l) {
+    for (int l = 0; l < p.n_traj * p.n_layers; ++l) {
       tma_prefetch_desc(&p.tmK[l]);
       tma_prefetch_desc(&p.tmQ[l]);
     }
@@ -321,9 +356,11 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       uint32_t par = 0, used = 0;  // per stage: parity of its next use / loaded at least once
       bool ok = true;
       auto load_tile = [&](int gt, int st) -> bool {
-        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
-        const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
+        const ItemLoc il = locate(p, gt);
+        const int u = il.u, tile = il.tile;
+        const int pair = p.pair0 + il.ul / g.n_rg, rg = il.ul % g.n_rg;
         const int layer = pair / g.Hkv, h = pair - layer * g.Hkv;
+        const int map = il.b * p.n_layers + layer;
         if (u != cur) {
           if (cur >= 0) {
             if (!mbar_wait(q_empty, qe_phase, abort_flag)) return false;
@@ -334,7 +371,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           mbar_arrive_expect_tx(q_full, (uint32_t)(r.n_blk * NCH * box_rows * 128));
           for (int b = 0; b < r.n_blk; ++b)
             for (int c = 0; c < NCH; ++c)
-              tma_load_3d(sQ + c * kQChunkBytes + b * r.blk_rows * 128, &p.tmQ[layer], c * 64, r.w0,
+              tma_load_3d(sQ + c * kQChunkBytes + b * r.blk_rows * 128, &p.tmQ[map], c * 64, r.w0,
                           h * g.G + r.g_first + b, q_full);
           ++q_issued;
           cur = u;
@@ -343,14 +380,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         if (!mbar_wait(&k_empty[st], ph ^ 1u, abort_flag)) return false;
         mbar_arrive_expect_tx(&k_full[st], (uint32_t)(NCH * kKChunkBytes));
         for (int c = 0; c < NCH; ++c)
-          tma_load_3d(sK + Cfg::chunk_off(st, c), &p.tmK[layer], c * 64, tile * kKeyTile, h, &k_full[st]);
+          tma_load_3d(sK + Cfg::chunk_off(st, c), &p.tmK[map], c * 64, tile * kKeyTile, h, &k_full[st]);
         used |= 1u << st;
         par ^= 1u << st;
         return true;
       };
       int slot = 0;
       for (int t = t_lo; t < t_hi && ok;) {
-        const int nt = item_tiles(t);
+        const int nt = item_tiles(locate(p, t), t);
         for (int i = 0; i < nt && ok; ++i) ok = load_tile(t + i, 2 * slot + i);
         t += nt;
         if (++slot == P1) slot = 0;
@@ -395,8 +432,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       // pass 1: S = Q K^T, one half per 128-row query tile, N = the item's keys (256 or 128)
       int slot = 0;
       for (int t = t_lo; t < t_hi && ok;) {
-        const int nt = item_tiles(t);
-        const int u = t / g.n_tiles;
+        const ItemLoc il = locate(p, t);
+        const int nt = item_tiles(il, t);
+        const int u = il.u;
         const RowGroup r = row_group(g, u % g.n_rg);
         if (!(ok = new_unit(u))) break;
         for (int i = 0; i < nt && ok; ++i) {
@@ -430,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       }
       // pass 2: S^T = K Q^T, the tile's keys on M, the query rows on N
       for (int k = 0; k < n1 && ok; ++k) {
-        const int u = (t_hi - 1 - k) / g.n_tiles;
+        const int u = locate(p, t_hi - 1 - k).u;
         const RowGroup r = row_group(g, u % g.n_rg);
         if (!(ok = new_unit(u))) break;
         int b;
@@ -485,14 +523,18 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     // The epilogue warps zero this CTA's share of t_acc while the first tiles stream in.  The stores
     // precede the warp's p1_flushed arrival, so the publisher's fence orders them before the CTA's flag,
     // hence before any pass-2 addition by any CTA.
-    if (p.zero_acc) {
-      for (int i = blockIdx.x * (kEpiWarps * 32) + (threadIdx.x - 64); i < g.T; i += gridDim.x * (kEpiWarps * 32))
-        p.t_acc[i] = 0ull;
+    if (p.accumulate) {
+      for (int b = 0; b < p.n_traj; ++b) {
+        unsigned long long* acc = p.traj[b].t_acc;
+        for (int i = blockIdx.x * (kEpiWarps * 32) + (threadIdx.x - 64); i < p.traj[b].T;
+             i += gridDim.x * (kEpiWarps * 32))
+          acc[i] = 0ull;
+      }
     }
 
     // ---- pass 1: per-row running (m, Z) over the keys this warp sees
     {
-      int cur = -1;
+      int cur = -1, Tb = 0;
       float m = -INFINITY, Z = 0.f;
       int my_row = 0, my_pw = 0, my_e = 0;
       bool row_ok = false, two = false;
@@ -501,10 +543,12 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         p.part[((size_t)(u + (int)blockIdx.x) * kPartEntries + my_e) * kMaxRows + my_row] = make_float2(m, Z);
       };
       for (int t = t_lo; t < t_hi && ok;) {
-        const int nt = item_tiles(t);
-        const int u = t / g.n_tiles, tile = t - u * g.n_tiles;
+        const ItemLoc il = locate(p, t);
+        const int nt = item_tiles(il, t);
+        const int u = il.u, tile = il.tile;
         t += nt;
         if (u != cur) {
+          Tb = p.traj[il.b].T;
           // Every warp flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
           // so each of the unit's partial entries is written.
           if (cur >= 0) flush_partial(cur);
@@ -518,7 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           my_e = two ? s2 : grp * 2 + s2;
           const int w = r.w0 + my_row % r.blk_rows;
           row_ok = my_row < r.rows && w < g.W;
-          my_pw = g.T - g.W + w;
+          my_pw = Tb - g.W + w;
           m = -INFINITY;
           Z = 0.f;
           cur = u;
@@ -534,7 +578,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         // chunks (one TMEM round trip per pair); the buffer is released once the last pair is loaded.
         const int half_keys = nt * 64;
         const int key0 = tile * kKeyTile + s2 * half_keys;
-        const bool need_mask = key0 + half_keys - 1 > g.T - g.W;  // reaches into the causal window
+        const bool need_mask = key0 + half_keys - 1 > Tb - g.W;  // reaches into the causal window
         const int n_pairs_ch = half_keys / 64;
 #pragma unroll 1
         for (int h2 = 0; h2 < n_pairs_ch; ++h2) {
@@ -585,7 +629,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       for (int k = 0; k < n1 && ok; ++k, ++hh) {
         if ((hh & 1u) != (uint32_t)grp) continue;
         const int gt = t_hi - 1 - k;
-        const int u = gt / g.n_tiles, tile = gt - u * g.n_tiles;
+        const ItemLoc il = locate(p, gt);
+        const int u = il.u, tile = il.tile;
+        const int Tb = p.traj[il.b].T;
         if (u != cur) {
           if (!others_done) {
             // Wait until every CTA has published its pass-1 partials (and zeroed its share of t_acc).
@@ -612,8 +658,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           // order (the group no longer reads the previous unit's offsets once all its warps arrive).
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
           r = row_group(g, u % g.n_rg);
-          const int c0 = (u * g.n_tiles) / p.tpc;
-          const int c1 = (u * g.n_tiles + g.n_tiles - 1) / p.tpc;
+          const int f0 = unit_first_item(p, u);
+          const int c0 = f0 / p.tpc;
+          const int c1 = (f0 + p.traj[il.b].n_tiles - 1) / p.tpc;
           const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
           const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
           const int w = r.w0 + row % r.blk_rows;
@@ -648,7 +695,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             off = M * c + __log2f(Zs);
           }
           negoff[row] = -off;
-          pw_tab[row] = valid ? g.T - g.W + w : -1;
+          pw_tab[row] = valid ? Tb - g.W + w : -1;
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
           cur = u;
         }
@@ -656,7 +703,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         acc_phase ^= 1;
         tc_fence_after();
         const int key0 = tile * kKeyTile;
-        const bool need_mask = key0 + kKeyTile - 1 > g.T - g.W;  // tile reaches into the causal window
+        const bool need_mask = key0 + kKeyTile - 1 > Tb - g.W;  // tile reaches into the causal window
         // Keys on the TMEM lanes: this warp sums its key's mass over query columns s2*32 + 64 i, one
         // 32-column chunk at a time (holding two chunks in registers spills).  The buffer is released
         // once the warp's last chunk is in registers.
@@ -675,19 +722,19 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           acc += key_mass(v, negoff + cc, pw_tab + cc, j, need_mask, c);
         }
         if (!released) release_buffer();
-        if (p.t_acc) {
+        if (p.accumulate) {
           // fused pass: each warp adds its share of the rows straight into the per-token fixed-point
           // sum (integer addition: the total does not depend on the order of arrival)
-          if (j < g.T) atomicAdd(&p.t_acc[j], to_fixed(acc * g.inv_G, p.acc_shift));
+          if (j < Tb) atomicAdd(&p.traj[il.b].t_acc[j], to_fixed(acc * g.inv_G, p.acc_shift));
         } else {
           // saliency rows: the group's two warps on this quarter combine in a fixed order (the slot
           // alternates between the group's items, so a write never meets a pending read)
           float* comb = combf + (n_done & 1) * 128;
           if (s2 == 1) comb[q * 32 + lane] = acc;
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
-          if (s2 == 0 && j < g.T) {
+          if (s2 == 0 && j < Tb) {
             const float val = (acc + comb[q * 32 + lane]) * g.inv_G;
-            const int pair = p.pair0 + u / g.n_rg, rg = u % g.n_rg;
+            const int pair = p.pair0 + il.ul / g.n_rg, rg = il.ul % g.n_rg;
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }
         }
@@ -765,13 +812,14 @@ int score_acc_shift(int n_pairs, int W) {
   return 60 - e;
 }
 
-// Pass-1 partial slots, then one pass-1-done flag per CTA.
-static size_t score_partial_slots_bytes(int n_layers, int Hkv, int Hq, int W) {
+// Pass-1 partial slots (one per (unit, CTA) pair a launch can form: units + grid), then one
+// pass-1-done flag per CTA.
+static size_t score_partial_slots_bytes(int n_traj, int n_layers, int Hkv, int Hq, int W) {
   const int n_rg = score_row_groups(Hkv, Hq, W);
-  return (size_t)(n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
+  return (size_t)(n_traj * n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
 }
-size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W) {
-  return score_partial_slots_bytes(n_layers, Hkv, Hq, W) + (size_t)kMaxGrid * sizeof(unsigned long long);
+size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W, int n_traj) {
+  return score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W) + (size_t)kMaxGrid * sizeof(unsigned long long);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -844,40 +892,51 @@ static cudaError_t launch_score(const ScoreLaunch& L, int grid, cudaStream_t str
   return cudaLaunchKernelEx(&cfg, kern, L);
 }
 
-stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
-                          int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
-                          int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
-                          cudaStream_t stream, unsigned long long selftest_wait_ns) {
-  const ScoreGeom g = make_geom(Hkv, Hq, d, T, W);
+stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_traj, int Hkv, int Hq, int d,
+                                int W, float* rows_out,
+                                int64_t out_stride, int acc_shift, float2* part, int32_t* status, cudaStream_t stream,
+                                unsigned long long selftest_wait_ns) {
+  if (n_traj < 1 || n_traj > kMaxScoreBatch || n_traj * n_layers > kMaxScoreMaps) return STEPKV_EUNSUPPORTED;
+  const ScoreGeom g = make_geom(Hkv, Hq, d, trajs[0].T, W);
   ScoreLaunch L;
   memset(&L, 0, sizeof(L));
   L.g = g;
+  L.n_traj = n_traj;
   L.n_layers = n_layers;
+  L.units_per = n_layers * Hkv * g.n_rg;
   L.part = part;
   L.flags = reinterpret_cast<unsigned long long*>(reinterpret_cast<uint8_t*>(part) +
-                                                  score_partial_slots_bytes(n_layers, Hkv, Hq, W));
+                                                  score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W));
   L.out = rows_out;
   L.out_stride = out_stride;
-  L.t_acc = t_acc;
+  L.accumulate = trajs[0].t_acc != nullptr ? 1 : 0;
   L.acc_shift = acc_shift;
   L.status = status;
   const int box_rows = std::min(g.W_pad, kMaxRows);
-  for (int l = 0; l < n_layers; ++l) {
-    if (!encode_3d(&L.tmK[l], K[l], d, T, Hkv, k_head_stride, kKeyTile)) return STEPKV_ECUDA;
-    if (!encode_3d(&L.tmQ[l], Q[l], d, W, Hq, q_head_stride, box_rows)) return STEPKV_ECUDA;
+  int items = 0;
+  for (int b = 0; b < n_traj; ++b) {
+    const ScoreTrajSpec& t = trajs[b];
+    if ((t.t_acc != nullptr) != (L.accumulate != 0)) return STEPKV_EINVAL;
+    for (int l = 0; l < n_layers; ++l) {
+      if (!encode_3d(&L.tmK[b * n_layers + l], t.K[l], d, t.T, Hkv, t.k_head_stride, kKeyTile)) return STEPKV_ECUDA;
+      if (!encode_3d(&L.tmQ[b * n_layers + l], t.Q[l], d, W, Hq, t.q_head_stride, box_rows)) return STEPKV_ECUDA;
+    }
+    L.traj[b].T = t.T;
+    L.traj[b].n_tiles = (t.T + kKeyTile - 1) / kKeyTile;
+    L.traj[b].item_off = items;
+    L.traj[b].t_acc = t.t_acc;
+    items += L.units_per * L.traj[b].n_tiles;
   }
   int n_sm = 0;
   cudaError_t e = device_sm_count(&n_sm);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   const int grid_cap = std::max(1, std::min(n_sm, kMaxGrid));
-  // all (layer, KV head) pairs in one launch: every CTA gets a contiguous range of (unit, tile) items
+  // all (trajectory, layer, KV head) pairs in one launch: every CTA gets a contiguous range of items
   L.pair0 = 0;
-  L.zero_acc = t_acc != nullptr ? 1 : 0;
-  L.n_units = n_layers * Hkv * g.n_rg;
-  const int U = L.n_units * g.n_tiles;
-  const int grid0 = std::min(grid_cap, U);
-  L.tpc = (U + grid0 - 1) / grid0;
-  const int grid = (U + L.tpc - 1) / L.tpc;
+  L.n_items = items;
+  const int grid0 = std::min(grid_cap, items);
+  L.tpc = (items + grid0 - 1) / grid0;
+  const int grid = (items + L.tpc - 1) / L.tpc;
   L.token = next_launch_token();
   // Self-test of the failure path: the pass-2 wait looks for a value no CTA ever publishes, so every
   // CTA's wait runs out after selftest_wait_ns and the kernel takes its abort path.
@@ -886,6 +945,15 @@ stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_str
   e = d == 128 ? launch_score<2>(L, grid, stream) : launch_score<1>(L, grid, stream);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }
   return STEPKV_OK;
+}
+
+stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                          int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
+                          int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
+                          cudaStream_t stream, unsigned long long selftest_wait_ns) {
+  const ScoreTrajSpec one{K, Q, T, t_acc, k_head_stride, q_head_stride};
+  return score_run_batch(n_layers, &one, 1, Hkv, Hq, d, W, rows_out, out_stride, acc_shift, part, status, stream,
+                         selftest_wait_ns);
 }
 
 stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal,

@@ -406,3 +406,26 @@ def test_compress_full_32k_32layer(B):
         assert torch.equal(g.K_out[l][:, :n], K[l].index_select(1, kept))
         assert torch.equal(g.V_out[l][:, :n], V[l].index_select(1, kept))
     print(f"full-size swaps: {swaps}")
+
+
+def test_compress_batched_short_trajectories(B):
+    """Short trajectories of one head shape share one saliency launch (lengths and strides differ; a
+    different shape in the middle starts a new launch); every trajectory matches the oracle."""
+    import torch
+    shapes = [(64, 1200), (64, 2048), (64, 777), (128, 1500), (64, 3100), (64, 2500), (64, 1000), (64, 640),
+              (64, 1800), (64, 2222)]
+    trs = [wl.custom(200 + i, L=2, Hq=8, Hkv=2, d=d, T=T, W=24, n_steps=4 + i % 5, budget=wl.Budget.ratio(1, 4))
+           for i, (d, T) in enumerate(shapes)]
+    gs = [TL.GpuTraj(tr) for tr in trs]
+    probs = [g.problem() for g in gs]
+    st = B.stepkv_compress(probs, B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for g, tr in zip(gs, trs):
+        out = TL.run_oracle(tr, TL.oracle_params(B.Params()))
+        TL.check_select_outputs(g, out)
+        n = int(g.out.n_kept.item())
+        gk = g.out.kept_idx[:n].cpu().numpy()
+        for l in range(tr.shape.L):
+            assert np.array_equal(TL.bits_of(g.K_out[l])[:, :n], O.compact_rows(tr.keys(l), gk))
+            assert np.array_equal(TL.bits_of(g.V_out[l])[:, :n], O.compact_rows(tr.values(l), gk))

@@ -142,6 +142,9 @@ static stepkv_status_t check_compact_args(int n_layers, const void* const* K_in,
   if (n_layers < 0 || Hkv < 1 || d < 8 || T < 1 || kept_cap < 0) return STEPKV_EINVAL;
   if (!kept_idx || !n_kept) return STEPKV_EINVAL;
   if ((d * 2) % 16 || d > 256) return STEPKV_EUNSUPPORTED;
+  // one launch's row items of a trajectory (at most 96 layers x K, V x heads x kept_cap) use 32-bit indices
+  if ((int64_t)std::min(n_layers, 96) * 2 * Hkv * std::max(kept_cap, 1) >= ((int64_t)1 << 30))
+    return STEPKV_EUNSUPPORTED;
   if (n_layers > 0) {
     if (!K_in || !K_out) return STEPKV_EINVAL;
     if ((V_in == nullptr) != (V_out == nullptr)) return STEPKV_EINVAL;
@@ -502,7 +505,9 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   // stages 2-4 for all trajectories in one launch (one cluster per trajectory)
   stepkv_status_t st = select_run_batch(specs.data(), n_traj, s);
   if (st != STEPKV_OK) return st;
-  // stage 5 (out of place, or in place by hole filling when the outputs are the inputs)
+  // stage 5: in place by hole filling where the outputs are the inputs (one plan and one move launch per
+  // trajectory), the rest out of place, sharing launches
+  std::vector<CompactSpec> outs;
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     bool inplace = false;
@@ -516,11 +521,11 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
       if (st != STEPKV_OK) return st;
       continue;
     }
-    st = compact_run(p.L, c.K.data(), c.V.data(), p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
-                     p.sel.kept_cap, c.K_out.data(), c.V_out.data(), p.out_head_stride, p.step_id, p.pos_in,
-                     p.step_id_out, p.pos_out, dev_status, s);
-    if (st != STEPKV_OK) return st;
+    outs.push_back(CompactSpec{p.L, c.K.data(), c.V.data(), p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx,
+                               p.sel.n_kept, p.sel.kept_cap, c.K_out.data(), c.V_out.data(), p.out_head_stride,
+                               p.step_id, p.pos_in, p.step_id_out, p.pos_out});
   }
+  if (!outs.empty()) return compact_run_batch(outs.data(), (int)outs.size(), dev_status, s);
   return STEPKV_OK;
 }
 

@@ -142,6 +142,26 @@ stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride,
                               cudaStream_t stream);
 
 // ---- compact (compact.cu)
+// One out-of-place compaction (as stepkv_compact's arguments).
+struct CompactSpec {
+  int n_layers;
+  const void* const* K_in;
+  const void* const* V_in;
+  int64_t in_head_stride;
+  int Hkv, d, T;
+  const int32_t* kept_idx;
+  const int32_t* n_kept;
+  int kept_cap;
+  void* const* K_out;
+  void* const* V_out;
+  int64_t out_head_stride;
+  const int32_t* step_id_in;
+  const int32_t* pos_in;
+  int32_t* step_id_out;
+  int32_t* pos_out;
+};
+// Several compactions, sharing launches where they fit.
+stepkv_status_t compact_run_batch(const CompactSpec* specs, int n, int32_t* status, cudaStream_t stream);
 stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* const* V_in, int64_t in_head_stride,
                             int Hkv, int d, int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
                             void* const* K_out, void* const* V_out, int64_t out_head_stride,

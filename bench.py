@@ -645,10 +645,10 @@ def main():
     args = ap.parse_args()
     if args.compact_traffic is None and args.T == 32768 and args.layers == 32:
         # dram__bytes_read.sum + dram__bytes_write.sum of compact_kernel from one ncu capture of the
-        # 8-layer variant of this workload (109.78 MB read + 59.16 MB written), scaled by row sets (x4):
+        # 8-layer variant of this workload (109.80 MB read + 58.67 MB written), scaled by row sets (x4):
         # the kernel does the same work per row set.  Writes below the algorithmic bytes are dirty lines
         # still in L2 when the kernel ends.
-        args.compact_traffic = 4 * (109.782528e6 + 59.157760e6)
+        args.compact_traffic = 4 * (109.800960e6 + 58.666496e6)
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -71,6 +71,16 @@ struct SelectBatch {
 };
 static_assert(sizeof(SelectBatch) <= 32000, "kernel parameter space");
 
+// Inclusive suffix sum over the warp: lane l gets v[l] + v[l + 1] + ... + v[31].
+__device__ __forceinline__ int warp_suffix_sum(int v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_down_sync(0xffffffffu, v, o);
+    if (lane + o < 32) v += y;
+  }
+  return v;
+}
+
 template <int NT>
 __device__ __forceinline__ int block_reduce_sum_int(int v, int* scratch) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -218,7 +228,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int rank = cl.rank();
   extern __shared__ __align__(16) uint8_t smem_raw[];
   // layout: [chunk] float/uint32 keys | [chunk] u16 step id (0xFFFF = protected) | 2 x 2048 int hist |
-  //         SelShared (own) | SelShared[NC] (gathered) | scratch[64] | S_k (when s_in_smem)
+  //         SelShared (own) | SelShared[NC] (gathered) | scratch[64] | coarse[2][64] | S_k (when s_in_smem)
   uint32_t* sKey = reinterpret_cast<uint32_t*>(smem_raw);
   float* sT = reinterpret_cast<float*>(smem_raw);
   uint16_t* sSid = reinterpret_cast<uint16_t*>(smem_raw + (size_t)a.chunk * 4);
@@ -227,7 +237,8 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   SelShared* all = ex + 1;
   int* scratch = reinterpret_cast<int*>(all + NC);  // 64 ints
   int* bcast = scratch + 48;                        // radix decision
-  float* sS = reinterpret_cast<float*>(scratch + 64);
+  int* coarse = scratch + 64;                       // 2 x 64 coarse counts (alternate passes)
+  float* sS = reinterpret_cast<float*>(coarse + 128);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
@@ -468,59 +479,57 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         const int i = i0 + tid;
         const uint32_t k = i < len ? sKey[i] : 0u;
         const bool hit = i < len && sSid[i] != 0xFFFF && (k & mask) == prefix;
+        if (__ballot_sync(0xffffffffu, hit) == 0u) continue;  // after the first pass most keys miss the prefix
         const int bin = hit ? (int)((k >> sh) & (nb - 1)) : -1;
         const unsigned peers = __match_any_sync(0xffffffffu, bin);
         if (hit && (__ffs(peers) - 1) == lane) atomicAdd(&h[bin], __popc(peers));
       }
-      cl.sync();  // every CTA's histogram of this pass is complete
-      // global histogram; thread t owns bins [t*bpt, (t+1)*bpt)
-      const int bpt = nb / NT;  // 1, 2 or 4
-      int cnt[4] = {0, 0, 0, 0};
-      if (bpt == 4) {
-        int4 v[NC];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) v[r] = reinterpret_cast<const int4*>(cl.peer(h, r))[tid];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) {
-          cnt[0] += v[r].x;
-          cnt[1] += v[r].y;
-          cnt[2] += v[r].z;
-          cnt[3] += v[r].w;
-        }
-      } else if (bpt == 2) {
-        int2 v[NC];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) v[r] = reinterpret_cast<const int2*>(cl.peer(h, r))[tid];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) {
-          cnt[0] += v[r].x;
-          cnt[1] += v[r].y;
-        }
-      } else {
-        int v[NC];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) v[r] = cl.peer(h, r)[tid];
-#pragma unroll
-        for (int r = 0; r < NC; ++r) cnt[0] += v[r];
-      }
-      const int mine = cnt[0] + cnt[1] + cnt[2] + cnt[3];
-      // keys in bins owned by higher threads: suffix scan over the block
-      int x = mine;
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_down_sync(0xffffffffu, x, o);
-        if (lane + o < 32) x += y;
-      }
-      if (lane == 0) scratch[warp] = x;
       __syncthreads();
-      int after = 0;
-      for (int w = warp + 1; w < NW; ++w) after += scratch[w];
-      int above = after + x - mine;
-      for (int q = bpt - 1; q >= 0; --q) {
-        if (above < remaining && remaining <= above + cnt[q]) {
-          bcast[0] = tid * bpt + q;
-          bcast[1] = above;
+      // this CTA's coarse counts: sums of 32 consecutive bins (64 coarse bins for 11 bits, 32 for 10)
+      int* hc = coarse + (pass & 1) * 64;
+      const int ncoarse = nb >> 5;
+      for (int c = warp; c < ncoarse; c += NW) {
+        int v = h[c * 32 + lane];
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) hc[c] = v;
+      }
+      cl.sync();  // every CTA's histogram and coarse counts of this pass are complete
+      if (warp == 0) {
+        // The digit in two small cluster-wide steps (keys in descending order): first the coarse bin that
+        // holds the remaining-th largest key, then the bin within it.  Lane l holds coarse bins l and
+        // 32 + l, then fine bin 32 * c* + l.
+        int clo = 0, chi = 0;
+#pragma unroll
+        for (int r = 0; r < NC; ++r) {
+          const int* pc = cl.peer(hc, r);
+          clo += pc[lane];
+          if (ncoarse > 32) chi += pc[32 + lane];
         }
-        above += cnt[q];
+        const int shi = warp_suffix_sum(chi, lane);                                    // keys in bins >= 32 + l
+        const int slo = warp_suffix_sum(clo, lane) + __shfl_sync(0xffffffffu, shi, 0);  // keys in bins >= l
+        const unsigned mhi = __ballot_sync(0xffffffffu, shi - chi < remaining && remaining <= shi);
+        const unsigned mlo = __ballot_sync(0xffffffffu, slo - clo < remaining && remaining <= slo);
+        const int lhi = __ffs(mhi) - 1, llo = __ffs(mlo) - 1;
+        const int above_hi = __shfl_sync(0xffffffffu, shi - chi, lhi < 0 ? 0 : lhi);
+        const int above_lo = __shfl_sync(0xffffffffu, slo - clo, llo < 0 ? 0 : llo);
+        bool found = mhi != 0 || mlo != 0;
+        const int cstar = mhi ? 32 + lhi : (mlo ? llo : 0);
+        const int above_c = mhi ? above_hi : (mlo ? above_lo : 0);
+        int f = 0;
+#pragma unroll
+        for (int r = 0; r < NC; ++r) f += cl.peer(h, r)[cstar * 32 + lane];
+        const int sf = warp_suffix_sum(f, lane);
+        const unsigned mf = __ballot_sync(0xffffffffu, above_c + sf - f < remaining && remaining <= above_c + sf);
+        const int lf = __ffs(mf) - 1;
+        found = found && mf != 0;
+        const int above_f = __shfl_sync(0xffffffffu, above_c + sf - f, lf < 0 ? 0 : lf);
+        if (lane == 0) {
+          // the counts always hold the remaining-th key; the guard only keeps every index in range
+          if (!found) record_status(a.status, STEPKV_EDATA);
+          bcast[0] = found ? cstar * 32 + lf : 0;
+          bcast[1] = found ? above_f : 0;
+        }
       }
       __syncthreads();
       const int bstar = bcast[0];
@@ -713,7 +722,8 @@ static SelectArgs make_select_args(const SelectSpec& sp) {
 // Shared memory of one trajectory's CTA: keys + step ids of its chunk, histograms, exchange blocks,
 // scratch, and S_k when it fits.
 static size_t select_smem(int chunk, int nc, int n_steps, int* s_in_smem) {
-  const size_t fixed = (((size_t)chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) + 64 * 4;
+  const size_t fixed = (((size_t)chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) +
+                       (64 + 128) * 4;
   const size_t budget_smem = 232448 - 1024;
   *s_in_smem = fixed + (size_t)n_steps * 4 <= budget_smem ? 1 : 0;
   return fixed + (*s_in_smem ? (size_t)n_steps * 4 : 0);

@@ -160,26 +160,38 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
         }
       }
     }
+    // probabilities of the block's keys per head (state rescaled once per block), then one pass over
+    // the value rows: each is converted once and accumulated into every head
+    float p[kDecBlockSteps][G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       float mb = m[g];
 #pragma unroll
       for (int t = 0; t < kDecBlockSteps; ++t) mb = fmaxf(mb, s[t][g]);
-      if (mb == -INFINITY) continue;
+      if (mb == -INFINITY) {
+#pragma unroll
+        for (int t = 0; t < kDecBlockSteps; ++t) p[t][g] = 0.f;
+        continue;
+      }
       const float sc = ex2_approx(m[g] - mb);
       l[g] *= sc;
 #pragma unroll
       for (int e = 0; e < 8; ++e) acc[g][e] *= sc;
 #pragma unroll
       for (int t = 0; t < kDecBlockSteps; ++t) {
-        const float p = ex2_approx(s[t][g] - mb);
-        float vf[8];
-        bf16x8_to_f32(vr[t], vf);
-        l[g] += p;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
+        p[t][g] = ex2_approx(s[t][g] - mb);
+        l[g] += p[t][g];
       }
       m[g] = mb;
+    }
+#pragma unroll
+    for (int t = 0; t < kDecBlockSteps; ++t) {
+      float vf[8];
+      bf16x8_to_f32(vr[t], vf);
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p[t][g], vf[e], acc[g][e]);
     }
   }
   // merge the key slots of the warp (lanes with the same hl), then the warps through shared memory

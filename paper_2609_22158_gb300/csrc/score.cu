@@ -16,7 +16,7 @@
 // into a double-buffered TMEM accumulator (2 x 256 columns); 16 epilogue warps in two groups (one per
 // accumulator buffer, alternate items) read TMEM with tcgen05.ld and spend one MUFU ex2 per logit.
 // A unit has a few pass-1 partials (one set per contributing CTA); the pass-2 epilogue combines them
-// in a fixed order (deterministic) once every CTA has raised its pass-1 flag.
+// in a fixed order (deterministic) once the CTAs that cover the unit have raised their pass-1 flags.
 #include <math.h>
 
 #include <algorithm>
@@ -74,6 +74,7 @@ struct ScoreLaunch {
   int accumulate;     // 1: pass 2 adds into each trajectory's t_acc (zeroed first) instead of writing rows
   int acc_shift;      // k: fixed-point scale 2^k of t_acc
   unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores `token` once its partials are written
+  unsigned long long* zflags; // [grid] CTA b stores `token` once its share of the accumulators is zeroed
   unsigned long long token;   // unique per launch, so flags left by earlier launches never match
   unsigned long long wait_token;     // the value the pass-2 wait looks for (token, except in the self-test)
   unsigned long long wait_limit_ns;  // the pass-2 wait gives up (STEPKV_ETIMEOUT) after this long
@@ -273,9 +274,9 @@ __device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned l
 // forward for pass 1 (in pairs of tiles: one N = 256 MMA per query half) and backward for pass 2, so
 // the TMA ring, the MMA issuer and the Q staging run on without a break at the change of pass (the
 // first pass-2 tile is the last pass-1 tile, same Q).  Only the pass-2 epilogue depends on other CTAs:
-// it starts once every CTA has published its pass-1 partials (a flag per CTA set to this launch's
-// token; the launch is cooperative, so all CTAs are resident and the wait ends, else it gives up after
-// the wait limit).
+// each unit starts once the CTAs covering it have published their pass-1 partials (a flag per CTA set
+// to this launch's token; the launch is cooperative, so all CTAs are resident and the wait ends, else it
+// gives up after the wait limit).
 //
 // Accumulator work is counted in "halves": a pass-1 pair item gives one half per 128-row query tile,
 // a pass-2 item one half.  Half h goes to TMEM buffer h & 1 and is drained by epilogue group h & 1.
@@ -520,15 +521,18 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       if (lane == 0) mbar_arrive(&acc_empty[grp]);
     };
 
-    // The epilogue warps zero this CTA's share of t_acc while the first tiles stream in.  The stores
-    // precede the warp's p1_flushed arrival, so the publisher's fence orders them before the CTA's flag,
-    // hence before any pass-2 addition by any CTA.
-    if (p.accumulate) {
+    // The first epilogue warp zeroes this CTA's share of the accumulators while the first tiles stream
+    // in, then publishes it (fence + release store of the launch's token): a CTA adds into the
+    // accumulators only after it has seen every CTA's zero flag.
+    if (p.accumulate && ew == 0) {
       for (int b = 0; b < p.n_traj; ++b) {
         unsigned long long* acc = p.traj[b].t_acc;
-        for (int i = blockIdx.x * (kEpiWarps * 32) + (threadIdx.x - 64); i < p.traj[b].T;
-             i += gridDim.x * (kEpiWarps * 32))
-          acc[i] = 0ull;
+        for (int i = blockIdx.x * 32 + lane; i < p.traj[b].T; i += gridDim.x * 32) acc[i] = 0ull;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        __threadfence();
+        st_release_u64(&p.zflags[blockIdx.x], p.token);
       }
     }
 
@@ -622,7 +626,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     if (ok) {
       int cur = -1, n_done = 0;  // n_done: pass-2 items this group has drained
       RowGroup r{};
-      bool others_done = false;
+      bool zeros_seen = !p.accumulate;
       float* negoff = sNegOff + grp * kMaxRows;  // this group's per-row offsets and causal limits
       int* pw_tab = sPw + grp * kMaxRows;
       float* combf = sComb + grp * (2 * 128);     // rows output: [2 parity][128]
@@ -633,34 +637,37 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         const int u = il.u, tile = il.tile;
         const int Tb = p.traj[il.b].T;
         if (u != cur) {
-          if (!others_done) {
-            // Wait until every CTA has published its pass-1 partials (and zeroed its share of t_acc).
-            if (leader) {
-              // Relaxed polls (the lanes' loads overlap), then one acquire fence once all flags match.
-              bool all = false;
-              const uint64_t t0 = globaltimer_ns();
-              for (uint32_t it = 0; !all; ++it) {
-                bool mine = true;
+          // The CTAs whose pass-1 ranges cover unit u: their partials are combined below.
+          const int f0 = unit_first_item(p, u);
+          const int c0 = f0 / p.tpc;
+          const int c1 = (f0 + p.traj[il.b].n_tiles - 1) / p.tpc;
+          // Wait until those CTAs have published their pass-1 partials (and, before the first addition,
+          // every CTA its zeroed accumulators): the unit starts as soon as its own producers are done.
+          if (leader) {
+            // Relaxed polls (the lanes' loads overlap), then one acquire fence once all flags match.
+            bool all = false;
+            const uint64_t t0 = globaltimer_ns();
+            for (uint32_t it = 0; !all; ++it) {
+              bool mine = true;
+              for (int b = c0 + lane; b <= c1; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.wait_token;
+              if (!zeros_seen) {
 #pragma unroll 4
-                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.wait_token;
-                all = __all_sync(0xffffffffu, mine);
-                if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > p.wait_limit_ns)) break;
+                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.zflags[b]) == p.wait_token;
               }
-              fence_acquire_gpu();
-              if (!all) {
-                *abort_flag = 1;
-                if (lane == 0) record_status(p.status, STEPKV_ETIMEOUT);
-              }
+              all = __all_sync(0xffffffffu, mine);
+              if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > p.wait_limit_ns)) break;
             }
-            others_done = true;
+            fence_acquire_gpu();
+            if (!all) {
+              *abort_flag = 1;
+              if (lane == 0) record_status(p.status, STEPKV_ETIMEOUT);
+            }
           }
+          zeros_seen = true;
           // Combine the pass-1 partials of unit u into this group's per-row offsets, in contributing-CTA
           // order (the group no longer reads the previous unit's offsets once all its warps arrive).
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
           r = row_group(g, u % g.n_rg);
-          const int f0 = unit_first_item(p, u);
-          const int c0 = f0 / p.tpc;
-          const int c1 = (f0 + p.traj[il.b].n_tiles - 1) / p.tpc;
           const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
           const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
           const int w = r.w0 + row % r.blk_rows;
@@ -813,13 +820,13 @@ int score_acc_shift(int n_pairs, int W) {
 }
 
 // Pass-1 partial slots (one per (unit, CTA) pair a launch can form: units + grid), then one
-// pass-1-done flag per CTA.
+// pass-1-done flag and one accumulators-zeroed flag per CTA.
 static size_t score_partial_slots_bytes(int n_traj, int n_layers, int Hkv, int Hq, int W) {
   const int n_rg = score_row_groups(Hkv, Hq, W);
   return (size_t)(n_traj * n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
 }
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W, int n_traj) {
-  return score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W) + (size_t)kMaxGrid * sizeof(unsigned long long);
+  return score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W) + 2 * (size_t)kMaxGrid * sizeof(unsigned long long);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -876,7 +883,7 @@ static cudaError_t launch_score(const ScoreLaunch& L, int grid, cudaStream_t str
   void (*kern)(ScoreLaunch) = score_kernel<NCH>;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(kern), Cfg::kDynSmem);
   if (e != cudaSuccess) return e;
-  // Cooperative: the pass-2 epilogue of each CTA waits for every CTA's pass-1 flag, so all CTAs must be
+  // Cooperative: the pass-2 epilogue of each CTA waits for other CTAs' flags, so all CTAs must be
   // resident at once (the launch fails instead of starting if they cannot be).
   cudaLaunchConfig_t cfg;
   memset(&cfg, 0, sizeof(cfg));
@@ -907,6 +914,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.part = part;
   L.flags = reinterpret_cast<unsigned long long*>(reinterpret_cast<uint8_t*>(part) +
                                                   score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W));
+  L.zflags = L.flags + kMaxGrid;
   L.out = rows_out;
   L.out_stride = out_stride;
   L.accumulate = trajs[0].t_acc != nullptr ? 1 : 0;

@@ -178,6 +178,18 @@ def test_select_large_T(B):
     TL.check_select_outputs(g, out)
 
 
+@pytest.mark.parametrize("n_steps", [2048, 2600])
+def test_select_many_steps(B, n_steps):
+    """Thousands of reasoning steps (a few tokens each): per-step statistics, S_k and the selection."""
+    T = 24000
+    tr = wl.custom(31 + n_steps, L=1, Hq=8, Hkv=2, d=64, T=T, W=32, n_steps=n_steps, budget=wl.Budget.ratio(1, 6))
+    rng = np.random.default_rng(n_steps)
+    sal = rng.random((2, T)).astype(np.float32) ** 3
+    g, out, st = _select_case(B, tr, B.Params(), sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
 def test_select_reuse_in_place(B):
     """reuse_out may alias reuse_in (the caller keeps one c_k array across boundaries)."""
     import torch

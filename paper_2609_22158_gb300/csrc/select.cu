@@ -247,6 +247,9 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int base = rank * a.chunk;
   const int len = max(0, min(a.chunk, T - base));
   const bool s_in_smem = a.s_in_smem != 0;
+  // per-step statistics are outputs only (they do not enter P): skip them when none is requested
+  const bool want_stats = a.out.step_count || a.out.step_sal_sum || a.out.step_sal_max;
+  const bool want_kept = a.out.step_kept != nullptr;
 
   // Launched with programmatic dependent launch: everything up to pdl_wait() reads only the call's
   // inputs (step signals, step ids, mask) and writes only this kernel's workspace and outputs, so it
@@ -434,21 +437,23 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         const float P = fmaf(a.prm.alpha, th, a.prm.beta * Sk[sid]);
         key = float_to_ordered(P);
         if (a.out.priority) a.out.priority[gi] = P;
-        const float thc = fmaxf(th, 0.f);
-        if (sid != run_sid) {
-          if (run_c) {
-            atomicAdd(&a.acc_cnt[run_sid], run_c);
-            atomicAdd(&a.acc_sum[run_sid], run_s);
-            atomicMax(&a.acc_max[run_sid], run_m);
+        if (want_stats) {
+          const float thc = fmaxf(th, 0.f);
+          if (sid != run_sid) {
+            if (run_c) {
+              atomicAdd(&a.acc_cnt[run_sid], run_c);
+              atomicAdd(&a.acc_sum[run_sid], run_s);
+              atomicMax(&a.acc_max[run_sid], run_m);
+            }
+            run_sid = sid;
+            run_c = 0;
+            run_s = 0ull;
+            run_m = 0u;
           }
-          run_sid = sid;
-          run_c = 0;
-          run_s = 0ull;
-          run_m = 0u;
+          ++run_c;
+          run_s += to_fixed(thc, fx_shift);
+          run_m = max(run_m, __float_as_uint(thc));
         }
-        ++run_c;
-        run_s += to_fixed(thc, fx_shift);
-        run_m = max(run_m, __float_as_uint(thc));
       } else if (a.out.priority) {
         a.out.priority[gi] = -INFINITY;
       }
@@ -625,7 +630,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       if (keep) a.out.kept_idx[out_pos + __popc(km & lt)] = base + i;
       out_pos += __popc(km);
       tie_rank += __popc(em);
-      if (keep && !pr) {
+      if (want_kept && keep && !pr) {
         if (sid != run_sid) {
           if (run_c) atomicAdd(&a.acc_kept[run_sid], run_c);
           run_sid = sid;
@@ -636,15 +641,17 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
     }
     step_stat_flush(run_c > 0, run_sid, run_c, 0ull, 0u, a.acc_kept, nullptr, nullptr);
   }
-  cl.sync();  // (C) all step accumulators final
+  if (want_stats || want_kept) {
+    cl.sync();  // (C) all step accumulators final
 
-  // ---- per-step outputs
-  const double fx_unit = ldexp(1.0, -fx_shift);
-  for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
-    if (a.out.step_count) a.out.step_count[k] = a.acc_cnt[k];
-    if (a.out.step_sal_sum) a.out.step_sal_sum[k] = (float)((double)a.acc_sum[k] * fx_unit);
-    if (a.out.step_sal_max) a.out.step_sal_max[k] = __uint_as_float(a.acc_max[k]);
-    if (a.out.step_kept) a.out.step_kept[k] = a.acc_kept[k];
+    // ---- per-step outputs
+    const double fx_unit = ldexp(1.0, -fx_shift);
+    for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
+      if (a.out.step_count) a.out.step_count[k] = a.acc_cnt[k];
+      if (a.out.step_sal_sum) a.out.step_sal_sum[k] = (float)((double)a.acc_sum[k] * fx_unit);
+      if (a.out.step_sal_max) a.out.step_sal_max[k] = __uint_as_float(a.acc_max[k]);
+      if (a.out.step_kept) a.out.step_kept[k] = a.acc_kept[k];
+    }
   }
   if (NC > 1) cl.sync();  // no CTA exits while another may still read its shared memory
 }

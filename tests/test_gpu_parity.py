@@ -335,6 +335,32 @@ def test_compress_batched_ragged(B):
         assert np.array_equal(TL.bits_of(g.K_out[0])[:, :n], O.compact_rows(tr.keys(0), gk))
 
 
+def test_compress_minimal_outputs_same_selection(B):
+    """Without the optional outputs (per-step statistics, priorities) the kernel skips their work; the
+    retained set and the compacted rows are the same as with every output requested."""
+    import torch
+    tr = wl.custom(404, L=3, Hq=8, Hkv=2, d=128, T=9000, W=32, n_steps=12, budget=wl.Budget.ratio(1, 8))
+    g = TL.GpuTraj(tr)
+    full = g.problem()
+    st = B.stepkv_compress([full], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    n = int(g.out.n_kept.item())
+    kept_full = g.out.kept_idx[:n].clone()
+    K0 = [k[:, :n].clone() for k in g.K_out]
+    lean = g.problem()
+    g.out = B.SelectOutputs.allocate(tr.T, tr.n_steps, g.kept_cap, "cuda", full=False)
+    lean.out = g.out
+    lean.refresh()
+    st = B.stepkv_compress([lean], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    assert int(g.out.n_kept.item()) == n
+    assert torch.equal(g.out.kept_idx[:n], kept_full)
+    for l in range(tr.shape.L):
+        assert torch.equal(g.K_out[l][:, :n], K0[l])
+
+
 def test_compress_all_protected(B):
     """N_t = 0: nothing is prunable, every slot is kept, B_t = 0."""
     import torch

@@ -164,3 +164,36 @@ def test_ctypes_structs_mirror_the_header(tmp_path):
         assert got[(cname, "size")] == ctypes.sizeof(py), cname
         for f, _ in py._fields_:
             assert got[(cname, f)] == getattr(py, f).offset, (cname, f)
+
+
+def _build_c_program(tmp_path):
+    """tests/c/compress_from_c.c compiled with the system C compiler against include/stepkv.h and the
+    in-tree library (plain C: no Python, no PyTorch on the path)."""
+    import shutil
+    import subprocess
+    from paper_2609_22158_gb300 import build
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    lib_path = build.build_library()
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    exe = tmp_path / "compress_from_c"
+    cmd = [cc, "-std=c99", "-O1", "-I", os.path.join(ROOT, "include"), "-I", os.path.join(cuda, "include"),
+           os.path.join(ROOT, "tests", "c", "compress_from_c.c"), "-o", str(exe), lib_path,
+           "-Wl,-rpath," + os.path.dirname(lib_path), "-L" + os.path.join(cuda, "lib64"), "-lcudart",
+           "-Wl,-rpath," + os.path.join(cuda, "lib64")]
+    subprocess.run(cmd, check=True)
+    return exe
+
+
+def test_c_program_uses_the_abi(tmp_path):
+    import subprocess
+    exe = _build_c_program(tmp_path)
+    out = subprocess.run([str(exe), "host"], check=True, capture_output=True, text=True).stdout.split("\n")
+    fields = dict((ln.split(" ", 1)[0], ln.split(" ", 1)[1]) for ln in out if ln)
+    assert [float(x) for x in fields["params"].split()] == pytest.approx(
+        [0.3, 0.85, 0.15, -1.0, 2.0, 8.0, 1.5, 0.2, 0.8, 0.0], abs=1e-6)
+    from paper_2609_22158_gb300 import binding
+    assert fields["status"] == binding.load_library().stepkv_status_string(1).decode()
+    assert int(fields["compress_null"]) == 1  # STEPKV_EINVAL before anything is enqueued
+    assert int(fields["workspace_empty"]) == 0

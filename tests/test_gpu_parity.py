@@ -335,6 +335,21 @@ def test_compress_batched_ragged(B):
         assert np.array_equal(TL.bits_of(g.K_out[0])[:, :n], O.compact_rows(tr.keys(0), gk))
 
 
+@pytest.mark.parametrize("Hq,Hkv,W", [(10, 2, 128), (4, 2, 300)])
+def test_compress_batched_row_groups(B, Hq, Hkv, W):
+    """Short trajectories whose query rows need several row groups (GQA 5 x W 128 = 640 rows; a
+    300-row window split over two groups) share one saliency launch."""
+    import torch
+    trs = [wl.custom(500 + i + W, L=2, Hq=Hq, Hkv=Hkv, d=128, T=T, W=W, n_steps=4 + i, budget=wl.Budget.ratio(1, 3))
+           for i, T in enumerate((700, 1300, 2100))]
+    gs = [TL.GpuTraj(tr) for tr in trs]
+    st = B.stepkv_compress([g.problem() for g in gs], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for g, tr in zip(gs, trs):
+        TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(B.Params())))
+
+
 def test_compress_minimal_outputs_same_selection(B):
     """Without the optional outputs (per-step statistics, priorities) the kernel skips their work; the
     retained set and the compacted rows are the same as with every output requested."""

@@ -350,6 +350,43 @@ def test_compress_batched_row_groups(B, Hq, Hkv, W):
         TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(B.Params())))
 
 
+def test_compress_twenty_trajectories_mixed_in_place(B):
+    """20 trajectories in one call (more than one selection launch of 16 and more than one compaction
+    launch), every fourth compacted in place: each matches the oracle."""
+    import torch
+    trs = [wl.custom(600 + i, L=2, Hq=4, Hkv=2, d=64, T=400 + 37 * i, W=16, n_steps=3 + i % 4,
+                     budget=wl.Budget.ratio(1, 5)) for i in range(20)]
+    gs = [TL.GpuTraj(tr) for tr in trs]
+    probs = []
+    src = []
+    for i, (g, tr) in enumerate(zip(gs, trs)):
+        prob = g.problem()
+        if i % 4 == 3:
+            # in place: the outputs are the inputs (rows [0, n_kept) end up holding the retained set)
+            src.append(([TL.bits_of(k) for k in g.K], [TL.bits_of(v) for v in g.V]))
+            prob = B.Problem(g.K, g.V, g.Q, tr.T, g.step_id, g.prot, g.steps(), g.budget(), g.K, g.V, g.out,
+                             pos_in=g.pos, step_id_out=g.step_id_out, pos_out=g.pos_out)
+        else:
+            src.append(None)
+        probs.append(prob)
+    st = B.stepkv_compress(probs, B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for g, tr, sv in zip(gs, trs, src):
+        out = TL.run_oracle(tr, TL.oracle_params(B.Params()))
+        TL.check_select_outputs(g, out)
+        n = int(g.out.n_kept.item())
+        gk = g.out.kept_idx[:n].cpu().numpy().astype(np.int64)
+        if sv is None:
+            assert np.array_equal(TL.bits_of(g.K_out[1])[:, :n], O.compact_rows(tr.keys(1), gk))
+        else:
+            slot_of_pos = {int(x): j for j, x in enumerate(tr.pos)}
+            srcs = np.array([slot_of_pos[int(x)] for x in g.pos_out[:n].cpu().numpy()], np.int64)
+            assert np.array_equal(np.sort(srcs), gk)
+            assert np.array_equal(TL.bits_of(g.K[1])[:, :n], sv[0][1][:, srcs])
+            assert np.array_equal(TL.bits_of(g.V[0])[:, :n], sv[1][0][:, srcs])
+
+
 def test_compress_minimal_outputs_same_selection(B):
     """Without the optional outputs (per-step statistics, priorities) the kernel skips their work; the
     retained set and the compacted rows are the same as with every output requested."""

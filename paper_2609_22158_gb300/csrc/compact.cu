@@ -80,6 +80,8 @@ struct CompactBatchArgs {
   int32_t* status;
 };
 
+static_assert(sizeof(CompactBatchArgs) <= 32000, "kernel parameter space");
+
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_constant__ CompactBatchArgs a) {
   pdl_wait();  // kept_idx / n_kept come from the selection kernel
   pdl_launch_dependents();

@@ -41,6 +41,8 @@ struct DecodeArgs {
   int32_t* status;
 };
 
+static_assert(sizeof(DecodeArgs) <= 32000, "kernel parameter space");
+
 __device__ __forceinline__ int decode_n(const DecodeArgs& a) {
   const int n = a.n_dev ? *a.n_dev : a.n_host;
   return n;

@@ -81,6 +81,8 @@ struct ScoreLaunch {
   int32_t* status;
 };
 
+static_assert(sizeof(ScoreLaunch) <= 32000, "kernel parameter space");
+
 struct RowGroup {
   int g_first;   // first local query head (0..G-1) of this group
   int n_blk;     // head blocks

@@ -355,21 +355,42 @@ def run_ours(args):
         host_Kout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.K_out]
         host_Vout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.V_out]
         host_idx = torch.empty(dt.cap + 1, dtype=torch.int32).pin_memory()
-        hprob = B.Problem(host_K, host_V, dt.Q, s_.T, dt.step_id, dt.prot, dt.steps, dt.budget, host_Kout, host_Vout,
-                          dt.out, pos_in=dt.pos, step_id_out=dt.step_id_out, pos_out=dt.pos_out,
-                          kv_location=B.STEPKV_MEM_HOST, out_location=B.STEPKV_MEM_HOST, K_sal=K_sal)
+        sig_dev = [dt.steps.valid, dt.steps.gain, dt.steps.red, dt.steps.reuse_in, dt.steps.obs_sim]
+        host_sig = [x.cpu().pin_memory() for x in sig_dev]
         nb = lambda ts: sum(t.numel() * t.element_size() for t in ts)
         row_bytes = 2 * s_.L * s_.Hkv * s_.d * 2  # K and V of one retained slot, all layers
         k2 = max(1, min(args.steps, args.e2e_steps))
+        # Two sets of device input buffers, so that the next step's host->device copies (on their own
+        # stream) run while the current step gathers its rows across the link in the other direction.
+        copy_stream = torch.cuda.Stream(device=dev)
+        bufs = []
+        for _ in range(2):
+            Qb = [torch.empty_like(q) for q in dt.Q]
+            smallb = [torch.empty_like(x) for x in dev_small]
+            sigb = [torch.empty_like(x) for x in sig_dev]
+            Ksb = [torch.empty_like(dt.K[l]) for l in sal_ids]
+            stepsb = B.StepSignals(sigb[0], sigb[1], sigb[2], sigb[3], sigb[4], dt.steps.reuse_out)
+            probb = B.Problem(host_K, host_V, Qb, s_.T, smallb[0], smallb[1], stepsb, dt.budget, host_Kout,
+                              host_Vout, dt.out, pos_in=smallb[2], step_id_out=dt.step_id_out, pos_out=dt.pos_out,
+                              kv_location=B.STEPKV_MEM_HOST, out_location=B.STEPKV_MEM_HOST, K_sal=Ksb)
+            bufs.append((Qb + smallb + sigb + Ksb, probb, torch.cuda.Event(), torch.cuda.Event()))
+        step_inputs = host_Q + host_small + host_sig + [host_K[l] for l in sal_ids]
+        n_step = [0]
 
         def e2e_step():
-            for h, d in zip(host_Q + host_small, dt.Q + dev_small):
-                d.copy_(h, non_blocking=True)
-            for h, d in zip([host_K[l] for l in sal_ids], K_sal):
-                d.copy_(h, non_blocking=True)
-            B.stepkv_compress([hprob], params, ws=dt.ws, status=dt.status, stream=stream)
-            host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
-            host_idx[dt.cap:].copy_(dt.out.n_kept, non_blocking=True)
+            dsts, probb, copied, done = bufs[n_step[0] % 2]
+            n_step[0] += 1
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(done)  # the step that last used these buffers has finished with them
+                for h, d in zip(step_inputs, dsts):
+                    d.copy_(h, non_blocking=True)
+                copied.record(copy_stream)
+            stream.wait_event(copied)
+            B.stepkv_compress([probb], params, ws=dt.ws, status=dt.status, stream=stream)
+            done.record(stream)
+            with torch.cuda.stream(stream):
+                host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
+                host_idx[dt.cap:].copy_(dt.out.n_kept, non_blocking=True)
 
         def timed(step):
             # one untimed step first: the first transfer from freshly pinned pages runs at about a third
@@ -378,6 +399,7 @@ def run_ours(args):
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
+            copy_stream.wait_event(e0)
             for i in range(k2):
                 step()
             e1.record(stream)
@@ -391,12 +413,14 @@ def run_ours(args):
         for l in (0, s_.L - 1):  # the host outputs hold the retained rows
             assert torch.equal(host_Kout[l][:, :n_k], host_K[l].index_select(1, kept_h))
             assert torch.equal(host_Vout[l][:, :n_k], host_V[l].index_select(1, kept_h))
-        h2d = nb(host_Q + host_small) + nb([host_K[l] for l in sal_ids]) + n_k * row_bytes
+        h2d = nb(step_inputs) + n_k * row_bytes
         d2h = n_k * row_bytes + host_idx.numel() * 4
         e2e = {"value": MR.job_throughput(tokens, e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": k2,
-               "path": "cache in pinned host memory: saliency layers' K copied to the device, retained rows "
-                       "gathered across the CPU-GPU link into pinned host outputs"}
+               "path": "cache in pinned host memory: window queries, token metadata, step signals and the "
+                       "saliency layers' K copied to the device (two buffer sets: the next step's copies overlap "
+                       "the current step's gather), retained rows gathered across the CPU-GPU link into pinned "
+                       "host outputs"}
 
         def copy_all_step():
             for h, d in zip(host_K + host_V + host_Q + host_small, dt.K + dt.V + dt.Q + dev_small):
@@ -629,7 +653,7 @@ def main():
     ap.add_argument("--T", type=int, default=32768)
     ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-stages", action="store_true")
     ap.add_argument("--no-decode", action="store_true")

@@ -154,3 +154,34 @@ def test_host_location_rejects_other_memory(B):
     assert lib.stepkv_compress(arr, 1, ctypes.byref(cp), wp, need, st.data_ptr(), s) == B.STEPKV_EINVAL
     torch.cuda.synchronize()
     assert st.item() == 0
+
+
+def test_host_resident_batch_of_trajectories(B):
+    """Several host-resident trajectories in one call (one shared saliency launch, one compaction
+    launch): each equals its own all-device pass."""
+    import torch
+    trs = [wl.custom(71 + i, L=3, Hq=8, Hkv=2, d=64, T=T, W=16, n_steps=4 + i, budget=wl.Budget.ratio(1, 4))
+           for i, T in enumerate((900, 1500, 2300))]
+    refs, probs, outs = [], [], []
+    for tr in trs:
+        g = TL.GpuTraj(tr, kept_cap=tr.shape.T)
+        refs.append(_device_run(B, g))
+        s = tr.shape
+        Kh = [k.cpu().pin_memory() for k in g.K]
+        Vh = [v.cpu().pin_memory() for v in g.V]
+        K_out = [torch.zeros((s.Hkv, s.T, s.d), dtype=torch.bfloat16).pin_memory() for _ in range(s.L)]
+        V_out = [torch.zeros((s.Hkv, s.T, s.d), dtype=torch.bfloat16).pin_memory() for _ in range(s.L)]
+        out = B.SelectOutputs.allocate(s.T, tr.n_steps, s.T, "cuda")
+        probs.append(B.Problem(Kh, Vh, g.Q, s.T, g.step_id, g.prot, g.steps(), g.budget(), K_out, V_out, out,
+                               pos_in=g.pos, kv_location=B.STEPKV_MEM_HOST, out_location=B.STEPKV_MEM_HOST,
+                               K_sal=[g.K[l] for l in tr.sal_layer_ids()]))
+        outs.append((out, K_out, V_out))
+    st = B.stepkv_compress(probs, B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for (n_ref, kept_ref, Kref, Vref), (out, K_out, V_out) in zip(refs, outs):
+        n = int(out.n_kept.item())
+        assert n == n_ref and torch.equal(out.kept_idx[:n], kept_ref)
+        for l in range(len(K_out)):
+            assert torch.equal(K_out[l][:, :n].cuda(), Kref[l])
+            assert torch.equal(V_out[l][:, :n].cuda(), Vref[l])

@@ -19,24 +19,14 @@ constexpr int kCompactCtasPerSm = 8;
 constexpr int kCompactUnroll = 4;
 constexpr int kCompactLayersPerLaunch = 96;
 
-struct CompactArgs {
-  const uint8_t* src[2 * kCompactLayersPerLaunch];  // per (layer, tensor): base of [Hkv][rows][d]
-  uint8_t* dst[2 * kCompactLayersPerLaunch];
+// The in-place move kernel's arguments: the row sets of up to kCompactLayersPerLaunch layers.
+struct CompactMoveArgs {
+  uint8_t* dst[2 * kCompactLayersPerLaunch];  // per (layer, tensor): base of [Hkv][rows][d]
   int n_sets;               // n_layers_in_launch * n_tensors * Hkv
   int Hkv;
   int row_bytes;            // d * 2
-  int64_t in_head_bytes;
   int64_t out_head_bytes;
   int T;
-  const int32_t* kept_idx;
-  const int32_t* n_kept;
-  int kept_cap;
-  const int32_t* step_id_in;
-  const int32_t* pos_in;
-  int32_t* step_id_out;
-  int32_t* pos_out;
-  int gather_meta;          // this launch also gathers step_id / pos
-  int32_t* status;
 };
 
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
@@ -233,7 +223,7 @@ __global__ void __launch_bounds__(kCompactThreads) compact_plan_kernel(
   }
 }
 
-__global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __grid_constant__ CompactArgs a,
+__global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __grid_constant__ CompactMoveArgs a,
                                                                        const int32_t* plan) {
   pdl_wait();
   pdl_launch_dependents();
@@ -291,7 +281,7 @@ stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V
   for (int l0 = 0; e == cudaSuccess && l0 < std::max(n_layers, 1); l0 += kCompactLayersPerLaunch) {
     const int nl = std::min(kCompactLayersPerLaunch, n_layers - l0);
     if (nl <= 0) break;
-    CompactArgs a;
+    CompactMoveArgs a;
     memset(&a, 0, sizeof(a));
     for (int l = 0; l < nl; ++l) {
       a.dst[l * n_tensors] = static_cast<uint8_t*>(K[l0 + l]);
@@ -302,7 +292,6 @@ stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V
     a.row_bytes = d * 2;
     a.out_head_bytes = head_stride * 2;
     a.T = T;
-    a.status = status;
     const int64_t rows_max = (int64_t)a.n_sets * std::max(std::min(kept_cap, T - 1), 1);
     const int64_t want = (rows_max + 31) / 32;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * kCompactCtasPerSm, want));

@@ -193,14 +193,10 @@ __device__ __forceinline__ float tree_max(const float* v) {
   }
 }
 
-// Pass 1: fold NCHUNK x 32 logits of one query row into its running (m, Z), Z = sum 2^((s - m) c).
+// Sum over NCHUNK x 32 logits of one query row of 2^((s - ref) c).
 template <int NCHUNK>
-__device__ __forceinline__ void row_stats_update(const float (&va)[32], const float (&vb)[32], float c, float& m,
-                                                 float& Z) {
-  float mn = fmaxf(tree_max<32>(va), m);
-  if (NCHUNK == 2) mn = fmaxf(mn, tree_max<32>(vb));
-  if (mn == -INFINITY) return;
-  const float nmc = -mn * c;
+__device__ __forceinline__ float chunk_sum(const float (&va)[32], const float (&vb)[32], float c, float ref) {
+  const float nmc = -ref * c;
   const uint64_t c2 = f2_pack(c, c), b2 = f2_pack(nmc, nmc);
   uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
@@ -221,7 +217,28 @@ __device__ __forceinline__ void row_stats_update(const float (&va)[32], const fl
   f2_unpack(acc2[1], s2, s3);
   f2_unpack(acc2[2], s4, s5);
   f2_unpack(acc2[3], s6, s7);
-  Z = Z * ex2_approx((m - mn) * c) + (((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7)));
+  return ((s0 + s1) + (s2 + s3)) + ((s4 + s5) + (s6 + s7));
+}
+
+// Pass 1: fold NCHUNK x 32 logits of one query row into its running (m, Z), Z = sum 2^((s - m) c).
+// m is a reference point, not necessarily the maximum: any m that keeps every term below fp32
+// overflow gives the same m c + log2 Z.  A chunk is summed against the current m and kept if the sum
+// stays below 2^60; only the row's first chunk and a chunk with a logit far above m (sum >= 2^60,
+// inf or nan) take the running maximum as the new m, so the per-chunk maximum is almost never needed.
+template <int NCHUNK>
+__device__ __forceinline__ void row_stats_update(const float (&va)[32], const float (&vb)[32], float c, float& m,
+                                                 float& Z) {
+  if (m != -INFINITY) {
+    const float s = chunk_sum<NCHUNK>(va, vb, c, m);
+    if (s < 0x1p60f) {
+      Z += s;
+      return;
+    }
+  }
+  float mn = fmaxf(tree_max<32>(va), m);
+  if (NCHUNK == 2) mn = fmaxf(mn, tree_max<32>(vb));
+  if (mn == -INFINITY) return;  // every logit so far masked
+  Z = Z * ex2_approx((m - mn) * c) + chunk_sum<NCHUNK>(va, vb, c, mn);
   m = mn;
 }
 

@@ -86,6 +86,30 @@ def test_score_outlier_channels(B):
         TL.assert_close(sal[l].cpu().numpy(), O.window_attention_saliency(Ks[l], Qs[l]), "sal outliers")
 
 
+def test_score_logit_jumps(B):
+    """Logits that jump far above everything a row has seen earlier in its key range: the last 32 keys
+    of every 128 sit 4.5 higher in every channel along the queries' common direction (about 2^73 above
+    the rest after the log2(e)/sqrt(d) scale), and the last 32 of every 512 sit 9 higher (2^147: a sum
+    taken against the earlier maximum overflows fp32).  Masses below 1e-30 are compared absolutely (the
+    kernel's exponential flushes results below 2^-126 to zero)."""
+    import torch
+    rng = np.random.default_rng(77)
+    Hkv, G, d, T, W = 2, 2, 128, 2000, 16
+    j = np.arange(T)
+    t = np.where(j % 512 >= 480, 9.0, np.where(j % 128 >= 96, 4.5, 0.0)).astype(np.float32)
+    K = wl.f32_to_bf16_bits(rng.standard_normal((Hkv, T, d)).astype(np.float32) * 0.25 + t[None, :, None])
+    Q = wl.f32_to_bf16_bits(rng.standard_normal((Hkv * G, W, d)).astype(np.float32) * 0.25 + 1.0)
+    st = B.new_status()
+    sal = B.stepkv_score([TL.bf16_dev(K)], [TL.bf16_dev(Q)], T, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    g = sal[0].cpu().numpy()
+    ref = O.window_attention_saliency(K, Q)
+    assert np.all(np.isfinite(g))
+    TL.assert_close(g, ref, "sal (logit jumps)", floor=1e-30)
+    assert np.allclose(g.sum(axis=1), W, rtol=1e-4)
+
+
 # ------------------------------------------------------------------------------------ stages 2-4
 def _select_case(B, tr, p, sal_fp32, kept_cap=None):
     import torch

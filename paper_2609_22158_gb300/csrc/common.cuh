@@ -129,7 +129,9 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t base, uint32_t ncols) {
 
 // 32 lanes x 32 consecutive 32-bit columns: thread i of the warp receives row (lane base + i).  The load
 // and its completion wait sit in one asm statement, so no use of the registers can be scheduled before
-// the data has arrived.
+// the data has arrived.  The statement reads and writes no memory (no memory clobber), so shared-memory
+// loads that do not depend on the registers may be scheduled across it; being volatile, it keeps its
+// place among the mbarrier waits and tcgen05 fences.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   uint32_t r[32];
   asm volatile(
@@ -141,8 +143,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
         "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
         "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
         "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr)
-      : "memory");
+      : "r"(taddr));
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }

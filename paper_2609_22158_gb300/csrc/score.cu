@@ -242,41 +242,44 @@ __device__ __forceinline__ void row_stats_update(const float (&va)[32], const fl
   m = mn;
 }
 
-// Pass 2: sum over 32 query columns of 2^(s c - off_r) for key j; columns whose causal limit pw_r is
-// below j contribute nothing (only tiles that reach into the window need the test).
-__device__ __forceinline__ float key_mass(const float (&v)[32], const float* negoff, const int* pw, int j,
-                                          bool need_mask, float c) {
+// Pass 2: one 32-column chunk of a warp's 32 keys, read with two 16x256b loads (ra: the quarter's lanes
+// 0-15, rb: lanes 16-31).  Register 4k + e of a load holds lane lane/4 + 8 (e >= 2) and column
+// 8k + 2 (lane % 4) + (e & 1), so a thread sees 4 keys, lane/4 + 8 kk (kk < 4), and 8 columns of the
+// chunk, whose offsets o2[k] (pairs of columns) it loaded from the unit's table.  acc2[kk] collects
+// 2^(s c - off_r) over those columns for key kk in pairs; columns whose causal limit pw_r is below the
+// key contribute nothing (only tiles that reach into the window need the test, jq = key of kk = 0).
+__device__ __forceinline__ void chunk_mass(const uint32_t (&ra)[16], const uint32_t (&rb)[16], const uint64_t (&o2)[4],
+                                           const int* pw, int jq, bool need_mask, float c, uint64_t (&acc2)[4]) {
   if (!need_mask) {
     const uint64_t c2 = f2_pack(c, c);
-    uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
-    for (int i = 0; i < 32; i += 8) {
+    for (int k = 0; k < 4; ++k) {
 #pragma unroll
-      for (int k2 = 0; k2 < 4; ++k2) {
-        const float2 o = *reinterpret_cast<const float2*>(&negoff[i + 2 * k2]);
+      for (int kk = 0; kk < 4; ++kk) {
+        const uint32_t* r = kk < 2 ? ra : rb;
+        const int e = 4 * k + (kk & 1) * 2;
         float lo, hi;
-        f2_unpack(f2_fma(f2_pack(v[i + 2 * k2], v[i + 2 * k2 + 1]), c2, f2_pack(o.x, o.y)), lo, hi);
-        acc2[k2] = f2_add(acc2[k2], f2_pack(ex2_approx(lo), ex2_approx(hi)));
+        f2_unpack(f2_fma(f2_pack(__uint_as_float(r[e]), __uint_as_float(r[e + 1])), c2, o2[k]), lo, hi);
+        acc2[kk] = f2_add(acc2[kk], f2_pack(ex2_approx(lo), ex2_approx(hi)));
       }
     }
-    float t0, t1, t2, t3, t4, t5, t6, t7;
-    f2_unpack(acc2[0], t0, t1);
-    f2_unpack(acc2[1], t2, t3);
-    f2_unpack(acc2[2], t4, t5);
-    f2_unpack(acc2[3], t6, t7);
-    return ((t0 + t1) + (t2 + t3)) + ((t4 + t5) + (t6 + t7));
+    return;
   }
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-  for (int i = 0; i < 32; i += 4) {
-    const float4 o = *reinterpret_cast<const float4*>(&negoff[i]);
-    const int4 w = *reinterpret_cast<const int4*>(&pw[i]);
-    s0 += j <= w.x ? ex2_approx(fmaf(v[i + 0], c, o.x)) : 0.f;
-    s1 += j <= w.y ? ex2_approx(fmaf(v[i + 1], c, o.y)) : 0.f;
-    s2 += j <= w.z ? ex2_approx(fmaf(v[i + 2], c, o.z)) : 0.f;
-    s3 += j <= w.w ? ex2_approx(fmaf(v[i + 3], c, o.w)) : 0.f;
+  for (int k = 0; k < 4; ++k) {
+    const int2 w = *reinterpret_cast<const int2*>(&pw[8 * k]);
+    float ox, oy;
+    f2_unpack(o2[k], ox, oy);
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      const uint32_t* r = kk < 2 ? ra : rb;
+      const int e = 4 * k + (kk & 1) * 2;
+      const int jk = jq + 8 * kk;
+      const float t0 = jk <= w.x ? ex2_approx(fmaf(__uint_as_float(r[e]), c, ox)) : 0.f;
+      const float t1 = jk <= w.y ? ex2_approx(fmaf(__uint_as_float(r[e + 1]), c, oy)) : 0.f;
+      acc2[kk] = f2_add(acc2[kk], f2_pack(t0, t1));
+    }
   }
-  return (s0 + s1) + (s2 + s3);
 }
 
 __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
@@ -730,24 +733,43 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         tc_fence_after();
         const int key0 = tile * kKeyTile;
         const bool need_mask = key0 + kKeyTile - 1 > Tb - g.W;  // tile reaches into the causal window
-        // Keys on the TMEM lanes: this warp sums its key's mass over query columns s2*32 + 64 i, one
-        // 32-column chunk at a time (holding two chunks in registers spills).  The buffer is released
-        // once the warp's last chunk is in registers.
+        // Keys on the TMEM lanes: this warp covers its quarter's 32 keys over query columns s2*32 + 64 i
+        // (32-column chunks, one TMEM round trip each; holding two chunks in registers spills).  Per
+        // chunk a thread needs 8 row offsets, so the shared-memory reads per logit drop fourfold against
+        // the one-key-per-thread 32x32b layout.  The buffer is released once the warp's last chunk is in
+        // registers.
         const int n_cols = (r.rows + 31) & ~31;
-        const int j = key0 + q * 32 + lane;
-        float acc = 0.f;
-        bool released = false;
-#pragma unroll 1
-        for (int cc = s2 * 32; cc < n_cols; cc += 64) {
-          float v[32];
-          tmem_ld32(lane_base + (uint32_t)cc, v);
-          if (cc + 64 >= n_cols) {
-            release_buffer();
-            released = true;
+        const int lq = lane & 3;
+        const int jq = key0 + q * 32 + (lane >> 2);
+        uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int cc = s2 * 32 + 64 * i;
+          if (cc < n_cols) {
+            uint64_t o2[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) o2[k] = *reinterpret_cast<const uint64_t*>(&negoff[cc + 8 * k + 2 * lq]);
+            uint32_t ra[16], rb[16];
+            tmem_ld16x256x4_pair(lane_base + (uint32_t)cc, lane_base + (16u << 16) + (uint32_t)cc, ra, rb);
+            if (cc + 64 >= n_cols) release_buffer();
+            chunk_mass(ra, rb, o2, pw_tab + cc + 2 * lq, jq, need_mask, c, acc2);
           }
-          acc += key_mass(v, negoff + cc, pw_tab + cc, j, need_mask, c);
         }
-        if (!released) release_buffer();
+        if (s2 * 32 >= n_cols) release_buffer();  // no chunk for this warp
+        // each key's sum is spread over the 4 threads of a quad (lane % 4): reduce in a fixed order, then
+        // thread `lane` reports key lane/4 + 8 (lane % 4) of the quarter
+        float sk[4];
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          float lo, hi;
+          f2_unpack(acc2[kk], lo, hi);
+          sk[kk] = lo + hi;
+          sk[kk] += __shfl_xor_sync(0xffffffffu, sk[kk], 1);
+          sk[kk] += __shfl_xor_sync(0xffffffffu, sk[kk], 2);
+        }
+        const float acc = lq == 0 ? sk[0] : lq == 1 ? sk[1] : lq == 2 ? sk[2] : sk[3];
+        const int lk = (lane >> 2) + 8 * lq;
+        const int j = key0 + q * 32 + lk;
         if (p.accumulate) {
           // fused pass: each warp adds its share of the rows straight into the per-token fixed-point
           // sum (integer addition: the total does not depend on the order of arrival)
@@ -756,10 +778,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           // saliency rows: the group's two warps on this quarter combine in a fixed order (the slot
           // alternates between the group's items, so a write never meets a pending read)
           float* comb = combf + (n_done & 1) * 128;
-          if (s2 == 1) comb[q * 32 + lane] = acc;
+          if (s2 == 1) comb[q * 32 + lk] = acc;
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
           if (s2 == 0 && j < Tb) {
-            const float val = (acc + comb[q * 32 + lane]) * g.inv_G;
+            const float val = (acc + comb[q * 32 + lk]) * g.inv_G;
             const int pair = p.pair0 + il.ul / g.n_rg, rg = il.ul % g.n_rg;
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }

@@ -668,11 +668,10 @@ def main():
                          "(default: the capture of the current compaction kernel for the 32-layer 32K workload)")
     args = ap.parse_args()
     if args.compact_traffic is None and args.T == 32768 and args.layers == 32:
-        # dram__bytes_read.sum + dram__bytes_write.sum of compact_kernel from one ncu capture of the
-        # 8-layer variant of this workload (109.80 MB read + 58.67 MB written), scaled by row sets (x4):
-        # the kernel does the same work per row set.  Writes below the algorithmic bytes are dirty lines
-        # still in L2 when the kernel ends.
-        args.compact_traffic = 4 * (109.800960e6 + 58.666496e6)
+        # dram__bytes_read.sum + dram__bytes_write.sum of compact_kernel from one single-pass ncu capture
+        # of this workload at full size (the timed step's launch): 438.94 MB read + 388.77 MB written.
+        # The ~50 MB of writes below the algorithmic bytes are dirty lines still in L2 when it ends.
+        args.compact_traffic = 438.94e6 + 388.77e6
     if args.impl == "reference":
         run_reference(args)
     else:

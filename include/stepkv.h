@@ -26,6 +26,13 @@
  *    aligned).  Calls on different streams with different workspaces may run concurrently.
  *    The one exception is stepkv_select_static_scratch (below), which takes no workspace and uses
  *    a fixed scratch array compiled into the library instead.
+ *  - CUDA graphs: the calls issue kernel launches only (no copies, memsets or synchronisation), so a
+ *    call can be captured into a CUDA graph and replayed, with new data in the same buffers between
+ *    replays.  The saliency kernel orders its blocks through flags in the workspace; the value a
+ *    launch publishes mixes a per-call host value with an epoch kept in the workspace and advanced
+ *    by every launch, so a replay never mistakes the previous launch's flags for its own.  The
+ *    workspace needs no initialisation.  Make one ordinary call before capturing (it sets the
+ *    kernels' shared-memory limits, which must not happen during a capture).
  *  - Errors: argument problems are detected on the host and returned (STEPKV_EINVAL,
  *    STEPKV_EUNSUPPORTED, STEPKV_ENOSPACE) before anything is enqueued.  A failed launch returns
  *    STEPKV_ECUDA.  Data-dependent problems found on the device (a step id out of range, kept_cap

@@ -73,10 +73,11 @@ struct ScoreLaunch {
   int64_t out_stride;
   int accumulate;     // 1: pass 2 adds into each trajectory's t_acc (zeroed first) instead of writing rows
   int acc_shift;      // k: fixed-point scale 2^k of t_acc
-  unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores `token` once its partials are written
-  unsigned long long* zflags; // [grid] CTA b stores `token` once its share of the accumulators is zeroed
-  unsigned long long token;   // unique per launch, so flags left by earlier launches never match
-  unsigned long long wait_token;     // the value the pass-2 wait looks for (token, except in the self-test)
+  unsigned long long* flags;  // [grid] pass-1-done flags: CTA b stores the launch token once its partials are written
+  unsigned long long* zflags; // [grid] CTA b stores the launch token once its share of the accumulators is zeroed
+  unsigned long long* epoch;  // per-workspace launch counter, advanced by CTA 0 at the end of every launch
+  unsigned long long token;   // host value, unique per call; mixed with the epoch into the launch token
+  int selftest;               // 1: the pass-2 wait looks for a value no CTA publishes (failure-path self-test)
   unsigned long long wait_limit_ns;  // the pass-2 wait gives up (STEPKV_ETIMEOUT) after this long
   int32_t* status;
 };
@@ -292,6 +293,17 @@ __device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned l
   asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
+// The launch token every CTA publishes in its flags.  It mixes the host's per-call value with the
+// workspace's epoch, which CTA 0 advances at the end of each launch, so a launch replayed from a CUDA
+// graph (same host value) still differs from the launch before it, and flags left in the workspace by
+// earlier launches never match.  All CTAs read the epoch after the stream's earlier work is complete
+// and before CTA 0 can advance it: CTA 0 advances it only after every CTA has published its zero flag.
+__device__ __forceinline__ unsigned long long launch_token(const ScoreLaunch& p) {
+  const unsigned long long e = ld_relaxed_u64(p.epoch);
+  const unsigned long long t = p.token ^ ((e + 1ull) * 0x9E3779B97F4A7C15ull);
+  return t == 0ull ? 1ull : t;
+}
+
 // Both passes in one launch.  A CTA owns a contiguous range of (unit, key tile) items; it streams them
 // forward for pass 1 (in pairs of tiles: one N = 256 MMA per query half) and backward for pass 2, so
 // the TMA ring, the MMA issuer and the Q staging run on without a break at the change of pass (the
@@ -366,6 +378,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   // Every thread waits for the earlier kernels on the stream before its first global access.
   pdl_wait();
   pdl_launch_dependents();
+  const unsigned long long tok = launch_token(p);
+  const unsigned long long wait_tok = p.selftest ? ~tok : tok;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -543,18 +557,21 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       if (lane == 0) mbar_arrive(&acc_empty[grp]);
     };
 
-    // The first epilogue warp zeroes this CTA's share of the accumulators while the first tiles stream
-    // in, then publishes it (fence + release store of the launch's token): a CTA adds into the
-    // accumulators only after it has seen every CTA's zero flag.
-    if (p.accumulate && ew == 0) {
-      for (int b = 0; b < p.n_traj; ++b) {
-        unsigned long long* acc = p.traj[b].t_acc;
-        for (int i = blockIdx.x * 32 + lane; i < p.traj[b].T; i += gridDim.x * 32) acc[i] = 0ull;
+    // The first epilogue warp zeroes this CTA's share of the accumulators (when the launch accumulates)
+    // while the first tiles stream in, then publishes its zero flag (fence + release store of the launch
+    // token): a CTA adds into the accumulators only after it has seen every CTA's zero flag, and CTA 0
+    // advances the epoch only after that too.
+    if (ew == 0) {
+      if (p.accumulate) {
+        for (int b = 0; b < p.n_traj; ++b) {
+          unsigned long long* acc = p.traj[b].t_acc;
+          for (int i = blockIdx.x * 32 + lane; i < p.traj[b].T; i += gridDim.x * 32) acc[i] = 0ull;
+        }
       }
       __syncwarp();
       if (lane == 0) {
         __threadfence();
-        st_release_u64(&p.zflags[blockIdx.x], p.token);
+        st_release_u64(&p.zflags[blockIdx.x], tok);
       }
     }
 
@@ -635,7 +652,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         if (ew == 0 && lane == 0) {
           if (mbar_wait(p1_flushed, 0, abort_flag)) {
             __threadfence();
-            st_release_u64(&p.flags[blockIdx.x], p.token);
+            st_release_u64(&p.flags[blockIdx.x], tok);
           } else {
             ok = false;
           }
@@ -671,10 +688,10 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const uint64_t t0 = globaltimer_ns();
             for (uint32_t it = 0; !all; ++it) {
               bool mine = true;
-              for (int b = c0 + lane; b <= c1; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == p.wait_token;
+              for (int b = c0 + lane; b <= c1; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == wait_tok;
               if (!zeros_seen) {
 #pragma unroll 4
-                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.zflags[b]) == p.wait_token;
+                for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.zflags[b]) == wait_tok;
               }
               all = __all_sync(0xffffffffu, mine);
               if (!all && (it & 15u) == 15u && (*abort_flag || globaltimer_ns() - t0 > p.wait_limit_ns)) break;
@@ -802,6 +819,18 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
+  if (blockIdx.x == 0 && warp == 0) {
+    // every CTA has read the epoch once its zero flag carries this launch's token (bounded wait; the
+    // epoch advances in any case, so the next launch's token differs from this one)
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 0;; ++it) {
+      bool mine = true;
+      for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.zflags[b]) == tok;
+      if (__all_sync(0xffffffffu, mine)) break;
+      if ((it & 15u) == 15u && globaltimer_ns() - t0 > p.wait_limit_ns) break;
+    }
+    if (lane == 0) atomicAdd(p.epoch, 1ull);
+  }
 }
 
 // -------------------------------------------------------------------------------------------------
@@ -867,7 +896,8 @@ static size_t score_partial_slots_bytes(int n_traj, int n_layers, int Hkv, int H
   return (size_t)(n_traj * n_layers * Hkv * n_rg + kMaxGrid) * kPartEntries * kMaxRows * sizeof(float2);
 }
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W, int n_traj) {
-  return score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W) + 2 * (size_t)kMaxGrid * sizeof(unsigned long long);
+  // partial slots, pass-1 flags, zero flags, launch epoch (16 B)
+  return score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W) + 2 * (size_t)kMaxGrid * sizeof(unsigned long long) + 16;
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -956,6 +986,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.flags = reinterpret_cast<unsigned long long*>(reinterpret_cast<uint8_t*>(part) +
                                                   score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W));
   L.zflags = L.flags + kMaxGrid;
+  L.epoch = L.zflags + kMaxGrid;
   L.out = rows_out;
   L.out_stride = out_stride;
   L.accumulate = trajs[0].t_acc != nullptr ? 1 : 0;
@@ -989,7 +1020,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.token = next_launch_token();
   // Self-test of the failure path: the pass-2 wait looks for a value no CTA ever publishes, so every
   // CTA's wait runs out after selftest_wait_ns and the kernel takes its abort path.
-  L.wait_token = selftest_wait_ns ? ~L.token : L.token;
+  L.selftest = selftest_wait_ns ? 1 : 0;
   L.wait_limit_ns = selftest_wait_ns ? selftest_wait_ns : kWaitLimitNs;
   e = d == 128 ? launch_score<2>(L, grid, stream) : launch_score<1>(L, grid, stream);
   if (e != cudaSuccess) { set_last_cuda_error(e); return STEPKV_ECUDA; }

@@ -383,11 +383,12 @@ static const void* const* sal_keys(const stepkv_problem_t& p) {
 
 // Saliency batches of the fused pass: runs of consecutive trajectories with one head shape (lengths and
 // strides may differ), up to kMaxScoreBatch trajectories and kMaxScoreMaps tensor maps each, share one
-// launch -- as long as the batch's saliency keys fit in half of L2.  The second pass walks each CTA's
-// tiles backwards and finds the ones the first pass read last still in L2; a trajectory whose keys fit
-// in L2 gets all of them there when it runs alone, and a batch only pays if that still holds, so short
-// trajectories (where the launch's fixed costs dominate) are batched and long ones run one per launch.
-constexpr size_t kSalBatchBytes = 64ull << 20;
+// launch while the batch's saliency keys total at most kSalBatchBytes.  Each launch has fixed costs (the
+// ring's first fill, the change of pass, the exit skew: ~20 us), which a batch pays once; against that,
+// the second pass finds fewer of the tiles the first pass read last still in L2 the more keys a launch
+// streams.  512 MB is the measured optimum for 16 trajectories of 8K-32K tokens (Llama-3-8B heads:
+// 64 MB 2.68 ms, 256 MB 2.58, 512 MB 2.48, 1 GB 2.54, one launch for all 2.82 ms at a 10% budget).
+constexpr size_t kSalBatchBytes = 512ull << 20;
 struct SalBatch {
   int first, n;
 };

@@ -42,7 +42,7 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 // trajectories share it, so short ones do not each pay a launch and a tail).  The row items of all
 // trajectories form one list, in trajectory order, split into equal contiguous ranges per CTA.
 constexpr int kCompactMaxTraj = 16;
-constexpr int kCompactMaxTensors = 192;  // (layer, tensor) entries per launch
+constexpr int kCompactMaxTensors = 1024;  // (layer, tensor) entries per launch: 16 trajectories x 32 layers x K, V
 
 struct CompactTraj {
   int tensor0;              // first (layer, tensor) entry of this trajectory in src / dst

@@ -5,8 +5,9 @@
 // GB300 design.  The softmax normalises over keys while A sums over query rows, so the two
 // reductions run in two tensor-core passes over K, each in the orientation that makes its
 // reduction a per-thread loop over TMEM columns:
-//   pass 1  S   = Q . K^T  (M = 128 query rows, N = 128 keys): per-row running max m and
-//                 Z = sum 2^((s - m) c), c = log2(e)/sqrt(d); one partial (m, Z) per CTA segment;
+//   pass 1  S   = Q . K^T  (M = 128 query rows, N = 256 keys): per-row reference point m (a running
+//                 maximum, moved only when a chunk would overflow) and Z = sum 2^((s - m) c),
+//                 c = log2(e)/sqrt(d); one partial (m, Z) per CTA segment;
 //   pass 2  S^T = K . Q^T  (M = 128 keys, N = up to 256 query rows): per-key
 //                 sum_r 2^(s c - off_r), off_r = m_r c + log2 Z_r combined from the pass-1 partials.
 // Both passes run in one cooperative launch.  Each CTA (one per SM) owns a contiguous range of

@@ -200,7 +200,8 @@ def compact_rows(X: np.ndarray, kept: np.ndarray) -> np.ndarray:
 
 def step_statistics(T_hat, step_id, prunable, chosen, n_steps: int) -> Dict[str, np.ndarray]:
     """Per-step accounting over prunable tokens (the evicted/retained-by-step view of Figs. 2 and 8):
-    token count, sum and max of normalised saliency, and retained count."""
+    token count, sum and max of normalised saliency, and retained count.  Keyed by each token's own
+    step id; protected tokens enter no figure; a step with no prunable token reports zeros."""
     T_hat = np.asarray(T_hat, np.float64)
     count = np.zeros(n_steps, np.int64)
     ssum = np.zeros(n_steps, np.float64)

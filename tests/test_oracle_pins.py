@@ -418,6 +418,55 @@ def test_boundary_invariants_tiny():
         assert np.array_equal(C[:, r, :], V[:, kept[r], :])
 
 
+# ------------------------------------------------------------------ per-step accounting (hand table)
+def _step_table():
+    rows = _load_table("step_statistics.txt")
+    tok = [r[1:] for r in rows if r[0] == "tok"]
+    step = [r[1:] for r in rows if r[0] == "step"]
+    step_id = np.array([int(r[1]) for r in tok], np.int32)
+    prot = np.array([int(r[2]) for r in tok], np.uint8)
+    T_raw = np.array([float(r[3]) for r in tok])
+    T_hat = np.array([float(r[4]) for r in tok])
+    exp = {"count": np.array([int(r[1]) for r in step]), "sal_sum": np.array([float(r[2]) for r in step]),
+           "sal_max": np.array([float(r[3]) for r in step]), "kept": np.array([int(r[4]) for r in step])}
+    return step_id, prot, T_raw, T_hat, exp
+
+
+def _assert_step_stats(st, exp, prefix=""):
+    assert np.array_equal(st[prefix + "count"], exp["count"]), (st[prefix + "count"], exp["count"])
+    assert np.allclose(st[prefix + "sal_sum"], exp["sal_sum"], rtol=0, atol=1e-12), st[prefix + "sal_sum"]
+    assert np.allclose(st[prefix + "sal_max"], exp["sal_max"], rtol=0, atol=1e-12), st[prefix + "sal_max"]
+    assert np.array_equal(st[prefix + "kept"], exp["kept"]), (st[prefix + "kept"], exp["kept"])
+
+
+def check_step_statistics_table(O):
+    """step_statistics on the table's T_hat and retained set {4, 5, 9}."""
+    step_id, prot, _, T_hat, exp = _step_table()
+    st = O.step_statistics(T_hat, step_id, ~prot.astype(bool), np.array([4, 5, 9]), len(exp["count"]))
+    _assert_step_stats(st, exp)
+
+
+def check_boundary_step_statistics(O):
+    """The whole boundary from raw saliency: normalisation over prunable tokens, alpha = 1, beta = 0,
+    count budget 3 -- the per-step figures must be those of the table (computed on T_hat)."""
+    step_id, prot, T_raw, T_hat, exp = _step_table()
+    n = len(exp["count"])
+    p = O.Params(alpha=1.0, beta=0.0)
+    z = np.zeros(n)
+    out = O.stepkv_boundary([T_raw[None, :]], step_id, prot, z + 1.0, z, z, None, z, p, "count", count=3)
+    assert np.allclose(out["T_hat"], T_hat, rtol=0, atol=1e-15)
+    assert out["N"] == 7 and out["B"] == 3 and list(out["chosen"]) == [4, 5, 9]
+    _assert_step_stats(out, exp, prefix="step_")
+
+
+def test_step_statistics_table():
+    check_step_statistics_table(REAL)
+
+
+def test_boundary_step_statistics():
+    check_boundary_step_statistics(REAL)
+
+
 # ------------------------------------------------------------------ planted mistakes
 def _mutant(**overrides):
     ns = types.SimpleNamespace(**{k: getattr(REAL, k) for k in dir(REAL) if not k.startswith("__")})
@@ -541,6 +590,41 @@ def _decode_unnormalised(q, K, V):
     return out
 
 
+def _stats_keyed_previous_step(T_hat, step_id, prunable, chosen, n_steps):
+    # keyed by step_id - 1: step 0's tokens wrap into the last step (totals unchanged)
+    return REAL.step_statistics(T_hat, np.asarray(step_id) - 1, prunable, chosen, n_steps)
+
+
+def _stats_max_over_all(T_hat, step_id, prunable, chosen, n_steps):
+    # maximum taken over protected tokens of a step as well
+    st = REAL.step_statistics(T_hat, step_id, prunable, chosen, n_steps)
+    smax = np.zeros(n_steps)
+    for i in range(len(T_hat)):
+        k = int(step_id[i])
+        if 0 <= k < n_steps:
+            smax[k] = max(smax[k], T_hat[i])
+    st["sal_max"] = smax
+    return st
+
+
+def _stats_count_protected(T_hat, step_id, prunable, chosen, n_steps):
+    # counts every token of a step, protected ones included
+    st = REAL.step_statistics(T_hat, step_id, prunable, chosen, n_steps)
+    sid = np.asarray(step_id)
+    st["count"] = np.array([int((sid == k).sum()) for k in range(n_steps)])
+    return st
+
+
+def _boundary_stats_on_raw(A_layers, step_id, prot, valid, gain, red, obs_sim, reuse_prev, p, budget_mode,
+                           num=1, den=1, count=0):
+    # per-step sums and maxima of the raw saliency T instead of the normalised T_hat
+    out = REAL.stepkv_boundary(A_layers, step_id, prot, valid, gain, red, obs_sim, reuse_prev, p, budget_mode,
+                               num, den, count)
+    st = REAL.step_statistics(out["T"], step_id, ~np.asarray(prot).astype(bool), out["chosen"], len(valid))
+    out.update({"step_" + k: v for k, v in st.items()})
+    return out
+
+
 @pytest.mark.parametrize("check, mutant", [
     (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
     (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
@@ -556,6 +640,10 @@ def _decode_unnormalised(q, K, V):
     (check_decode_two_key_analytic, _mutant(decode_attention=_decode_no_scale)),
     (check_decode_identical_keys, _mutant(decode_attention=_decode_unnormalised)),
     (check_decode_bruteforce, _mutant(decode_attention=_decode_no_scale)),
+    (check_step_statistics_table, _mutant(step_statistics=_stats_keyed_previous_step)),
+    (check_step_statistics_table, _mutant(step_statistics=_stats_max_over_all)),
+    (check_step_statistics_table, _mutant(step_statistics=_stats_count_protected)),
+    (check_boundary_step_statistics, _mutant(stepkv_boundary=_boundary_stats_on_raw)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

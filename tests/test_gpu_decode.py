@@ -1,8 +1,9 @@
 """GPU parity of decode attention over a (compacted) cache against the CPU oracle, through the C ABI.
 
-Tolerance: per layer and query head, max |gpu - oracle| <= 2e-3 x max |oracle| over the head's output
-row.  The GPU computes logits in fp32 from exact bf16 products, exponentials with the MUFU ex2 and
-fp32 sums over at most a few thousand weighted rows, so its error is orders of magnitude below that.
+Tolerance: element by element, |gpu - oracle| <= 2e-3 x max(|oracle|, 1e-3 x m), where m is the magnitude
+of the weighted sum's terms, sum_j p_j |V[j]| (stepkv_testlib.DECODE_FLOOR).  The GPU computes logits in
+fp32 from exact bf16 products, exponentials with the MUFU ex2 and fp32 sums over at most a few thousand
+weighted rows, so its error is orders of magnitude below that.
 """
 import numpy as np
 import pytest
@@ -27,13 +28,6 @@ def B():
 
 def _bits(rng, shape, scale=1.0):
     return wl.f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32) * np.float32(scale))
-
-
-def _assert_heads_close(g, o, what):
-    for h in range(o.shape[0]):
-        scale = np.abs(o[h]).max()
-        err = np.abs(g[h] - o[h]).max()
-        assert err <= TOL * scale, f"{what} head {h}: max error {err:.3e} vs scale {scale:.3e}"
 
 
 DECODE_CASES = [
@@ -61,8 +55,7 @@ def test_decode_matches_oracle(B, Hkv, G, d, n, rows, L, ks):
     torch.cuda.synchronize()
     assert st.item() == 0
     for l in range(L):
-        ref = O.decode_attention(qs[l], Ks[l][:, :n], Vs[l][:, :n])
-        _assert_heads_close(out[l].cpu().numpy(), ref, f"layer {l}")
+        TL.assert_decode_close(out[l].cpu().numpy(), qs[l], Ks[l][:, :n], Vs[l][:, :n], f"layer {l}")
 
 
 def test_decode_n_on_device_equals_host_n(B):
@@ -109,5 +102,5 @@ def test_decode_over_compacted_cache(B):
     n = int(g.out.n_kept.item())
     kept = g.out.kept_idx[:n].cpu().numpy()
     for l in range(tr.shape.L):
-        ref = O.decode_attention(qs[l], O.compact_rows(tr.keys(l), kept), O.compact_rows(tr.values(l), kept))
-        _assert_heads_close(out[l].cpu().numpy(), ref, f"layer {l}")
+        TL.assert_decode_close(out[l].cpu().numpy(), qs[l], O.compact_rows(tr.keys(l), kept),
+                               O.compact_rows(tr.values(l), kept), f"layer {l}")

@@ -82,6 +82,26 @@ class _Case:
             _assert_close(getattr(s, name).cpu().numpy(), getattr(w, name).cpu().numpy(), name)
         _assert_close(self.reuse_out["static"].cpu().numpy(), self.reuse_out["ws"].cpu().numpy(), "reuse_out")
 
+    def compare_oracle(self):
+        """The static-scratch outputs against the CPU oracle on the same saliency rows (T_i = mean of the
+        three rows, then Eqs. 1-5 and Algorithm 1)."""
+        from oracle import stepkv_oracle as O
+        tr, o = self.tr, self.out["static"]
+        b = tr.budget
+        ref = O.stepkv_boundary([self.sal.cpu().numpy().astype(np.float64)], tr.step_id, tr.prot, tr.valid, tr.gain,
+                                tr.red, tr.obs_sim, tr.reuse, O.Params(), b.mode, b.num, b.den, b.count)
+        n = int(o.n_kept.item())
+        assert n == len(ref["kept"])
+        assert TL.compare_kept(o.kept_idx[:n].cpu().numpy().astype(np.int64), ref) == 0
+        prunable = ~tr.prot.astype(bool)
+        TL.assert_close(o.priority.cpu().numpy()[prunable], ref["P"][prunable], "P vs oracle", floor=1e-6)
+        TL.assert_close(o.step_util.cpu().numpy(), ref["S"], "S_k vs oracle", floor=1e-6)
+        TL.assert_close(self.reuse_out["static"].cpu().numpy(), ref["reuse"], "c_k vs oracle", floor=1e-6)
+        assert np.array_equal(o.step_count.cpu().numpy(), ref["step_count"])
+        assert np.array_equal(o.step_kept.cpu().numpy(), ref["step_kept"])
+        TL.assert_close(o.step_sal_sum.cpu().numpy(), ref["step_sal_sum"], "step_sal_sum vs oracle", floor=1e-9)
+        TL.assert_close(o.step_sal_max.cpu().numpy(), ref["step_sal_max"], "step_sal_max vs oracle", floor=1e-9)
+
 
 def test_static_scratch_matches_workspace_entry_point_twice_in_a_row(B):
     """Two static-scratch calls back to back on one stream (a cluster-sized trajectory, then a
@@ -98,17 +118,23 @@ def test_static_scratch_matches_workspace_entry_point_twice_in_a_row(B):
     torch.cuda.synchronize()
     for c in cases:
         c.compare()
+        c.compare_oracle()
 
 
 def test_static_scratch_call_allocates_nothing(B):
-    """After the first call on the device (the set-up), a call leaves torch's allocator untouched."""
+    """After the first call on the device (the set-up), a call leaves torch's allocator untouched and
+    the device's free memory (cudaMemGetInfo) unchanged: nothing inside the library allocates either."""
     import torch
     c = _Case(B, wl.custom(43, L=1, Hq=4, Hkv=1, d=64, T=7000, W=32, n_steps=12, budget=wl.Budget.ratio(1, 5)), 3)
     c.run(B, "static")
     torch.cuda.synchronize()
     alloc, reserved = torch.cuda.memory_allocated(), torch.cuda.memory_reserved()
+    free0, _ = torch.cuda.mem_get_info()
     c.run(B, "static")
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
     assert torch.cuda.memory_allocated() == alloc and torch.cuda.memory_reserved() == reserved
+    assert free1 == free0, (free0, free1)
     c.run(B, "ws")
     torch.cuda.synchronize()
     c.compare()

@@ -1,14 +1,25 @@
 """Benchmark of the fused StepKV compression pass (score -> reduce/fuse -> select -> compact).
 
-Workload (default): one Llama-3-8B-shaped trajectory per GPU -- 32 layers, 32 query / 8 KV heads,
-head dim 128, bf16, T = 32768 cached tokens, 40 reasoning steps, 64-token observation window,
-budget 10% of the prunable tokens -- drawn by the seeded generator (saliency layers, step layout,
-signals) and by torch's seeded device RNG (K/V of the other layers).  Inputs are resident in HBM when
-the timed region starts; an L2 flush (a 512 MB write) runs between timed steps, outside their events.
+Workloads (``--config``), all drawn by the seeded generator (saliency layers, step layout, signals) and
+by torch's seeded device RNG (K/V of the other layers):
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  1  tiny: 1 layer, Hq 8 / Hkv 2, d 64, T 2048, W 32, 8 steps, budget 25% (latency-bound)
+  2  (default) Llama-3-8B-shaped trajectory: 32 layers, Hq 32 / Hkv 8, d 128, T 32768, 40 steps,
+     W 64, 3 needle spans, budget 10%
+  3  16 ragged Llama-3-8B-shaped trajectories (T ~ U(8K, 32K), 4 outlier key channels) in one call,
+     budgets 5% / 10% / 20% (the line's value is the 10% figure)
+  4  Qwen2.5-32B-shaped trajectory: 64 layers, Hq 40 / Hkv 8, d 128, T 65536, 120 steps, W 128,
+     fixed budget 4096
+  5  incremental agent loop: Llama-3-8B heads, 200 boundaries growing from 4096 to 131072 tokens,
+     the compacted cache plus the new step compressed in place under a fixed 8192-token budget, 64
+     single-token decode reads after each compression
 
-Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank compresses its own trajectory
+Inputs are resident in HBM when the timed region starts; an L2 flush (a 512 MB write) runs between timed
+passes, outside their events.
+
+    python bench.py [--config N] [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line (rank 0).  Under torchrun (N > 1) every rank compresses its own trajectories
 (independent problems: weak scaling, no collective on the data path); timing is the max over ranks.
 """
 from __future__ import annotations
@@ -29,39 +40,72 @@ if ROOT not in sys.path:
 
 METRIC = "compressed tokens/sec (score+select+compact) at 32K ctx; % HBM roofline"
 UNIT = "tokens/s"
+# MUFU ex2 issue rate per SM per clock on this part: 32 (a standalone probe measured 9.4e12 ex2/s on
+# 152 SMs at 1.95 GHz); the peak below uses the maximum SM clock.
+MUFU_PER_CLK_SM = 32
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from single-pass, full-size ncu captures of the
+# current kernels (profiles/compact_kernel_llama8b_32k.md, profiles/score_kernel_llama8b_32k.md):
+# {config: {kernel: bytes}}.  A kernel absent here reports traffic null.
+NCU_TRAFFIC = {
+    2: {"compact_kernel": 438.94e6 + 388.77e6},
+}
 
 
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+        return {"hbm": float(d["hbm_gbs"]), "bf16": float(d["bf16_tflops"]),
+                "bf16_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "sm_mhz": float(d.get("sm_max_mhz", 2070.0)), "kind": "measured"}
     except Exception:
-        return 6800.0, 1900.0, "fallback"
+        return {"hbm": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "sm_mhz": 2070.0, "kind": "fallback"}
 
 
-# ---------------------------------------------------------------------------------- workload
-def make_traj(args):
+# ---------------------------------------------------------------------------------- workloads
+def make_trajs(cfg: int, seed=None):
+    """The trajectories of one bench configuration (config 5 is the incremental loop: see run_incremental)."""
     from paper_2609_22158_gb300 import workload as wl
-    return wl.llama8b_32k(seed=args.seed, T=args.T, L=args.layers)
+    if cfg == 1:
+        return [wl.tiny(0 if seed is None else seed)]
+    if cfg == 2:
+        return [wl.llama8b_32k(seed=1 if seed is None else seed)]
+    if cfg == 3:
+        return wl.ragged_batch(seed=2 if seed is None else seed)
+    if cfg == 4:
+        return [wl.qwen32b_64k(seed=3 if seed is None else seed)]
+    raise ValueError(cfg)
 
 
-def workload_config(tr, args, n):
+def describe(trs, budget_label=None):
+    tr = trs[0]
     s = tr.shape
     b = tr.budget
+    bud = budget_label or (f"{b.num}/{b.den} of prunable" if b.mode == "ratio" else f"{b.count} tokens")
+    if len(trs) == 1:
+        name = {"tiny": "tiny trajectory", "llama8b_32k": "llama3-8b-shaped agent trajectory",
+                "qwen32b_64k": "qwen2.5-32b-shaped long-horizon trajectory"}.get(tr.name, tr.name)
+        return (f"{name}: L={s.L}, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, T={s.T}, W={s.W}, {tr.n_steps} steps, saliency "
+                f"from last {s.Ls} layers, budget {bud}")
+    Ts = [t.T for t in trs]
+    return (f"{len(trs)} ragged llama3-8b-shaped trajectories in one call: L={s.L}, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, "
+            f"T in [{min(Ts)}, {max(Ts)}] (sum {sum(Ts)}), W={s.W}, 24-60 steps each, 4 key channels x8, budget {bud}")
+
+
+def workload_config(trs, cfg, n, budget_label=None):
     return {
-        "workload": (f"llama3-8b-shaped agent trajectory: L={s.L}, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, T={s.T}, "
-                     f"W={s.W}, {tr.n_steps} steps, saliency from last {s.Ls} layers, budget "
-                     + (f"{b.num}/{b.den} of prunable" if b.mode == "ratio" else f"{b.count} tokens")),
-        "global_batch": n, "seq_len": s.T, "parallelism": f"dp{n} (independent trajectories)",
-        "l2": "flushed between timed steps (512 MB write outside the step events); inputs 4 GB > L2",
+        "workload": describe(trs, budget_label), "bench_config": cfg,
+        "global_batch": n * len(trs), "seq_len": max(t.T for t in trs),
+        "parallelism": f"dp{n} (independent trajectories)",
+        "l2": "flushed between timed steps (512 MB write outside the step events)",
     }
 
 
 class DeviceTraj:
     """Device-resident inputs/outputs of one trajectory and the C-ABI problem descriptor."""
 
-    def __init__(self, tr, device, seed=1234):
+    def __init__(self, tr, device, seed=1234, budget=None, full_outputs=False):
         import numpy as np
         import torch
         from paper_2609_22158_gb300 import binding as B
@@ -83,43 +127,102 @@ class DeviceTraj:
         self.step_id, self.prot, self.pos = t(tr.step_id), t(tr.prot), t(tr.pos)
         self.steps = B.StepSignals(t(tr.valid), t(tr.gain), t(tr.red), t(tr.reuse), t(tr.obs_sim),
                                    torch.empty(tr.n_steps, dtype=torch.float32, device=device))
+        self.K_out = self.V_out = None
+        self.set_budget(budget or tr.budget, full_outputs)
+
+    def set_budget(self, budget, full_outputs=False):
+        """(Re)allocate the outputs for a budget (workload.Budget) and rebuild the problem descriptor."""
+        import torch
+        from paper_2609_22158_gb300 import binding as B
+        tr, s = self.tr, self.tr.shape
+        device = self.step_id.device
         n_prot = int(tr.prot.sum())
         N = s.T - n_prot
-        B_t = (max(1, tr.budget.num * N // tr.budget.den) if tr.budget.mode == "ratio" else tr.budget.count)
+        B_t = (max(1, budget.num * N // budget.den) if budget.mode == "ratio" else budget.count)
         self.n_kept_expected = n_prot + min(B_t, N)
         self.cap = self.n_kept_expected
+        self.K_out = self.V_out = None
         self.K_out = [torch.empty((s.Hkv, self.cap, s.d), dtype=torch.bfloat16, device=device) for _ in range(s.L)]
         self.V_out = [torch.empty((s.Hkv, self.cap, s.d), dtype=torch.bfloat16, device=device) for _ in range(s.L)]
-        self.out = B.SelectOutputs.allocate(s.T, tr.n_steps, self.cap, device, full=False)
+        self.out = B.SelectOutputs.allocate(s.T, tr.n_steps, self.cap, device, full=full_outputs)
         self.step_id_out = torch.empty(self.cap, dtype=torch.int32, device=device)
         self.pos_out = torch.empty(self.cap, dtype=torch.int32, device=device)
-        b = tr.budget
-        self.budget = B.budget_ratio(b.num, b.den) if b.mode == "ratio" else B.budget_count(b.count)
+        self.budget = B.budget_ratio(budget.num, budget.den) if budget.mode == "ratio" else B.budget_count(budget.count)
         self.problem = B.Problem(self.K, self.V, self.Q, s.T, self.step_id, self.prot, self.steps, self.budget,
                                  self.K_out, self.V_out, self.out, pos_in=self.pos, step_id_out=self.step_id_out,
                                  pos_out=self.pos_out)
-        self.ws = torch.empty(B.stepkv_workspace_size([self.problem]) + 512, dtype=torch.uint8, device=device)
-        self.status = B.new_status(device)
-
-    def compress(self, params, stream=None):
-        from paper_2609_22158_gb300 import binding as B
-        B.stepkv_compress([self.problem], params, ws=self.ws, status=self.status, stream=stream)
 
 
-def launches_per_pass(tr) -> int:
-    """Kernel launches of one stepkv_compress call (mirrors the library's launch plan)."""
-    s = tr.shape
-    return 1 + 1 + math.ceil(s.L / 96)  # score (both passes, one cooperative launch), select, compaction
+def launches_per_call(trs) -> int:
+    """Kernel launches of one stepkv_compress call over these trajectories (mirrors the library's plan:
+    saliency launches of up to 16 trajectories and 512 MB of keys, one selection launch per 16
+    trajectories, compaction launches of up to 16 trajectories and 1024 (layer, tensor) entries)."""
+    n = len(trs)
+    score, keys, cnt = 0, 0, 0
+    for tr in trs:
+        s = tr.shape
+        kb = s.Ls * s.Hkv * s.T * s.d * 2
+        if cnt == 0 or cnt == 16 or keys + kb > (512 << 20):
+            score += 1
+            keys, cnt = 0, 0
+        keys += kb
+        cnt += 1
+    select = math.ceil(n / 16)
+    ent = sum(2 * tr.shape.L for tr in trs)
+    compact = max(math.ceil(n / 16), math.ceil(ent / 1024))
+    return score + select + compact
 
 
 def algorithmic_bytes(tr, n_kept):
-    """Bytes the pass must move at minimum (stage by stage)."""
+    """Bytes the pass must move at minimum (stage by stage), and the saliency contraction's work."""
     s = tr.shape
-    G = s.Hq // s.Hkv
     score = s.Ls * s.Hkv * s.T * s.d * 2 + s.Ls * s.Hq * s.W * s.d * 2 + s.Ls * s.Hkv * s.T * 4
     select = s.Ls * s.Hkv * s.T * 4 + s.T * (4 + 1) + n_kept * 4
     compact = 2 * s.L * s.Hkv * n_kept * s.d * 2 * 2 + n_kept * 4 * 3
-    return {"score": score, "select": select, "compact": compact, "total": score + select + compact}
+    # pass 1 (row statistics) and pass 2 (per-key mass): each a Q.K^T over the visible keys
+    flops_pass = 2.0 * s.Ls * s.Hq * s.W * s.T * s.d
+    exps_pass = 1.0 * s.Ls * s.Hq * s.W * s.T
+    return {"score": score, "select": select, "compact": compact, "total": score + select + compact,
+            "score_flops_one_pass": flops_pass, "score_exps_one_pass": exps_pass}
+
+
+def kernel_rooflines(tr, stage_us, n_kept, peaks, cfg):
+    """Per-kernel achieved fractions from the stage times (CUDA events around each entry point)."""
+    ab = algorithmic_bytes(tr, n_kept)
+    tr_ncu = NCU_TRAFFIC.get(cfg, {})
+    hbm = peaks["hbm"]
+    mufu_peak = MUFU_PER_CLK_SM * 152 * peaks["sm_mhz"] * 1e6
+    out = {}
+    us = stage_us["score"]
+    gbs = ab["score"] / (us * 1e-6) / 1e9
+    tfs2 = 2 * ab["score_flops_one_pass"] / (us * 1e-6) / 1e12
+    exps2 = 2 * ab["score_exps_one_pass"] / (us * 1e-6)
+    out["score_kernel"] = {
+        "stage": "1-2: saliency, two tcgen05 passes (row statistics, per-key mass) + fixed-point T accumulation",
+        "bound": "hbm", "launch_us": round(us, 2), "algorithmic_bytes": ab["score"],
+        "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4),
+        "tensor": {"achieved_tflops_both_passes": round(tfs2, 1), "peak": peaks["bf16"],
+                   "frac": round(tfs2 / peaks["bf16"], 4), "one_pass_roof_us": round(
+                       ab["score_flops_one_pass"] / (peaks["bf16"] * 1e12) * 1e6, 2)},
+        "mufu": {"achieved_ex2_per_s_both_passes": round(exps2 / 1e12, 3) * 1e12,
+                 "peak": mufu_peak, "frac": round(exps2 / mufu_peak, 4),
+                 "peak_derivation": f"{MUFU_PER_CLK_SM} ex2/clk/SM x 152 SMs x {peaks['sm_mhz']:.0f} MHz"},
+        "traffic": tr_ncu.get("score_kernel")}
+    us = stage_us["select"]
+    gbs = ab["select"] / (us * 1e-6) / 1e9
+    out["select_kernel"] = {
+        "stage": "2-4: normalisation, per-step statistics, Eqs. 2-5, exact top-B (one 8-CTA cluster)",
+        "bound": "latency", "launch_us": round(us, 2), "algorithmic_bytes": ab["select"],
+        "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4),
+        "traffic": tr_ncu.get("select_kernel")}
+    us = stage_us["compact"]
+    gbs = ab["compact"] / (us * 1e-6) / 1e9
+    out["compact_kernel"] = {
+        "stage": "5: retained K/V row gather, all layers",
+        "bound": "hbm", "launch_us": round(us, 2), "algorithmic_bytes": ab["compact"],
+        "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4),
+        "traffic": tr_ncu.get("compact_kernel")}
+    return out
 
 
 # ---------------------------------------------------------------------------------- clocks
@@ -137,10 +240,6 @@ class ClockSampler:
                                           "-lms", "100", "-i", str(gpu_index)], stdout=self.f, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
-        self.marks = []
-
-    def mark(self, name):
-        self.marks.append((name, time.time()))
 
     def stop(self):
         if self.proc is None:
@@ -171,75 +270,126 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------------------------- oracle timing
-ORACLE_SNIPPET = r"""
-import json, sys, time
-sys.path.insert(0, {root!r})
-import numpy as np
-from oracle import stepkv_oracle as O
-from paper_2609_22158_gb300 import workload as wl
-tr = wl.llama8b_32k(seed={seed}, T={T}, L={L})
-s = tr.shape
-pairs = {pairs}
-Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
-Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
-V0 = tr.values(tr.sal_layer_ids()[0])
-G = s.Hq // s.Hkv
-t0 = time.perf_counter()
-A = []
-done = 0
-for li in range(len(Ks)):
-    rows = []
-    for h in range(s.Hkv):
-        if done < pairs:
-            rows.append(O.window_attention_saliency(Ks[li][h:h + 1], Qs[li][h * G:(h + 1) * G])[0])
-            done += 1
-        else:
-            rows.append(np.zeros(s.T))
-    A.append(np.stack(rows))
-t1 = time.perf_counter()
-b = tr.budget
-out = O.stepkv_boundary(A, tr.step_id, tr.prot, tr.valid, tr.gain, tr.red, tr.obs_sim, tr.reuse, O.Params(),
-                        b.mode, b.num, b.den, b.count)
-t2 = time.perf_counter()
-for rep in range({compact_sets}):
-    C = O.compact_rows(V0[rep % s.Hkv:rep % s.Hkv + 1], out["kept"])
-t3 = time.perf_counter()
-print(json.dumps({{"score_s": t1 - t0, "select_s": t2 - t1, "compact_s": t3 - t2, "n_kept": int(len(out["kept"]))}}))
-"""
+def oracle_worker(spec: dict) -> dict:
+    """Runs in a fresh CPU-only process (never one that touched the GPU).  Times the oracle, as it stands,
+    on the trajectories of a configuration: saliency of every (trajectory, layer, KV head) pair, the
+    boundary (Eqs. 1-5, Algorithm 1) of every trajectory, and the gather of every (layer, tensor, KV head)
+    row set.  With workers > 1 the independent pairs and row sets are spread over a fork pool of
+    single-threaded processes (the oracle itself is unchanged).  Row-set contents do not change a gather's
+    cost, so the row sets are drawn from one generated layer per trajectory."""
+    import multiprocessing as mp
+
+    import numpy as np
+
+    from oracle import stepkv_oracle as O
+    global _ORACLE_STATE
+    trs = make_trajs(spec["cfg"])
+    pick = spec.get("trajs")
+    if pick is not None:
+        trs = [trs[i] for i in pick]
+    data = []
+    for tr in trs:
+        Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+        Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+        data.append((tr, Ks, Qs, tr.values(tr.sal_layer_ids()[0])))
+    _ORACLE_STATE = data
+    workers = int(spec["workers"])
+    pairs = [(b, li, h) for b, (tr, Ks, _, _) in enumerate(data) for li in range(len(Ks)) for h in range(tr.shape.Hkv)]
+    pool = mp.get_context("fork").Pool(workers) if workers > 1 else None
+    times = []
+    try:
+        for _ in range(int(spec.get("reps", 1))):
+            t0 = time.perf_counter()
+            A = (pool.map(_oracle_pair, pairs, chunksize=1) if pool else [_oracle_pair(x) for x in pairs])
+            t1 = time.perf_counter()
+            outs = []
+            i = 0
+            for (tr, Ks, _, _) in data:
+                s = tr.shape
+                layers = []
+                for li in range(len(Ks)):
+                    layers.append(np.stack(A[i:i + s.Hkv]))
+                    i += s.Hkv
+                b = tr.budget
+                outs.append(O.stepkv_boundary(layers, tr.step_id, tr.prot, tr.valid, tr.gain, tr.red, tr.obs_sim,
+                                              tr.reuse, O.Params(), b.mode, b.num, b.den, b.count))
+            t2 = time.perf_counter()
+            sets = [(b, r, out["kept"]) for b, out in enumerate(outs) for r in range(2 * data[b][0].shape.L
+                                                                                     * data[b][0].shape.Hkv)]
+            if pool:
+                pool.map(_oracle_gather, [(b, r, k) for (b, r, k) in sets], chunksize=max(1, len(sets) // (4 * workers)))
+            else:
+                for x in sets:
+                    _oracle_gather(x)
+            t3 = time.perf_counter()
+            times.append({"score_s": t1 - t0, "select_s": t2 - t1, "compact_s": t3 - t2, "total_s": t3 - t0})
+    finally:
+        if pool:
+            pool.close()
+            pool.join()
+    return {"passes": times, "tokens": int(sum(tr.T for tr in trs)), "pairs": len(pairs),
+            "n_kept": [int(len(o["kept"])) for o in outs]}
 
 
-def oracle_pass_seconds(args, pairs: int, compact_sets: int, threads: int = 1):
-    """Run the oracle (as it stands) on a bounded sample in a fresh single-threaded process and scale
-    each stage to the whole pass.  Returns (seconds per full pass, description, threads)."""
-    from paper_2609_22158_gb300 import workload as wl
-    tr = make_traj(args)
-    s = tr.shape
-    code = ORACLE_SNIPPET.format(root=ROOT, seed=args.seed, T=args.T, L=args.layers, pairs=pairs,
-                                 compact_sets=compact_sets)
+_ORACLE_STATE = None
+
+
+def _oracle_pair(x):
+    from oracle import stepkv_oracle as O
+    b, li, h = x
+    tr, Ks, Qs, _ = _ORACLE_STATE[b]
+    G = tr.shape.Hq // tr.shape.Hkv
+    return O.window_attention_saliency(Ks[li][h:h + 1], Qs[li][h * G:(h + 1) * G])[0]
+
+
+def _oracle_gather(x):
+    from oracle import stepkv_oracle as O
+    b, r, kept = x
+    V0 = _ORACLE_STATE[b][3]
+    h = r % V0.shape[0]
+    return O.compact_rows(V0[h:h + 1], kept).shape
+
+
+def oracle_timing(cfg: int, workers: int, reps: int = 1, trajs=None) -> dict:
+    """Run oracle_worker in a fresh process with single-threaded numpy (``workers`` processes)."""
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS"):
-        env[k] = str(threads)
+        env[k] = "1"
     env["CUDA_VISIBLE_DEVICES"] = ""
-    r = subprocess.run([sys.executable, "-c", code], stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True,
-                       env=env, timeout=1800)
+    spec = {"cfg": cfg, "workers": workers, "reps": reps, "trajs": trajs}
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker", json.dumps(spec)],
+                       stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True, env=env, timeout=3600)
     if r.returncode != 0:
-        raise RuntimeError("oracle run failed: " + r.stderr[-2000:])
-    m = json.loads(r.stdout.strip().splitlines()[-1])
-    n_pairs = s.Ls * s.Hkv
-    n_sets = 2 * s.L * s.Hkv
-    total = m["score_s"] * n_pairs / pairs + m["select_s"] + m["compact_s"] * n_sets / compact_sets
-    desc = (f"oracle (numpy fp64, {threads} thread) on the same workload: saliency of {pairs} of {n_pairs} "
-            f"(layer, KV head) pairs, full selection, compaction of {compact_sets} of {n_sets} (layer, tensor, head) "
-            f"row sets; each stage's time scaled to the whole pass")
-    return total, desc, m
+        raise RuntimeError("oracle run failed: " + r.stderr[-3000:])
+    return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-# ---------------------------------------------------------------------------------- ours
-def run_ours(args):
-    import numpy as np
+def cpu_baseline(cfg: int, trs) -> dict:
+    """The oracle on the host cores: all cores (headline) and one thread, each on a bounded sample."""
+    cores = os.cpu_count() or 1
+    pick = None
+    if len(trs) > 4:  # the 16-trajectory batch: time 4 trajectories, scale by tokens
+        pick = [0, 5, 10, 15]
+    res_all = oracle_timing(cfg, cores, reps=1, trajs=pick)
+    res_one = oracle_timing(cfg, 1, reps=1, trajs=pick[:1] if pick else None)
+    def tps(res):
+        return res["tokens"] / res["passes"][-1]["total_s"]
+    what = (f"{len(pick)} of {len(trs)} trajectories (every stage of each), throughput in their tokens"
+            if pick else "the whole pass: saliency of every (layer, KV head) pair, the boundary, every row set's gather")
+    return {"value": tps(res_all), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"oracle (numpy fp64) on {what}; {cores} single-threaded processes over the independent "
+                      f"(trajectory, layer, KV head) pairs and row sets; row sets gathered from one generated layer",
+            "seconds_per_pass": round(res_all["passes"][-1]["total_s"], 3),
+            "stages_s": {k: round(v, 3) for k, v in res_all["passes"][-1].items()},
+            "single_thread": {"value": tps(res_one), "cores": 1,
+                              "seconds_per_pass": round(res_one["passes"][-1]["total_s"], 3),
+                              "sample": "first trajectory only" if pick else "the whole pass"}}
+
+
+# ---------------------------------------------------------------------------------- GPU helpers
+def _setup_gpu():
     import torch
-    from paper_2609_22158_gb300 import binding as B
-
+    from paper_2609_22158_gb300 import binding as B, build
     from paper_2609_22158_gb300 import multirank as MR
     world, rank, local = MR.rank_env()
     dist = None
@@ -249,42 +399,28 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     dev = torch.device("cuda", local if world > 1 else 0)
     torch.cuda.set_device(dev)
-    from paper_2609_22158_gb300 import build
     build.build_library()
     B.load_library()
+    return world, rank, local, dist, dev
 
-    tr = make_traj(args)
-    s = tr.shape
-    dt = DeviceTraj(tr, dev, seed=MR.rank_seed(1234, rank))
-    params = B.Params()
-    stream = torch.cuda.current_stream(dev)
-    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
-    hbm, _, peak_kind = _peaks()
 
-    sampler = ClockSampler(dev.index if world == 1 else local) if rank == 0 else None
-
-    # warm-up
-    for _ in range(args.warmup):
-        dt.compress(params, stream)
+def _time_calls(call, steps, warmup, stream, flush, dist, dev):
+    """W untimed calls, then exactly K calls each bracketed by CUDA events on the launching stream, an L2
+    flush between them (outside the events).  Returns (mean ms per call over ranks' max, per-call ms, wall)."""
+    import torch
+    from paper_2609_22158_gb300 import multirank as MR
+    for _ in range(warmup):
+        call()
         flush.fill_(1)
     torch.cuda.synchronize()
-    st = int(dt.status.item())
-    if st != 0:
-        raise RuntimeError(f"device status {st} after warm-up")
-    n_kept = int(dt.out.n_kept.item())
-    assert n_kept == dt.n_kept_expected, (n_kept, dt.n_kept_expected)
-
-    # timed region: exactly K fused passes, each bracketed by CUDA events on the launching stream
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    if sampler:
-        sampler.mark("timed_start")
     wall0 = time.perf_counter()
-    for i in range(args.steps):
+    for i in range(steps):
         ev[i][0].record(stream)
-        dt.compress(params, stream)
+        call()
         ev[i][1].record(stream)
         flush.fill_(i & 0xFF)
     torch.cuda.synchronize()
@@ -293,139 +429,178 @@ def run_ours(args):
         dist.barrier()
     step_ms = [a.elapsed_time(b) for a, b in ev]
     ms = MR.max_over_ranks(sum(step_ms) / len(step_ms), dist, dev)
-    if int(dt.status.item()) != 0:
-        raise RuntimeError(f"device status {int(dt.status.item())} in the timed region")
-    tokens = MR.gather_tokens(s.T, dist, dev)
-    value = MR.job_throughput(tokens, ms * 1e-3)
+    return ms, step_ms, wall1 - wall0
 
-    # per-stage timing (same shapes, separate entry points, same stream) for the roofline
-    stage = {}
-    if rank == 0 and not args.no_stages:
-        sal = torch.empty((s.Ls, s.Hkv, s.T), dtype=torch.float32, device=dev)
-        ws_s = torch.empty(B.load_library().stepkv_score_workspace_size(s.Ls, s.Hkv, s.Hq, s.T, s.W) + 512,
-                           dtype=torch.uint8, device=dev)
-        ws_sel = torch.empty(B.load_library().stepkv_select_workspace_size(s.Ls * s.Hkv, s.T, tr.n_steps) + 512,
-                             dtype=torch.uint8, device=dev)
-        sel_out = B.SelectOutputs.allocate(s.T, tr.n_steps, dt.cap, dev, full=False)
-        Ksal = [dt.K[l] for l in tr.sal_layer_ids()]
-        reps = max(3, min(args.steps, 20))
-        times = {"score": [], "select": [], "compact": []}
-        for r in range(reps + 2):
-            e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-            flush.fill_(r & 0xFF)
-            torch.cuda._sleep(200_000)
-            e[0].record(stream)
-            B.stepkv_score(Ksal, dt.Q, s.T, sal=sal, ws=ws_s, status=dt.status, stream=stream)
-            e[1].record(stream)
-            B.stepkv_select(sal, dt.step_id, dt.prot, dt.steps, params, dt.budget, sel_out, ws=ws_sel,
-                            status=dt.status, stream=stream)
-            e[2].record(stream)
-            flush.fill_((r + 1) & 0xFF)
-            # keep the device busy while the host marshals the 64 per-layer tensors of the call, so the
-            # events time the kernel and not the host
-            torch.cuda._sleep(400_000)
-            e3 = torch.cuda.Event(enable_timing=True)
-            e3.record(stream)
-            B.stepkv_compact(dt.K, dt.V, s.T, sel_out.kept_idx, sel_out.n_kept, dt.cap, dt.K_out, dt.V_out,
-                             dt.step_id, dt.pos, dt.step_id_out, dt.pos_out, status=dt.status, stream=stream)
-            e[3].record(stream)
-            torch.cuda.synchronize()
-            if r >= 2:
-                times["score"].append(e[0].elapsed_time(e[1]))
-                times["select"].append(e[1].elapsed_time(e[2]))
-                times["compact"].append(e3.elapsed_time(e[3]))
-        stage = {k: statistics.median(v) * 1e3 for k, v in times.items()}  # us
 
-    # e2e: host buffers through the same public call.  The cache lives in page-locked host memory and the
-    # compacted cache is written back to host memory: every step copies the window queries, the token
-    # metadata and the saliency layers' K host->device, the compaction reads the retained rows of all
-    # layers across the CPU-GPU link and writes them to the host outputs, and the retained slots come back
-    # device->host.  The second figure copies every input to the device and every output back instead.
-    e2e = None
-    e2e_copy_all = None
-    if not args.no_e2e:
-        s_ = tr.shape
-        host_K = [t.cpu().pin_memory() for t in dt.K]
-        host_V = [t.cpu().pin_memory() for t in dt.V]
-        host_Q = [t.cpu().pin_memory() for t in dt.Q]
-        host_small = [x.cpu().pin_memory() for x in (dt.step_id, dt.prot, dt.pos)]
-        dev_small = [dt.step_id, dt.prot, dt.pos]
-        sal_ids = list(tr.sal_layer_ids())
-        K_sal = [torch.empty_like(dt.K[l]) for l in sal_ids]
-        host_Kout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.K_out]
-        host_Vout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.V_out]
-        host_idx = torch.empty(dt.cap + 1, dtype=torch.int32).pin_memory()
-        sig_dev = [dt.steps.valid, dt.steps.gain, dt.steps.red, dt.steps.reuse_in, dt.steps.obs_sim]
-        host_sig = [x.cpu().pin_memory() for x in sig_dev]
-        nb = lambda ts: sum(t.numel() * t.element_size() for t in ts)
-        row_bytes = 2 * s_.L * s_.Hkv * s_.d * 2  # K and V of one retained slot, all layers
-        k2 = max(1, min(args.steps, args.e2e_steps))
-        # Two sets of device input buffers, so that the next step's host->device copies (on their own
-        # stream) run while the current step gathers its rows across the link in the other direction.
-        copy_stream = torch.cuda.Stream(device=dev)
-        bufs = []
-        for _ in range(2):
-            Qb = [torch.empty_like(q) for q in dt.Q]
-            smallb = [torch.empty_like(x) for x in dev_small]
-            sigb = [torch.empty_like(x) for x in sig_dev]
-            Ksb = [torch.empty_like(dt.K[l]) for l in sal_ids]
-            stepsb = B.StepSignals(sigb[0], sigb[1], sigb[2], sigb[3], sigb[4], dt.steps.reuse_out)
-            probb = B.Problem(host_K, host_V, Qb, s_.T, smallb[0], smallb[1], stepsb, dt.budget, host_Kout,
-                              host_Vout, dt.out, pos_in=smallb[2], step_id_out=dt.step_id_out, pos_out=dt.pos_out,
-                              kv_location=B.STEPKV_MEM_HOST, out_location=B.STEPKV_MEM_HOST, K_sal=Ksb)
-            bufs.append((Qb + smallb + sigb + Ksb, probb, torch.cuda.Event(), torch.cuda.Event()))
-        step_inputs = host_Q + host_small + host_sig + [host_K[l] for l in sal_ids]
-        n_step = [0]
+def stage_times(dt, params, stream, flush, reps):
+    """Per-stage CUDA-event times through the separate entry points on the same shapes (L2 flushed)."""
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+    tr, s = dt.tr, dt.tr.shape
+    dev = dt.step_id.device
+    sal = torch.empty((s.Ls, s.Hkv, s.T), dtype=torch.float32, device=dev)
+    lib = B.load_library()
+    ws_s = torch.empty(lib.stepkv_score_workspace_size(s.Ls, s.Hkv, s.Hq, s.T, s.W) + 512, dtype=torch.uint8,
+                       device=dev)
+    ws_sel = torch.empty(lib.stepkv_select_workspace_size(s.Ls * s.Hkv, s.T, tr.n_steps) + 512, dtype=torch.uint8,
+                         device=dev)
+    sel_out = B.SelectOutputs.allocate(s.T, tr.n_steps, dt.cap, dev, full=False)
+    Ksal = [dt.K[l] for l in tr.sal_layer_ids()]
+    times = {"score": [], "select": [], "compact": []}
+    for r in range(reps + 2):
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        flush.fill_(r & 0xFF)
+        torch.cuda._sleep(200_000)
+        e[0].record(stream)
+        B.stepkv_score(Ksal, dt.Q, s.T, sal=sal, ws=ws_s, status=dt.status, stream=stream)
+        e[1].record(stream)
+        B.stepkv_select(sal, dt.step_id, dt.prot, dt.steps, params, dt.budget, sel_out, ws=ws_sel,
+                        status=dt.status, stream=stream)
+        e[2].record(stream)
+        flush.fill_((r + 1) & 0xFF)
+        # keep the device busy while the host marshals the per-layer tensors of the call, so the events
+        # time the kernel and not the host
+        torch.cuda._sleep(400_000)
+        e3 = torch.cuda.Event(enable_timing=True)
+        e3.record(stream)
+        B.stepkv_compact(dt.K, dt.V, s.T, sel_out.kept_idx, sel_out.n_kept, dt.cap, dt.K_out, dt.V_out,
+                         dt.step_id, dt.pos, dt.step_id_out, dt.pos_out, status=dt.status, stream=stream)
+        e[3].record(stream)
+        torch.cuda.synchronize()
+        if r >= 2:
+            times["score"].append(e[0].elapsed_time(e[1]))
+            times["select"].append(e[1].elapsed_time(e[2]))
+            times["compact"].append(e3.elapsed_time(e[3]))
+    return {k: statistics.median(v) * 1e3 for k, v in times.items()}  # us
 
-        def e2e_step():
-            dsts, probb, copied, done = bufs[n_step[0] % 2]
-            n_step[0] += 1
-            with torch.cuda.stream(copy_stream):
-                copy_stream.wait_event(done)  # the step that last used these buffers has finished with them
-                for h, d in zip(step_inputs, dsts):
-                    d.copy_(h, non_blocking=True)
-                copied.record(copy_stream)
-            stream.wait_event(copied)
-            B.stepkv_compress([probb], params, ws=dt.ws, status=dt.status, stream=stream)
-            done.record(stream)
-            with torch.cuda.stream(stream):
-                host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
-                host_idx[dt.cap:].copy_(dt.out.n_kept, non_blocking=True)
 
-        def timed(step):
-            # one untimed step first: the first transfer from freshly pinned pages runs at about a third
-            # of the steady copy bandwidth
+def selection_report(dt, params, stream):
+    """Extra (untimed) passes with every selection output: the per-step retained histogram (the view of the
+    paper's Fig. 8) and, where the workload plants needle spans, how many needle tokens are retained at the
+    configured weights and with the saliency term alone (alpha = 1, beta = 0: the Table 3 ablation)."""
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+    tr = dt.tr
+
+    def one(p):
+        full = B.SelectOutputs.allocate(tr.T, tr.n_steps, dt.cap, dt.step_id.device, full=True)
+        prob = B.Problem(dt.K, dt.V, dt.Q, tr.T, dt.step_id, dt.prot, dt.steps, dt.budget, dt.K_out, dt.V_out, full,
+                         pos_in=dt.pos, step_id_out=dt.step_id_out, pos_out=dt.pos_out)
+        B.stepkv_compress([prob], p, ws=dt.ws, status=dt.status, stream=stream)
+        torch.cuda.synchronize()
+        n = int(full.n_kept.item())
+        return full, set(full.kept_idx[:n].cpu().numpy().tolist()), n
+
+    full, ks, n = one(params)
+    rep = {"step_count": full.step_count.cpu().numpy().tolist(), "step_kept": full.step_kept.cpu().numpy().tolist(),
+           "N_B": full.n_budget.cpu().numpy().tolist()}
+    if tr.needles:
+        toks = [j for (st, ln) in tr.needles for j in range(st, st + ln)]
+        hit = sum(1 for j in toks if j in ks)
+        sal_only = B.Params()
+        sal_only.alpha, sal_only.beta = 1.0, 0.0
+        _, ks1, _ = one(sal_only)
+        hit1 = sum(1 for j in toks if j in ks1)
+        rep["needle_recall"] = {"retained": hit, "planted": len(toks), "recall": round(hit / len(toks), 4),
+                                "recall_saliency_only": round(hit1 / len(toks), 4),
+                                "spans": [list(x) for x in tr.needles],
+                                "budget_fraction": round((n - int(tr.prot.sum())) / (tr.T - int(tr.prot.sum())), 4)}
+    return rep
+
+
+def e2e_single(dt, params, stream, dist, dev, tokens, steps, with_copy_all=True):
+    """End to end through stepkv_compress with HOST buffers: the cache lives in page-locked host memory and
+    the compacted cache is written back to host memory.  Every step copies the window queries, the token
+    metadata and the saliency layers' K host->device, the compaction reads the retained rows of all layers
+    across the CPU-GPU link and writes them to the host outputs, and the retained slots come back
+    device->host.  The second figure copies every input to the device and every output back instead."""
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+    from paper_2609_22158_gb300 import multirank as MR
+    tr, s_ = dt.tr, dt.tr.shape
+    host_K = [t.cpu().pin_memory() for t in dt.K]
+    host_V = [t.cpu().pin_memory() for t in dt.V]
+    host_Q = [t.cpu().pin_memory() for t in dt.Q]
+    host_small = [x.cpu().pin_memory() for x in (dt.step_id, dt.prot, dt.pos)]
+    dev_small = [dt.step_id, dt.prot, dt.pos]
+    sal_ids = list(tr.sal_layer_ids())
+    host_Kout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.K_out]
+    host_Vout = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in dt.V_out]
+    host_idx = torch.empty(dt.cap + 1, dtype=torch.int32).pin_memory()
+    sig_dev = [dt.steps.valid, dt.steps.gain, dt.steps.red, dt.steps.reuse_in, dt.steps.obs_sim]
+    host_sig = [x.cpu().pin_memory() for x in sig_dev]
+    nb = lambda ts: sum(t.numel() * t.element_size() for t in ts)
+    row_bytes = 2 * s_.L * s_.Hkv * s_.d * 2  # K and V of one retained slot, all layers
+    k2 = max(1, steps)
+    # Two sets of device input buffers, so that the next step's host->device copies (on their own stream)
+    # run while the current step gathers its rows across the link in the other direction.
+    copy_stream = torch.cuda.Stream(device=dev)
+    bufs = []
+    for _ in range(2):
+        Qb = [torch.empty_like(q) for q in dt.Q]
+        smallb = [torch.empty_like(x) for x in dev_small]
+        sigb = [torch.empty_like(x) for x in sig_dev]
+        Ksb = [torch.empty_like(dt.K[l]) for l in sal_ids]
+        stepsb = B.StepSignals(sigb[0], sigb[1], sigb[2], sigb[3], sigb[4], dt.steps.reuse_out)
+        probb = B.Problem(host_K, host_V, Qb, s_.T, smallb[0], smallb[1], stepsb, dt.budget, host_Kout,
+                          host_Vout, dt.out, pos_in=smallb[2], step_id_out=dt.step_id_out, pos_out=dt.pos_out,
+                          kv_location=B.STEPKV_MEM_HOST, out_location=B.STEPKV_MEM_HOST, K_sal=Ksb)
+        bufs.append((Qb + smallb + sigb + Ksb, probb, torch.cuda.Event(), torch.cuda.Event()))
+    step_inputs = host_Q + host_small + host_sig + [host_K[l] for l in sal_ids]
+    n_step = [0]
+
+    def e2e_step():
+        dsts, probb, copied, done = bufs[n_step[0] % 2]
+        n_step[0] += 1
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(done)  # the step that last used these buffers has finished with them
+            for h, d in zip(step_inputs, dsts):
+                d.copy_(h, non_blocking=True)
+            copied.record(copy_stream)
+        stream.wait_event(copied)
+        B.stepkv_compress([probb], params, ws=dt.ws, status=dt.status, stream=stream)
+        done.record(stream)
+        with torch.cuda.stream(stream):
+            host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
+            host_idx[dt.cap:].copy_(dt.out.n_kept, non_blocking=True)
+
+    def timed(step):
+        # one untimed step first: the first transfer from freshly pinned pages runs at about a third of the
+        # steady copy bandwidth
+        step()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        copy_stream.wait_event(e0)
+        for i in range(k2):
             step()
-            torch.cuda.synchronize()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            copy_stream.wait_event(e0)
-            for i in range(k2):
-                step()
-            e1.record(stream)
-            torch.cuda.synchronize()
-            return MR.max_over_ranks(e0.elapsed_time(e1) / k2, dist, dev)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return MR.max_over_ranks(e0.elapsed_time(e1) / k2, dist, dev)
 
-        e2e_ms = timed(e2e_step)
-        n_k = int(host_idx[dt.cap].item())
-        assert n_k == dt.n_kept_expected
-        kept_h = host_idx[:n_k].long()
-        for l in (0, s_.L - 1):  # the host outputs hold the retained rows
-            assert torch.equal(host_Kout[l][:, :n_k], host_K[l].index_select(1, kept_h))
-            assert torch.equal(host_Vout[l][:, :n_k], host_V[l].index_select(1, kept_h))
-        h2d = nb(step_inputs) + n_k * row_bytes
-        d2h = n_k * row_bytes + host_idx.numel() * 4
-        e2e = {"value": MR.job_throughput(tokens, e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": k2,
-               "path": "cache in pinned host memory: window queries, token metadata, step signals and the "
-                       "saliency layers' K copied to the device (two buffer sets: the next step's copies overlap "
-                       "the current step's gather), retained rows gathered across the CPU-GPU link into pinned "
-                       "host outputs"}
-
+    e2e_ms = timed(e2e_step)
+    n_k = int(host_idx[dt.cap].item())
+    assert n_k == dt.n_kept_expected
+    kept_h = host_idx[:n_k].long()
+    for l in (0, s_.L - 1):  # the host outputs hold the retained rows
+        assert torch.equal(host_Kout[l][:, :n_k], host_K[l].index_select(1, kept_h))
+        assert torch.equal(host_Vout[l][:, :n_k], host_V[l].index_select(1, kept_h))
+    h2d = nb(step_inputs) + n_k * row_bytes
+    d2h = n_k * row_bytes + host_idx.numel() * 4
+    e2e = {"value": MR.job_throughput(tokens, e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+           "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms, "steps": k2,
+           "link": {"h2d_gbs_measured_probe": 211, "d2h_gbs_measured_probe": 193,
+                    "h2d_bound_ms": round(h2d / 211e9 * 1e3, 3),
+                    "frac_of_h2d_link": round((h2d / 211e9 * 1e3) / e2e_ms, 4)},
+           "path": "cache in pinned host memory: window queries, token metadata, step signals and the saliency "
+                   "layers' K copied to the device (two buffer sets: the next step's copies overlap the current "
+                   "step's gather), retained rows gathered across the CPU-GPU link into pinned host outputs"}
+    e2e_copy_all = None
+    if with_copy_all:
         def copy_all_step():
             for h, d in zip(host_K + host_V + host_Q + host_small, dt.K + dt.V + dt.Q + dev_small):
                 d.copy_(h, non_blocking=True)
-            dt.compress(params, stream)
+            B.stepkv_compress([dt.problem], params, ws=dt.ws, status=dt.status, stream=stream)
             for h, d in zip(host_Kout + host_Vout, dt.K_out + dt.V_out):
                 h.copy_(d, non_blocking=True)
             host_idx[:dt.cap].copy_(dt.out.kept_idx, non_blocking=True)
@@ -438,47 +613,132 @@ def run_ours(args):
                         "d2h_bytes_per_step": int(nb(host_Kout + host_Vout) + host_idx.numel() * 4),
                         "ms_per_step": ca_ms, "steps": k2,
                         "path": "every input copied to the device, the device pass, every output copied back"}
+    return e2e, e2e_copy_all
 
-    # decode attention over a compacted cache (timed separately, not part of the metric): the incremental
-    # loop's shape, Llama-3-8B heads, 8192-token budget + 16 prompt + 64 window rows = 8272 rows per head
-    decode = None
-    if rank == 0 and not args.no_decode:
-        dec_rows = 8192 + 16 + 64
-        dgen = torch.Generator(device=dev).manual_seed(99)
-        Kd = [torch.randn((s.Hkv, dec_rows, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
-        Vd = [torch.randn((s.Hkv, dec_rows, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
-        qd = [torch.randn((s.Hq, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
-        outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
-        ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, dec_rows) + 512,
-                           dtype=torch.uint8, device=dev)
-        n_tok = 64
-        for _ in range(3):
-            B.stepkv_decode(qd, Kd, Vd, dec_rows, out=outd, ws=ws_d, status=dt.status, stream=stream)
-        flush.fill_(7)
-        torch.cuda.synchronize()
-        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        d0.record(stream)
-        for _ in range(n_tok):  # the cache (1.08 GB) exceeds L2, so every token reads it from HBM
-            B.stepkv_decode(qd, Kd, Vd, dec_rows, out=outd, ws=ws_d, status=dt.status, stream=stream)
-        d1.record(stream)
-        torch.cuda.synchronize()
-        us = d0.elapsed_time(d1) * 1e3 / n_tok
-        dbytes = 2 * s.L * s.Hkv * dec_rows * s.d * 2
-        decode = {"workload": f"decode attention, {n_tok} single-token reads over a compacted cache of {dec_rows} "
-                              f"rows x {s.L} layers x {s.Hkv} KV heads (Hq={s.Hq}, d={s.d})",
-                  "us_per_token": round(us, 2), "algorithmic_bytes_per_token": dbytes,
-                  "achieved_gbs": round(dbytes / (us * 1e-6) / 1e9, 1),
-                  "frac_of_measured_hbm": round(dbytes / (us * 1e-6) / 1e9 / hbm, 4), "launches_per_token": 2}
-        if int(dt.status.item()) != 0:
-            raise RuntimeError(f"device status {int(dt.status.item())} after decode")
-        del Kd, Vd
 
-    # the incremental agent loop (timed separately, not part of the metric): Llama-3-8B heads, a 4096-token
-    # start, one new step per boundary, the compacted cache plus the new step compressed under a fixed
-    # 8192-token budget, then 64 single-token decode reads over the compacted cache
-    incremental = None
-    if rank == 0 and not args.no_incremental:
-        incremental = run_incremental(args, s, dev, stream, hbm)
+def decode_report(s, dev, stream, flush, status, hbm):
+    """Decode attention over a compacted cache (timed separately, not part of the metric): the incremental
+    loop's shape, 8192-token budget + 16 prompt + 64 window rows = 8272 rows per head."""
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+    dec_rows = 8192 + 16 + 64
+    dgen = torch.Generator(device=dev).manual_seed(99)
+    Kd = [torch.randn((s.Hkv, dec_rows, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
+    Vd = [torch.randn((s.Hkv, dec_rows, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
+    qd = [torch.randn((s.Hq, s.d), generator=dgen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
+    outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
+    ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, dec_rows) + 512,
+                       dtype=torch.uint8, device=dev)
+    n_tok = 64
+    for _ in range(3):
+        B.stepkv_decode(qd, Kd, Vd, dec_rows, out=outd, ws=ws_d, status=status, stream=stream)
+    flush.fill_(7)
+    torch.cuda.synchronize()
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record(stream)
+    for _ in range(n_tok):  # the cache (1.08 GB) exceeds L2, so every token reads it from HBM
+        B.stepkv_decode(qd, Kd, Vd, dec_rows, out=outd, ws=ws_d, status=status, stream=stream)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    us = d0.elapsed_time(d1) * 1e3 / n_tok
+    dbytes = 2 * s.L * s.Hkv * dec_rows * s.d * 2
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} after decode")
+    return {"workload": f"decode attention, {n_tok} single-token reads over a compacted cache of {dec_rows} "
+                        f"rows x {s.L} layers x {s.Hkv} KV heads (Hq={s.Hq}, d={s.d})",
+            "us_per_token": round(us, 2), "algorithmic_bytes_per_token": dbytes,
+            "achieved_gbs": round(dbytes / (us * 1e-6) / 1e9, 1),
+            "frac_of_measured_hbm": round(dbytes / (us * 1e-6) / 1e9 / hbm, 4), "launches_per_token": 2}
+
+
+# ---------------------------------------------------------------------------------- ours
+def base_line(args, value, ms, world, cfg_obj, roof, cpu, e2e, launches, clocks, wall, step_ms):
+    return {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded generator + torch device RNG; no datasets or model weights)",
+        "config": cfg_obj, "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+        "clocks": clocks, "wall_s_timed_region": round(wall, 4),
+        "step_ms_min_max": [round(min(step_ms), 4), round(max(step_ms), 4)] if step_ms else None,
+    }
+
+
+def run_ours(args):
+    import torch
+    from paper_2609_22158_gb300 import binding as B
+    from paper_2609_22158_gb300 import multirank as MR
+    world, rank, local, dist, dev = _setup_gpu()
+    peaks = _peaks()
+    hbm = peaks["hbm"]
+    if args.config == 5:
+        return run_config5(args, world, rank, local, dist, dev, peaks)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
+    params = B.Params()
+    trs = make_trajs(args.config, None if world == 1 else MR.rank_seed(args.config, rank))
+    status = B.new_status(dev)
+    dts = []
+    for i, tr in enumerate(trs):
+        dt = DeviceTraj(tr, dev, seed=MR.rank_seed(1234 + i, rank))
+        dts.append(dt)
+    ws = torch.empty(B.stepkv_workspace_size([d.problem for d in dts]) + 512, dtype=torch.uint8, device=dev)
+    for d in dts:
+        d.ws, d.status = ws, status
+    sampler = ClockSampler(dev.index if world == 1 else local) if rank == 0 else None
+    tokens_local = sum(tr.T for tr in trs)
+
+    sweep = None
+    if args.config == 3:
+        from paper_2609_22158_gb300 import workload as wl
+        sweep = {}
+        for label, bud in (("5%", wl.Budget.ratio(1, 20)), ("20%", wl.Budget.ratio(1, 5)), ("10%", wl.Budget.ratio(1, 10))):
+            for d in dts:
+                d.set_budget(bud)
+            probs = [d.problem for d in dts]
+            need = B.stepkv_workspace_size(probs) + 512
+            if need > ws.numel():
+                ws = torch.empty(need, dtype=torch.uint8, device=dev)
+            call = lambda: B.stepkv_compress(probs, params, ws=ws, status=status, stream=stream)
+            ms_b, step_ms, wall = _time_calls(call, args.steps, args.warmup, stream, flush, dist, dev)
+            n_kept = [int(d.out.n_kept.item()) for d in dts]
+            assert n_kept == [d.n_kept_expected for d in dts], (n_kept, [d.n_kept_expected for d in dts])
+            byts = sum(algorithmic_bytes(d.tr, n)["total"] for d, n in zip(dts, n_kept))
+            gbs = byts / (ms_b * 1e-3) / 1e9
+            sweep[label] = {"ms_per_step": ms_b, "tokens_per_s": MR.job_throughput(MR.gather_tokens(tokens_local, dist, dev),
+                                                                                  ms_b * 1e-3),
+                            "algorithmic_bytes": byts, "achieved_gbs": round(gbs, 1),
+                            "frac_of_measured_hbm": round(gbs / hbm, 4)}
+        ms = sweep["10%"]["ms_per_step"]
+        probs = [d.problem for d in dts]
+    else:
+        dt = dts[0]
+        call = lambda: B.stepkv_compress([dt.problem], params, ws=ws, status=status, stream=stream)
+        ms, step_ms, wall = _time_calls(call, args.steps, args.warmup, stream, flush, dist, dev)
+    if int(status.item()) != 0:
+        raise RuntimeError(f"device status {int(status.item())} in the timed region")
+    n_kept = [int(d.out.n_kept.item()) for d in dts]
+    assert n_kept == [d.n_kept_expected for d in dts], (n_kept, [d.n_kept_expected for d in dts])
+    tokens = MR.gather_tokens(tokens_local, dist, dev)
+    value = MR.job_throughput(tokens, ms * 1e-3)
+
+    kernels = roof = sel = None
+    stage = None
+    if rank == 0 and len(dts) == 1 and not args.no_stages:
+        stage = stage_times(dts[0], params, stream, flush, max(3, min(args.steps, 20)))
+        kernels = kernel_rooflines(dts[0].tr, stage, n_kept[0], peaks, args.config)
+        roof = dict(kernels["compact_kernel"])
+        roof["kernel"] = "compact_kernel (dominant: ~half the pass)"
+        roof["peak_source"] = f"{peaks['kind']} hbm_gbs (burst copy)"
+        sel = selection_report(dts[0], params, stream)
+    e2e = e2e_copy_all = None
+    if not args.no_e2e and len(dts) == 1:
+        e2e, e2e_copy_all = e2e_single(dts[0], params, stream, dist, dev, tokens, args.e2e_steps,
+                                       with_copy_all=args.config != 4)
+    decode = incremental = None
+    if rank == 0 and args.config == 2 and not args.no_decode:
+        decode = decode_report(dts[0].tr.shape, dev, stream, flush, status, hbm)
+    if rank == 0 and args.config == 2 and not args.no_incremental:
+        incremental = run_incremental(args.inc_boundaries, dts[0].tr.shape, dev, stream, peaks, growth_total=None)
 
     clocks = sampler.stop() if sampler else None
     if dist:
@@ -488,53 +748,43 @@ def run_ours(args):
             dist.destroy_process_group()
         return
 
-    ab = algorithmic_bytes(tr, n_kept)
-    roof = None
-    if stage:
-        comp_gbs = ab["compact"] / (stage["compact"] * 1e-6) / 1e9
-        roof = {"kernel": "compact_kernel (stage 5: retained K/V row gather, all 32 layers)", "bound": "hbm",
-                "achieved": round(comp_gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
-                "peak_source": f"{peak_kind} hbm_gbs (burst copy)", "traffic": args.compact_traffic,
-                "algorithmic_bytes_per_launch": ab["compact"], "launch_us": round(stage["compact"], 2)}
-    pass_gbs = ab["total"] / (ms * 1e-3) / 1e9
+    total_bytes = sum(algorithmic_bytes(d.tr, n)["total"] for d, n in zip(dts, n_kept))
+    pass_gbs = total_bytes / (ms * 1e-3) / 1e9
     cpu = None
-    if not args.no_cpu_baseline:
-        secs, desc, _ = oracle_pass_seconds(args, pairs=args.oracle_pairs, compact_sets=args.oracle_compact_sets)
-        cpu = {"value": s.T / secs, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
-               "seconds_per_pass": round(secs, 3)}
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": ms, "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded generator + torch device RNG; no datasets or model weights)",
-        "config": workload_config(tr, args, world),
-        "roofline": roof,
-        "pass_hbm": {"algorithmic_bytes": ab["total"], "achieved_gbs": round(pass_gbs, 1),
+    if not args.no_cpu_baseline and world == 1:
+        cpu = cpu_baseline(args.config, trs)
+    launches = launches_per_call(trs) * args.steps
+    line = base_line(args, value, ms, world, workload_config(trs, args.config, world, "10% of prunable (sweep: 5/10/20%)"
+                                                            if sweep else None),
+                     roof, cpu, e2e, launches, clocks, wall, step_ms)
+    line.update({
+        "kernels": kernels,
+        "pass_hbm": {"algorithmic_bytes": total_bytes, "achieved_gbs": round(pass_gbs, 1),
                      "frac_of_measured": round(pass_gbs / hbm, 4), "frac_of_nominal_8tbs": round(pass_gbs / 8000, 4)},
         "stages_us": {k: round(v, 2) for k, v in stage.items()} if stage else None,
-        "cpu_baseline": cpu, "e2e": e2e, "e2e_copy_all": e2e_copy_all, "decode": decode, "incremental": incremental,
-        "gpu_launches": launches_per_pass(tr) * args.steps,
-        "clocks": clocks,
-        "wall_s_timed_region": round(wall1 - wall0, 4),
-        "step_ms_min_max": [round(min(step_ms), 4), round(max(step_ms), 4)],
-        "n_kept": n_kept,
-    }
+        "selection": sel, "budget_sweep": sweep,
+        "e2e_copy_all": e2e_copy_all, "decode": decode, "incremental": incremental, "n_kept": n_kept,
+    })
     print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
 
 
-def run_incremental(args, s, dev, stream, hbm):
+def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4096, n_dec=64, seed=5):
     """Boundaries of the incremental loop on device-random K/V/Q (layout and signals from the seeded
-    generator).  The cache lives in one capacity buffer per layer and is compacted in place (hole
-    filling); each new step is appended after the retained rows.  Events time each compression and each
-    group of 64 decode reads."""
+    generator).  The cache lives in one capacity buffer per layer and is compacted in place (hole filling);
+    each new step is appended after the retained rows.  Events time each compression and each group of
+    n_dec decode reads.  With growth_total, the new steps' lengths are rescaled to add that many tokens
+    over the loop."""
     import numpy as np
     import torch
     from paper_2609_22158_gb300 import binding as B, workload as wl
-    budget, t0, n_dec = 8192, 4096, 64
-    lp = wl.IncrementalLoop(5, L=s.L, Hq=s.Hq, Hkv=s.Hkv, d=s.d, W=s.W, t0=t0, budget_count=budget)
+    budget = 8192
+    lp = wl.IncrementalLoop(seed, L=s.L, Hq=s.Hq, Hkv=s.Hkv, d=s.d, W=s.W, t0=t0, budget_count=budget,
+                            n_boundaries=n_boundaries if growth_total else None, growth_total=growth_total)
     gen = torch.Generator(device=dev).manual_seed(55)
-    cap = budget + 16 + 4 * s.W + 2400  # retained rows + the largest new step
+    max_new = max(lp.step_length(b) for b in range(1, n_boundaries))
+    cap = max(t0, budget + 16 + 4 * s.W) + max_new + 64  # retained rows + the largest new step
     Kbuf = [torch.randn((s.Hkv, cap, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
     Vbuf = [torch.randn((s.Hkv, cap, s.d), generator=gen, device=dev, dtype=torch.bfloat16) for _ in range(s.L)]
     step_id, n_steps = lp.initial_layout()
@@ -548,7 +798,7 @@ def run_incremental(args, s, dev, stream, hbm):
     ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, cap) + 512,
                        dtype=torch.uint8, device=dev)
     outd = [torch.empty((s.Hq, s.d), dtype=torch.float32, device=dev) for _ in range(s.L)]
-    for b in range(args.inc_boundaries):
+    for b in range(n_boundaries):
         if b > 0:
             n_new = lp.step_length(b)
             n_steps += 1
@@ -604,54 +854,102 @@ def run_incremental(args, s, dev, stream, hbm):
     steady = [i for i in range(len(rows)) if rows[i] > budget + 2 * s.W]  # the budget binds
     pick = steady or list(range(len(rows)))
     mean = lambda xs: float(np.mean([xs[i] for i in pick]))
-    return {"workload": f"incremental loop: {args.inc_boundaries} boundaries from a {t0}-token start, one new "
-                        f"step each, fixed {budget}-token budget, cache compacted in place (hole filling), "
-                        f"{n_dec} decode reads after each compression; {s.L} layers, Hq={s.Hq}, Hkv={s.Hkv}, "
-                        f"d={s.d}, W={s.W}",
-            "boundaries_with_budget_binding": len(steady),
+    # algorithmic bytes of one in-place boundary: the saliency layers' keys read once, every moved row's K
+    # and V read and written in every layer and head, the selection's per-token metadata
+    row_b = s.d * 2
+    alg = [s.Ls * s.Hkv * rows[i] * row_b + 2 * 2 * s.L * s.Hkv * moved[i] * row_b + rows[i] * 25 for i in range(len(rows))]
+    gbs = mean(alg) / (mean(comp_us) * 1e-6) / 1e9
+    dbytes = [2 * s.L * s.Hkv * min(rows[i], budget + 16 + s.W) * row_b for i in range(len(rows))]
+    dgbs = mean(dbytes) / (mean(dec_us) * 1e-6) / 1e9
+    return {"workload": f"incremental loop: {n_boundaries} boundaries from a {t0}-token start, one new step each"
+                        + (f" ({growth_total} tokens added over the loop)" if growth_total else "")
+                        + f", fixed {budget}-token budget, cache compacted in place (hole filling), {n_dec} decode "
+                        f"reads after each compression; {s.L} layers, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, W={s.W}",
+            "boundaries": n_boundaries, "boundaries_with_budget_binding": len(steady),
+            "trajectory_tokens_final": int(next_pos),
             "cache_rows_mean": round(mean(rows), 1), "rows_moved_mean": round(mean(moved), 1),
             "compress_us_mean": round(mean(comp_us), 2),
+            "compress_us_p50_p90": [round(float(np.percentile([comp_us[i] for i in pick], q)), 2) for q in (50, 90)],
+            "compress_algorithmic_bytes_mean": int(mean(alg)),
+            "compress_achieved_gbs": round(gbs, 1), "compress_frac_of_measured_hbm": round(gbs / peaks["hbm"], 4),
             "decode_us_per_token_mean": round(mean(dec_us), 2),
-            "compress_tokens_per_s": round(mean(rows) / (mean(comp_us) * 1e-6))}
+            "decode_frac_of_measured_hbm": round(dgbs / peaks["hbm"], 4),
+            "compress_tokens_per_s": round(mean(rows) / (mean(comp_us) * 1e-6)),
+            "tokens_compressed": int(sum(rows)), "compress_us_total": round(float(sum(comp_us)), 1)}
+
+
+def run_config5(args, world, rank, local, dist, dev, peaks):
+    """Config 5 as the line: the incremental loop's compressions are the timed work (value = cache tokens
+    compressed per second over all boundaries), decode reported beside them."""
+    import torch
+    from paper_2609_22158_gb300 import workload as wl
+    stream = torch.cuda.current_stream(dev)
+    s = wl.Shape(L=32, Hq=32, Hkv=8, d=128, T=4096, W=64)
+    sampler = ClockSampler(dev.index if world == 1 else local) if rank == 0 else None
+    wall0 = time.perf_counter()
+    inc = run_incremental(args.inc_boundaries_cfg5, s, dev, stream, peaks, growth_total=131072 - 4096)
+    wall = time.perf_counter() - wall0
+    clocks = sampler.stop() if sampler else None
+    if rank != 0:
+        return
+    value = inc["tokens_compressed"] / (inc["compress_us_total"] * 1e-6)
+    ms = inc["compress_us_total"] / inc["boundaries"] / 1e3
+    roof = {"kernel": "fused in-place boundary (score + select + hole-filling compaction)", "bound": "hbm",
+            "achieved": inc["compress_achieved_gbs"], "peak": peaks["hbm"], "unit": "GB/s",
+            "frac": inc["compress_frac_of_measured_hbm"], "traffic": None,
+            "algorithmic_bytes_per_launch": inc["compress_algorithmic_bytes_mean"]}
+    cfg_obj = {"workload": inc["workload"], "bench_config": 5, "global_batch": 1, "seq_len": inc["trajectory_tokens_final"],
+               "parallelism": "dp1", "l2": "not flushed: each boundary's inputs (the compacted cache plus the new step) "
+                                           "were just written by the previous boundary and its decode reads"}
+    line = base_line(args, value, ms, world, cfg_obj, roof, None, None, 3 * inc["boundaries"], clocks, wall, [ms])
+    line["steps"] = inc["boundaries"]
+    line["warmup"] = 0
+    line["incremental"] = inc
+    print(json.dumps(line), flush=True)
 
 
 # ---------------------------------------------------------------------------------- reference arm
 def run_reference(args):
-    """The oracle as it stands on the host cores, same workload/metric; each step a bounded sample."""
+    """The oracle as it stands on the host cores, same workload/metric/unit; each step one whole pass of
+    the workload (config 3: 4 of its 16 trajectories), the independent pairs and row sets spread over one
+    single-threaded process per core."""
     from paper_2609_22158_gb300 import multirank as MR
     world, rank, _ = MR.rank_env()
     if rank != 0:
         return
-    tr = make_traj(args)
-    s = tr.shape
-    times = []
-    desc = ""
-    for i in range(args.warmup + args.steps):
-        secs, desc, _ = oracle_pass_seconds(args, pairs=args.ref_pairs, compact_sets=args.ref_compact_sets)
-        if i >= args.warmup:
-            times.append(secs)
+    cfg = args.config if args.config != 5 else 2
+    trs = make_trajs(cfg)
+    cores = os.cpu_count() or 1
+    pick = [0, 5, 10, 15] if len(trs) > 4 else None
+    res = oracle_timing(cfg, cores, reps=args.warmup + args.steps, trajs=pick)
+    times = [p["total_s"] for p in res["passes"][args.warmup:]]
     sec = sum(times) / len(times)
-    value = s.T / sec
+    value = res["tokens"] / sec
+    sample = (f"one whole pass per step over {'4 of the 16 trajectories' if pick else 'the workload'}: saliency of "
+              f"every (layer, KV head) pair ({res['pairs']}), the boundary, every row set's gather (row sets drawn from "
+              f"one generated layer); {cores} single-threaded processes; throughput in the sampled tokens")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator)",
-        "config": workload_config(tr, args, 1),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc},
+        "config": workload_config(trs, cfg, 1),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "stages_s_last_pass": {k: round(v, 3) for k, v in res["passes"][-1].items()},
     }
     print(json.dumps(line), flush=True)
 
 
 def main():
+    if len(sys.argv) >= 3 and sys.argv[1] == "--oracle-worker":
+        print(json.dumps(oracle_worker(json.loads(sys.argv[2]))), flush=True)
+        return
     ap = argparse.ArgumentParser()
+    ap.add_argument("--config", type=int, choices=[1, 2, 3, 4, 5], default=2)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--seed", type=int, default=1)
-    ap.add_argument("--T", type=int, default=32768)
-    ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -659,19 +957,8 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--no-incremental", action="store_true")
     ap.add_argument("--inc-boundaries", type=int, default=24)
-    ap.add_argument("--oracle-pairs", type=int, default=24)
-    ap.add_argument("--oracle-compact-sets", type=int, default=16)
-    ap.add_argument("--ref-pairs", type=int, default=2)
-    ap.add_argument("--ref-compact-sets", type=int, default=4)
-    ap.add_argument("--compact-traffic", type=float, default=None,
-                    help="dram bytes (read+write) per compaction launch from an ncu capture of this workload "
-                         "(default: the capture of the current compaction kernel for the 32-layer 32K workload)")
+    ap.add_argument("--inc-boundaries-cfg5", type=int, default=200)
     args = ap.parse_args()
-    if args.compact_traffic is None and args.T == 32768 and args.layers == 32:
-        # dram__bytes_read.sum + dram__bytes_write.sum of compact_kernel from one single-pass ncu capture
-        # of this workload at full size (the timed step's launch): 438.94 MB read + 388.77 MB written.
-        # The ~50 MB of writes below the algorithmic bytes are dirty lines still in L2 when it ends.
-        args.compact_traffic = 438.94e6 + 388.77e6
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -340,7 +340,8 @@ class IncrementalLoop:
     """
 
     def __init__(self, seed: int, L: int, Hq: int, Hkv: int, d: int, W: int, t0: int, budget_count: int,
-                 n_prompt: int = 16, n_steps0: int = 8, n_sal_layers: int = 3):
+                 n_prompt: int = 16, n_steps0: int = 8, n_sal_layers: int = 3, n_boundaries=None,
+                 growth_total=None):
         self.seed = int(seed)
         self.shape = Shape(L=L, Hq=Hq, Hkv=Hkv, d=d, T=t0, W=W, n_sal_layers=n_sal_layers)
         self.t0 = int(t0)
@@ -348,14 +349,28 @@ class IncrementalLoop:
         self.budget = Budget.fixed(budget_count)
         g = _rng(seed, _K_LAYOUT, 50_000)
         self.init_fields = _cycle_steps(g, n_steps0, (50, 300), (10, 50), (200, 2000), t0 - n_prompt, W)
+        # With growth_total, the steps of boundaries 1 .. n_boundaries-1 are drawn as below and then
+        # rescaled (largest remainder) to add exactly growth_total tokens over the loop, e.g. 200
+        # boundaries growing a 4096-token start to 131072 tokens (mean ~635 tokens per step).
+        self._scaled = None
+        if growth_total is not None:
+            raw = np.array([self._raw_step_length(b) for b in range(1, int(n_boundaries))], dtype=np.int64)
+            self._scaled = _rescale_lengths(raw, int(growth_total))
+            if self._scaled.min() < W + 1:
+                raise ValueError("rescaled steps shorter than the window")
 
     # ---- layout
-    def step_length(self, b: int) -> int:
-        """Tokens of the step added at boundary b >= 1 (Thought + Action + Observation)."""
+    def _raw_step_length(self, b: int) -> int:
         g = _rng(self.seed, _K_LAYOUT, 60_000 + b)
         th, act = int(g.integers(50, 301)), int(g.integers(10, 51))
         obs = max(int(g.integers(200, 2001)), self.shape.W + 1)
         return th + act + obs
+
+    def step_length(self, b: int) -> int:
+        """Tokens of the step added at boundary b >= 1 (Thought + Action + Observation)."""
+        if self._scaled is not None:
+            return int(self._scaled[b - 1])
+        return self._raw_step_length(b)
 
     def initial_layout(self):
         """(step_id [t0], n_steps) of the first boundary's trajectory."""

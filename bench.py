@@ -13,6 +13,9 @@ by torch's seeded device RNG (K/V of the other layers):
   5  incremental agent loop: Llama-3-8B heads, 200 boundaries growing from 4096 to 131072 tokens,
      the compacted cache plus the new step compressed in place under a fixed 8192-token budget, 64
      single-token decode reads after each compression
+  6  config 2 with saliency from the whole last Observation (--window tokens, default 2048) instead
+     of a 64-token window: the queries of the observation prefill
+  7  config 4 with saliency from the whole last Observation (--window tokens, default 2048)
 
 Inputs are resident in HBM when the timed region starts; an L2 flush (a 512 MB write) runs between timed
 passes, outside their events.
@@ -64,9 +67,13 @@ def _peaks():
 
 
 # ---------------------------------------------------------------------------------- workloads
-def make_trajs(cfg: int, seed=None):
+def make_trajs(cfg: int, seed=None, window: int = 2048):
     """The trajectories of one bench configuration (config 5 is the incremental loop: see run_incremental)."""
     from paper_2609_22158_gb300 import workload as wl
+    if cfg == 6:
+        return [wl.observation_prefill("llama8b_32k", window, seed)]
+    if cfg == 7:
+        return [wl.observation_prefill("qwen32b_64k", window, seed)]
     if cfg == 1:
         return [wl.tiny(0 if seed is None else seed)]
     if cfg == 2:
@@ -86,6 +93,10 @@ def describe(trs, budget_label=None):
     if len(trs) == 1:
         name = {"tiny": "tiny trajectory", "llama8b_32k": "llama3-8b-shaped agent trajectory",
                 "qwen32b_64k": "qwen2.5-32b-shaped long-horizon trajectory"}.get(tr.name, tr.name)
+        if "_obs" in tr.name:
+            base = tr.name.split("_obs")[0]
+            name = {"llama8b_32k": "llama3-8b-shaped", "qwen32b_64k": "qwen2.5-32b-shaped"}[base] + (
+                " trajectory, saliency from the whole last Observation (observation prefill)")
         return (f"{name}: L={s.L}, Hq={s.Hq}, Hkv={s.Hkv}, d={s.d}, T={s.T}, W={s.W}, {tr.n_steps} steps, saliency "
                 f"from last {s.Ls} layers, budget {bud}")
     Ts = [t.T for t in trs]
@@ -197,10 +208,14 @@ def kernel_rooflines(tr, stage_us, n_kept, peaks, cfg):
     gbs = ab["score"] / (us * 1e-6) / 1e9
     tfs2 = 2 * ab["score_flops_one_pass"] / (us * 1e-6) / 1e12
     exps2 = 2 * ab["score_exps_one_pass"] / (us * 1e-6)
+    # the bound: whichever roof allows the least time (both passes' contractions vs one read of the keys)
+    tensor_bound = 2 * ab["score_flops_one_pass"] / (peaks["bf16"] * 1e12) > ab["score"] / (hbm * 1e9)
+    head = ({"bound": "tensor", "achieved": round(tfs2, 1), "peak": peaks["bf16"], "unit": "TFLOP/s",
+             "frac": round(tfs2 / peaks["bf16"], 4), "hbm_achieved_gbs": round(gbs, 1)} if tensor_bound else
+            {"bound": "hbm", "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4)})
     out["score_kernel"] = {
         "stage": "1-2: saliency, two tcgen05 passes (row statistics, per-key mass) + fixed-point T accumulation",
-        "bound": "hbm", "launch_us": round(us, 2), "algorithmic_bytes": ab["score"],
-        "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4),
+        "launch_us": round(us, 2), "algorithmic_bytes": ab["score"], **head,
         "tensor": {"achieved_tflops_both_passes": round(tfs2, 1), "peak": peaks["bf16"],
                    "frac": round(tfs2 / peaks["bf16"], 4), "one_pass_roof_us": round(
                        ab["score_flops_one_pass"] / (peaks["bf16"] * 1e12) * 1e6, 2)},
@@ -283,7 +298,7 @@ def oracle_worker(spec: dict) -> dict:
 
     from oracle import stepkv_oracle as O
     global _ORACLE_STATE
-    trs = make_trajs(spec["cfg"])
+    trs = make_trajs(spec["cfg"], window=spec.get("window", 2048))
     pick = spec.get("trajs")
     if pick is not None:
         trs = [trs[i] for i in pick]
@@ -294,7 +309,9 @@ def oracle_worker(spec: dict) -> dict:
         data.append((tr, Ks, Qs, tr.values(tr.sal_layer_ids()[0])))
     _ORACLE_STATE = data
     workers = int(spec["workers"])
-    pairs = [(b, li, h) for b, (tr, Ks, _, _) in enumerate(data) for li in range(len(Ks)) for h in range(tr.shape.Hkv)]
+    all_pairs = [(b, li, h) for b, (tr, Ks, _, _) in enumerate(data) for li in range(len(Ks)) for h in range(tr.shape.Hkv)]
+    limit = spec.get("pair_limit")
+    pairs = all_pairs[:limit] if limit else all_pairs
     pool = mp.get_context("fork").Pool(workers) if workers > 1 else None
     times = []
     try:
@@ -302,6 +319,7 @@ def oracle_worker(spec: dict) -> dict:
             t0 = time.perf_counter()
             A = (pool.map(_oracle_pair, pairs, chunksize=1) if pool else [_oracle_pair(x) for x in pairs])
             t1 = time.perf_counter()
+            A += [np.zeros(data[b][0].T) for (b, _, _) in all_pairs[len(pairs):]]  # unsampled pairs (scaled below)
             outs = []
             i = 0
             for (tr, Ks, _, _) in data:
@@ -322,12 +340,15 @@ def oracle_worker(spec: dict) -> dict:
                 for x in sets:
                     _oracle_gather(x)
             t3 = time.perf_counter()
-            times.append({"score_s": t1 - t0, "select_s": t2 - t1, "compact_s": t3 - t2, "total_s": t3 - t0})
+            score_s = (t1 - t0) * len(all_pairs) / len(pairs)
+            times.append({"score_s": score_s, "select_s": t2 - t1, "compact_s": t3 - t2,
+                          "total_s": score_s + (t3 - t1)})
     finally:
         if pool:
             pool.close()
             pool.join()
-    return {"passes": times, "tokens": int(sum(tr.T for tr in trs)), "pairs": len(pairs),
+    return {"passes": times, "tokens": int(sum(tr.T for tr in trs)), "pairs": len(all_pairs),
+            "pairs_timed": len(pairs),
             "n_kept": [int(len(o["kept"])) for o in outs]}
 
 
@@ -350,13 +371,13 @@ def _oracle_gather(x):
     return O.compact_rows(V0[h:h + 1], kept).shape
 
 
-def oracle_timing(cfg: int, workers: int, reps: int = 1, trajs=None) -> dict:
+def oracle_timing(cfg: int, workers: int, reps: int = 1, trajs=None, window: int = 2048, pair_limit=None) -> dict:
     """Run oracle_worker in a fresh process with single-threaded numpy (``workers`` processes)."""
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS"):
         env[k] = "1"
     env["CUDA_VISIBLE_DEVICES"] = ""
-    spec = {"cfg": cfg, "workers": workers, "reps": reps, "trajs": trajs}
+    spec = {"cfg": cfg, "workers": workers, "reps": reps, "trajs": trajs, "window": window, "pair_limit": pair_limit}
     r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-worker", json.dumps(spec)],
                        stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True, env=env, timeout=3600)
     if r.returncode != 0:
@@ -364,14 +385,16 @@ def oracle_timing(cfg: int, workers: int, reps: int = 1, trajs=None) -> dict:
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def cpu_baseline(cfg: int, trs) -> dict:
+def cpu_baseline(cfg: int, trs, window: int = 2048) -> dict:
     """The oracle on the host cores: all cores (headline) and one thread, each on a bounded sample."""
     cores = os.cpu_count() or 1
     pick = None
     if len(trs) > 4:  # the 16-trajectory batch: time 4 trajectories, scale by tokens
         pick = [0, 5, 10, 15]
-    res_all = oracle_timing(cfg, cores, reps=1, trajs=pick)
-    res_one = oracle_timing(cfg, 1, reps=1, trajs=pick[:1] if pick else None)
+    # observation-length windows: one thread times one (layer, KV head) pair's saliency, scaled to all
+    one_limit = 1 if cfg in (6, 7) else None
+    res_all = oracle_timing(cfg, cores, reps=1, trajs=pick, window=window)
+    res_one = oracle_timing(cfg, 1, reps=1, trajs=pick[:1] if pick else None, window=window, pair_limit=one_limit)
     def tps(res):
         return res["tokens"] / res["passes"][-1]["total_s"]
     what = (f"{len(pick)} of {len(trs)} trajectories (every stage of each), throughput in their tokens"
@@ -383,7 +406,9 @@ def cpu_baseline(cfg: int, trs) -> dict:
             "stages_s": {k: round(v, 3) for k, v in res_all["passes"][-1].items()},
             "single_thread": {"value": tps(res_one), "cores": 1,
                               "seconds_per_pass": round(res_one["passes"][-1]["total_s"], 3),
-                              "sample": "first trajectory only" if pick else "the whole pass"}}
+                              "sample": ("first trajectory only" if pick else
+                                         "saliency of 1 pair scaled to all, the rest of the pass whole"
+                                         if one_limit else "the whole pass")}}
 
 
 # ---------------------------------------------------------------------------------- GPU helpers
@@ -675,7 +700,7 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     params = B.Params()
-    trs = make_trajs(args.config, None if world == 1 else MR.rank_seed(args.config, rank))
+    trs = make_trajs(args.config, None if world == 1 else MR.rank_seed(args.config, rank), window=args.window)
     status = B.new_status(dev)
     dts = []
     for i, tr in enumerate(trs):
@@ -726,14 +751,16 @@ def run_ours(args):
     if rank == 0 and len(dts) == 1 and not args.no_stages:
         stage = stage_times(dts[0], params, stream, flush, max(3, min(args.steps, 20)))
         kernels = kernel_rooflines(dts[0].tr, stage, n_kept[0], peaks, args.config)
-        roof = dict(kernels["compact_kernel"])
-        roof["kernel"] = "compact_kernel (dominant: ~half the pass)"
-        roof["peak_source"] = f"{peaks['kind']} hbm_gbs (burst copy)"
+        dom = max(kernels, key=lambda k: kernels[k]["launch_us"])
+        roof = dict(kernels[dom])
+        roof["kernel"] = f"{dom} (dominant: {100 * stage[dom.split('_')[0]] / sum(stage.values()):.0f}% of the stage time)"
+        roof["peak_source"] = (f"{peaks['kind']} hbm_gbs (burst copy)" if roof["bound"] == "hbm" else
+                               f"{peaks['kind']} bf16_tflops (burst cuBLAS)")
         sel = selection_report(dts[0], params, stream)
     e2e = e2e_copy_all = None
     if not args.no_e2e and len(dts) == 1:
         e2e, e2e_copy_all = e2e_single(dts[0], params, stream, dist, dev, tokens, args.e2e_steps,
-                                       with_copy_all=args.config != 4)
+                                       with_copy_all=args.config not in (4, 7))
     decode = incremental = None
     if rank == 0 and args.config == 2 and not args.no_decode:
         decode = decode_report(dts[0].tr.shape, dev, stream, flush, status, hbm)
@@ -752,7 +779,7 @@ def run_ours(args):
     pass_gbs = total_bytes / (ms * 1e-3) / 1e9
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        cpu = cpu_baseline(args.config, trs)
+        cpu = cpu_baseline(args.config, trs, args.window)
     launches = launches_per_call(trs) * args.steps
     line = base_line(args, value, ms, world, workload_config(trs, args.config, world, "10% of prunable (sweep: 5/10/20%)"
                                                             if sweep else None),
@@ -918,10 +945,10 @@ def run_reference(args):
     if rank != 0:
         return
     cfg = args.config if args.config != 5 else 2
-    trs = make_trajs(cfg)
+    trs = make_trajs(cfg, window=args.window)
     cores = os.cpu_count() or 1
     pick = [0, 5, 10, 15] if len(trs) > 4 else None
-    res = oracle_timing(cfg, cores, reps=args.warmup + args.steps, trajs=pick)
+    res = oracle_timing(cfg, cores, reps=args.warmup + args.steps, trajs=pick, window=args.window)
     times = [p["total_s"] for p in res["passes"][args.warmup:]]
     sec = sum(times) / len(times)
     value = res["tokens"] / sec
@@ -945,7 +972,8 @@ def main():
         print(json.dumps(oracle_worker(json.loads(sys.argv[2]))), flush=True)
         return
     ap = argparse.ArgumentParser()
-    ap.add_argument("--config", type=int, choices=[1, 2, 3, 4, 5], default=2)
+    ap.add_argument("--config", type=int, choices=[1, 2, 3, 4, 5, 6, 7], default=2)
+    ap.add_argument("--window", type=int, default=2048, help="observation length for configs 6 and 7")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)

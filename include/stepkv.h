@@ -312,6 +312,30 @@ STEPKV_API stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q,
                               float* const* out, void* ws, size_t ws_bytes, int32_t* dev_status,
                               void* stream);
 
+/* ---------------------------------------------------------------------------------------------
+ * Decode attention that also accumulates attention mass: the H2O-style token saliency (Sec. 4.2: T_i
+ * "can be supplied by existing token-level KV importance estimators"; H2O scores a token by the
+ * attention it has received).  Same arguments, outputs and rules as stepkv_decode, plus:
+ *
+ *  mass[l]  host array of device pointers, [Hkv][mass_head_stride >= n_cap] float32, read and
+ *           written (4-byte aligned): for every KV head h and key j < n the call ADDS
+ *             (1/G) * sum_{g = hG}^{hG+G-1} softmax_j( q[l][g] . K[l][h][j] / sqrt(d) )
+ *           i.e. the key's softmax weight averaged over the GQA group (each call adds a total of 1
+ *           per head over the keys).  The caller zeroes the rows (e.g. after a boundary) and reads
+ *           them as saliency rows, e.g. stepkv_select(sal = mass rows of chosen layers, n_sal =
+ *           layers x Hkv): T_i is then the mean accumulated attention of token i (Eq. 5's T_i).
+ *  ws       stepkv_decode_h2o_workspace_size bytes: the split partials and every key's logits.
+ *  out is bit-identical to stepkv_decode's on the same inputs; the masses are deterministic (one
+ *  writer per element and call, heads summed in a fixed order).
+ */
+STEPKV_API size_t stepkv_decode_h2o_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t d,
+                                                   int32_t n_cap);
+STEPKV_API stepkv_status_t stepkv_decode_h2o(int32_t n_layers, const void* const* q, const void* const* K,
+                                  const void* const* V, int64_t kv_head_stride, int32_t Hkv, int32_t Hq,
+                                  int32_t d, const int32_t* n_dev, int32_t n_host, int32_t n_cap,
+                                  float* const* out, float* const* mass, int64_t mass_head_stride,
+                                  void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
 /* Failure-detection self-test (no counterpart in the paper).  Runs the saliency kernel of stepkv_score
  * on the same arguments, except that the wait of its second pass (for every CTA's first-pass flag)
  * looks for a value no CTA ever publishes, so every CTA's wait runs out after wait_limit_ns

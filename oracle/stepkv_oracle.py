@@ -279,3 +279,25 @@ def decode_attention(q: np.ndarray, K: np.ndarray, V: np.ndarray) -> np.ndarray:
         e = np.exp(s)
         out[g] = (e / e.sum()) @ Vf[h]
     return out
+
+
+def decode_attention_mass(q: np.ndarray, K: np.ndarray) -> np.ndarray:
+    """Accumulated-attention token saliency of one decode read (Sec. 4.2: T_i "can be supplied by existing
+    token-level KV importance estimators"; H2O scores a token by the attention mass it receives).
+    q [Hq, d], K [Hkv, n, d] bf16 bits -> A [Hkv, n] float64 with
+        A[h, j] = (1/G) * sum_{g in group(h)} softmax_j(q_g . K[h, j] / sqrt(d)),
+    the softmax weight key j receives from the group's query heads (mean over the GQA group, as for the
+    window saliency).  Summed over the decode reads between two boundaries it is the H2O score."""
+    qf = bf16_to_f64(q)
+    Kf = bf16_to_f64(K)
+    Hq, d = qf.shape
+    Hkv, n, _ = Kf.shape
+    G = Hq // Hkv
+    A = np.zeros((Hkv, n))
+    for g in range(Hq):
+        h = g // G
+        s = Kf[h] @ qf[g] / math.sqrt(d)
+        s = s - s.max()
+        e = np.exp(s)
+        A[h] += e / e.sum()
+    return A / G

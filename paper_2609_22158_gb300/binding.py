@@ -90,6 +90,9 @@ SIGNATURES = {
     "stepkv_compact": (_I32, [_I32, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _VP, _I32, _VP, _VP, _I64, _VP, _VP,
                               _VP, _VP, _VP, _VP]),
     "stepkv_decode_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
+    "stepkv_decode_h2o_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
+    "stepkv_decode_h2o": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _I64, _VP,
+                                 _SZ, _VP, _VP]),
     "stepkv_decode": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _SZ, _VP,
                              _VP]),
     "stepkv_compress_workspace_size": (_SZ, [ctypes.POINTER(CProblem), _I32]),
@@ -421,6 +424,49 @@ def stepkv_decode(q: Sequence, K: Sequence, V: Sequence, n, out: Optional[Sequen
     code = lib.stepkv_decode(L, cv(arrs[0]), cv(arrs[1]), cv(arrs[2]), hs, Hkv, Hq, d, _ptr(n_dev), n_host, rows,
                              cv(arrs[3]), wp, wn, status.data_ptr(), _stream_handle(stream))
     _check(code, "stepkv_decode")
+    return out
+
+
+def stepkv_decode_h2o(q: Sequence, K: Sequence, V: Sequence, n, mass: Sequence, out: Optional[Sequence] = None,
+                      ws=None, status=None, stream=None):
+    """stepkv_decode that also adds each key's group-mean softmax weight to mass[l] ([Hkv, >= rows] fp32,
+    accumulated in place): the H2O-style accumulated attention.  Returns the outputs as stepkv_decode."""
+    torch = _torch()
+    lib = load_library()
+    L = len(q)
+    if L < 1 or len(K) != L or len(V) != L or len(mass) != L:
+        raise ValueError("q, K, V and mass need one tensor per layer")
+    hs = _rows_layout(list(K) + list(V), "K/V")
+    Hkv, rows, d = K[0].shape
+    for i, t in enumerate(q):
+        _need(t, torch.bfloat16, f"q[{i}]", 2)
+        if not t.is_contiguous():
+            raise ValueError(f"q[{i}] must be contiguous")
+    for i, t in enumerate(mass):
+        _need(t, torch.float32, f"mass[{i}]", 2)
+        if t.shape[0] != Hkv or t.shape[1] < rows or t.stride(1) != 1 or t.stride(0) != mass[0].stride(0):
+            raise ValueError("mass[l] must be [Hkv, >= rows] float32 with unit column stride and one row stride")
+    Hq = q[0].shape[0]
+    dev = q[0].device
+    if out is None:
+        out = [torch.empty((Hq, d), dtype=torch.float32, device=dev) for _ in range(L)]
+    for i, t in enumerate(out):
+        _need(t, torch.float32, f"out[{i}]", 2)
+    if isinstance(n, int):
+        n_dev, n_host = None, n
+    else:
+        _need(n, torch.int32, "n")
+        n_dev, n_host = n, 0
+    need = lib.stepkv_decode_h2o_workspace_size(L, Hkv, Hq, d, rows)
+    ws = _workspace(need + 256, ws, dev)
+    wp, wn = _aligned_ws(ws)
+    status = status if status is not None else new_status(dev)
+    arrs = [_ptr_array(q), _ptr_array(K), _ptr_array(V), _ptr_array(out), _ptr_array(mass)]
+    cv = lambda a: ctypes.cast(a, ctypes.c_void_p)
+    code = lib.stepkv_decode_h2o(L, cv(arrs[0]), cv(arrs[1]), cv(arrs[2]), hs, Hkv, Hq, d, _ptr(n_dev), n_host, rows,
+                                 cv(arrs[3]), cv(arrs[4]), mass[0].stride(0), wp, wn, status.data_ptr(),
+                                 _stream_handle(stream))
+    _check(code, "stepkv_decode_h2o")
     return out
 
 

@@ -375,6 +375,39 @@ stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q, const void
                     static_cast<cudaStream_t>(stream));
 }
 
+size_t stepkv_decode_h2o_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t d, int32_t n_cap) {
+  if (stepkv_decode_workspace_size(n_layers, Hkv, Hq, d, n_cap) == 0) return 0;
+  return decode_mass_ws_bytes(std::min(n_layers, kMaxDecodeLayers), Hkv, Hq, d, n_cap);
+}
+
+stepkv_status_t stepkv_decode_h2o(int32_t n_layers, const void* const* q, const void* const* K, const void* const* V,
+                                  int64_t kv_head_stride, int32_t Hkv, int32_t Hq, int32_t d, const int32_t* n_dev,
+                                  int32_t n_host, int32_t n_cap, float* const* out, float* const* mass,
+                                  int64_t mass_head_stride, void* ws, size_t ws_bytes, int32_t* dev_status,
+                                  void* stream) {
+  if (!mass || mass_head_stride < n_cap) return STEPKV_EINVAL;
+  for (int l = 0; l < n_layers; ++l)
+    if (!mass[l]) return STEPKV_EINVAL;
+  if (ws_bytes < stepkv_decode_h2o_workspace_size(n_layers, Hkv, Hq, d, n_cap)) return STEPKV_ENOSPACE;
+  // every other argument rule is stepkv_decode's
+  if (n_layers < 1 || !q || !K || !V || !out || !ws) return STEPKV_EINVAL;
+  if (Hkv < 1 || Hq < 1 || Hq % Hkv != 0 || n_cap < 1) return STEPKV_EINVAL;
+  if (d != 64 && d != 128) return STEPKV_EUNSUPPORTED;
+  const int G = Hq / Hkv;
+  if (G != 1 && G != 2 && G != 4 && G != 5 && G != 8) return STEPKV_EUNSUPPORTED;
+  if (kv_head_stride < (int64_t)n_cap * d) return STEPKV_EINVAL;
+  if (kv_head_stride % 8) return STEPKV_EUNSUPPORTED;
+  if (!n_dev && (n_host < 1 || n_host > n_cap)) return STEPKV_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
+  for (int l = 0; l < n_layers; ++l) {
+    if (!q[l] || !K[l] || !V[l] || !out[l]) return STEPKV_EINVAL;
+    if (!aligned16(q[l]) || !aligned16(K[l]) || !aligned16(V[l]) || !aligned16(out[l])) return STEPKV_EUNSUPPORTED;
+    if ((reinterpret_cast<uintptr_t>(mass[l]) & 3u) != 0) return STEPKV_EUNSUPPORTED;
+  }
+  return decode_run(n_layers, q, K, V, kv_head_stride, Hkv, Hq, d, n_dev, n_host, n_cap, out, ws, dev_status,
+                    static_cast<cudaStream_t>(stream), mass, mass_head_stride);
+}
+
 // K of the saliency layers as the score stage reads it (device memory in either cache location).
 static const void* const* sal_keys(const stepkv_problem_t& p) {
   const int Ls = std::min(p.n_sal_layers, p.L);

@@ -11,6 +11,13 @@
 // per block, and keeps a running (max, sum, weighted values) per head, rescaled once per block.  A
 // second kernel merges the per-split partials of each (pair, head) in split order (deterministic).
 // The number of keys may be read on the device (n_kept of a compaction), so no host sync is needed.
+//
+// Accumulated attention (the H2O-style token saliency, Sec. 4.2: T_i may come from an existing
+// token-level importance estimator): with mass rows given, the partial kernel also stores every key's
+// logits per head, and the merge runs one CTA per (layer, KV head): its warps merge the heads' splits
+// (same order as the plain merge, so the outputs are bit-identical) and record each head's log-sum-exp,
+// then its threads add (1/G) sum_g softmax_j(q_g . k_j / sqrt(d)) to mass[j] for every key (one writer
+// per element and call, fixed order over g: deterministic).
 #include <math.h>
 
 #include <algorithm>
@@ -38,6 +45,9 @@ struct DecodeArgs {
   int n_cap;
   float c;              // log2(e) / sqrt(d)
   float* part;          // [pairs][n_splits][G][d + 4]: m, l, -, -, acc[d]
+  float* logits;        // [pairs][n_cap][G] (accumulated-attention mode, else NULL): key logits in log2 units
+  float* mass[kMaxDecodeLayers];  // per layer [Hkv][mass_stride]: accumulated attention (+=), or NULL
+  int64_t mass_stride;
   int32_t* status;
 };
 
@@ -162,6 +172,18 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
         }
       }
     }
+    if (a.logits != nullptr && hl == 0) {
+      // every lane of a key row holds the row's logits of all G heads: the first one stores them
+#pragma unroll
+      for (int t = 0; t < kDecBlockSteps; ++t) {
+        const int j = kb + t * KPS + kslot;
+        if (ok[t]) {
+          float* dst = a.logits + ((size_t)pair * a.n_cap + j) * G;
+#pragma unroll
+          for (int g = 0; g < G; ++g) dst[g] = s[t][g];
+        }
+      }
+    }
     // probabilities of the block's keys per head (state rescaled once per block), then one pass over
     // the value rows: each is converted once and accumulated into every head
     float p[kDecBlockSteps][G];
@@ -269,9 +291,60 @@ __global__ void __launch_bounds__(128) decode_merge_kernel(const __grid_constant
   for (int e = 0; e < PER; ++e) o[e] = aa[e] * inv;
 }
 
+// Accumulated-attention merge: one CTA per (layer, KV head).  Warp w merges heads w, w + 4, ... exactly as
+// decode_merge_kernel does (bit-identical outputs) and keeps each head's log-sum-exp; then every thread adds
+// the group-mean softmax mass of its keys to the pair's mass row.
+template <int D, int G>
+__global__ void __launch_bounds__(128) decode_merge_mass_kernel(const __grid_constant__ DecodeArgs a) {
+  constexpr int PER = D / 32;
+  __shared__ float s_lse[G];
+  pdl_wait();
+  pdl_launch_dependents();
+  const int pair = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int layer = pair / a.Hkv, h = pair - layer * a.Hkv;
+  const int n = max(0, min(decode_n(a), a.n_cap));
+  const int used = max(0, min(a.n_splits, (n + kDecSplitKeys - 1) / kDecSplitKeys));
+  for (int g = warp; g < G; g += 4) {
+    float mm = -INFINITY, ll = 0.f, aa[PER];
+#pragma unroll
+    for (int e = 0; e < PER; ++e) aa[e] = 0.f;
+    for (int sp = 0; sp < used; ++sp) {
+      const float* src = a.part + ((size_t)(pair * a.n_splits + sp) * G + g) * (D + 4);
+      float a2[PER];
+#pragma unroll
+      for (int e = 0; e < PER; ++e) a2[e] = __ldcg(src + 4 + lane * PER + e);
+      merge_state<PER>(mm, ll, aa, __ldcg(src), __ldcg(src + 1), a2);
+    }
+    const float inv = ll > 0.f ? 1.f / ll : 0.f;
+    float* o = a.out[layer] + (size_t)(h * G + g) * D + lane * PER;
+#pragma unroll
+    for (int e = 0; e < PER; ++e) o[e] = aa[e] * inv;
+    if (lane == 0) s_lse[g] = ll > 0.f ? mm + __log2f(ll) : INFINITY;
+  }
+  __syncthreads();
+  float lse[G];
+#pragma unroll
+  for (int g = 0; g < G; ++g) lse[g] = s_lse[g];
+  const float inv_G = 1.f / (float)G;
+  float* mrow = a.mass[layer] + (size_t)h * a.mass_stride;
+  const float* lg = a.logits + (size_t)pair * a.n_cap * G;
+  for (int j = threadIdx.x; j < n; j += 128) {
+    float sum = 0.f;
+#pragma unroll
+    for (int g = 0; g < G; ++g) sum += ex2_approx(__ldcg(lg + (size_t)j * G + g) - lse[g]);
+    mrow[j] += sum * inv_G;
+  }
+}
+
 size_t decode_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap) {
   const int n_splits = std::max(1, (n_cap + kDecSplitKeys - 1) / kDecSplitKeys);
   return (size_t)n_layers * Hq * n_splits * (d + 4) * sizeof(float);
+}
+
+size_t decode_mass_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap) {
+  // partials (256-byte aligned), then the key logits of every head
+  const size_t part = (decode_ws_bytes(n_layers, Hkv, Hq, d, n_cap) + 255) & ~(size_t)255;
+  return part + (size_t)n_layers * Hq * std::max(1, n_cap) * sizeof(float);
 }
 
 template <int D, int G>
@@ -279,6 +352,7 @@ static cudaError_t decode_launch(const DecodeArgs& a, int pairs, cudaStream_t st
   cudaError_t e = launch_kernel(decode_partial_kernel<D, G>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
                                 stream, a);
   if (e != cudaSuccess) return e;
+  if (a.logits != nullptr) return launch_kernel(decode_merge_mass_kernel<D, G>, dim3(pairs), dim3(128), 0, stream, a);
   const int items = pairs * G;
   return launch_kernel(decode_merge_kernel<D, G>, dim3((items + 3) / 4), dim3(128), 0, stream, a, items);
 }
@@ -297,10 +371,15 @@ static cudaError_t decode_dispatch_g(const DecodeArgs& a, int G, int pairs, cuda
 
 stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const* K, const void* const* V,
                            int64_t head_stride, int Hkv, int Hq, int d, const int32_t* n_dev, int n_host, int n_cap,
-                           float* const* out, void* ws, int32_t* status, cudaStream_t stream) {
+                           float* const* out, void* ws, int32_t* status, cudaStream_t stream, float* const* mass,
+                           int64_t mass_stride) {
   const int G = Hq / Hkv;
   const int n_splits = std::max(1, (n_cap + kDecSplitKeys - 1) / kDecSplitKeys);
   float* part = static_cast<float*>(ws);
+  float* logits = nullptr;
+  if (mass != nullptr)
+    logits = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) +
+                                      ((decode_ws_bytes(n_layers, Hkv, Hq, d, n_cap) + 255) & ~(size_t)255));
   for (int l0 = 0; l0 < n_layers; l0 += kMaxDecodeLayers) {
     const int nl = std::min(kMaxDecodeLayers, n_layers - l0);
     DecodeArgs a;
@@ -310,7 +389,10 @@ stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const
       a.K[l] = static_cast<const uint16_t*>(K[l0 + l]);
       a.V[l] = static_cast<const uint16_t*>(V[l0 + l]);
       a.out[l] = out[l0 + l];
+      a.mass[l] = mass != nullptr ? mass[l0 + l] : nullptr;
     }
+    a.logits = logits;  // the chunk's pairs index their own slice of the logit scratch from 0
+    a.mass_stride = mass_stride;
     a.head_stride = head_stride;
     a.Hkv = Hkv;
     a.n_splits = n_splits;

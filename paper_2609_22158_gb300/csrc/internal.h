@@ -83,9 +83,12 @@ cudaError_t launch_cluster(void (*kern)(KArgs...), dim3 grid, dim3 block, int cl
 // ---- decode attention (decode.cu)
 constexpr int kMaxDecodeLayers = 64;  // layers per launch (pointer arrays travel in the kernel parameters)
 size_t decode_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap);
+size_t decode_mass_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap);
+// With mass (per layer [Hkv][mass_stride] fp32), each call also adds every key's group-mean softmax mass.
 stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const* K, const void* const* V,
                            int64_t head_stride, int Hkv, int Hq, int d, const int32_t* n_dev, int n_host, int n_cap,
-                           float* const* out, void* ws, int32_t* status, cudaStream_t stream);
+                           float* const* out, void* ws, int32_t* status, cudaStream_t stream,
+                           float* const* mass = nullptr, int64_t mass_stride = 0);
 
 // ---- score (score.cu)
 int score_row_groups(int Hkv, int Hq, int W);

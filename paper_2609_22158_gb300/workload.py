@@ -278,6 +278,32 @@ def llama8b_32k(seed: int = 1, budget: Optional[Budget] = None, T: int = 32768, 
                      needles_steps=5 if needles else 0)
 
 
+def observation_prefill(base: str = "llama8b_32k", W: int = 2048, seed: Optional[int] = None,
+                        budget: Optional[Budget] = None) -> Trajectory:
+    """Saliency from the whole last Observation instead of a short window: the queries are the |Obs_t| = W
+    tokens of the step just completed (the appendix's time-complexity passage collects T_i during the
+    observation prefill).  The layout is the base workload's (Llama-3-8B 32K: 40 steps, 10%; Qwen2.5-32B
+    64K: 120 steps, log-uniform Observations, 4096 tokens), except that the last step's Observation is
+    exactly W tokens long and is the protected window."""
+    if base == "llama8b_32k":
+        seed = 1 if seed is None else seed
+        shape = Shape(L=32, Hq=32, Hkv=8, d=128, T=32768, W=W)
+        n_steps, obs, obs_log, nd = 40, (200, 2000), False, 5
+        budget = budget or Budget.ratio(1, 10)
+    elif base == "qwen32b_64k":
+        seed = 3 if seed is None else seed
+        shape = Shape(L=64, Hq=40, Hkv=8, d=128, T=65536, W=W)
+        n_steps, obs, obs_log, nd = 120, (16, 4096), True, 0
+        budget = budget or Budget.fixed(4096)
+    else:
+        raise ValueError(base)
+    g = _rng(seed, _K_LAYOUT, 20_000 + W)
+    fl = _cycle_steps(g, n_steps, (50, 300), (10, 50), obs, shape.T - 16 - W, 0, obs_log=obs_log)
+    fl[-2, 2] += fl[-1, 2]  # the drawn last Observation joins the previous one; the last is exactly W
+    fl[-1, 2] = W
+    return _assemble(f"{base}_obs{W}", seed, shape, 16, fl, budget, _rng(seed, _K_SIGNALS), needles_steps=nd)
+
+
 def ragged_batch(seed: int = 2, n_traj: int = 16, budget: Optional[Budget] = None, L: int = 32,
                  t_lo: int = 8192, t_hi: int = 32768) -> List[Trajectory]:
     """16 trajectories, T ~ U(8K, 32K), Llama-3-8B head shapes, 24-60 steps each, 4 key channels

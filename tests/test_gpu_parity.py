@@ -60,6 +60,97 @@ def test_score_matches_oracle(B, Hkv, G, d, T, W, nl):
         assert np.allclose(g[l].sum(axis=1), W, rtol=1e-4)
 
 
+# Observation-length windows (the queries are a whole last Observation, hundreds to 4096 tokens): the
+# window is split over up to 16 row groups per query head, GQA 4 and 5.
+LONG_WINDOW_CASES = [
+    # Hkv, G, d, T, W
+    (1, 4, 128, 2500, 512),
+    (1, 5, 128, 3000, 1024),
+    pytest.param(1, 4, 128, 5000, 4096, marks=pytest.mark.slow),
+    pytest.param(1, 5, 128, 4300, 4096, marks=pytest.mark.slow),
+]
+
+
+@pytest.mark.parametrize("Hkv,G,d,T,W", LONG_WINDOW_CASES)
+def test_score_observation_length_window(B, Hkv, G, d, T, W):
+    import torch
+    rng = np.random.default_rng(2000 + T + W + G)
+    K = _rand_bits(rng, (Hkv, T, d))
+    Q = _rand_bits(rng, (Hkv * G, W, d))
+    st = B.new_status()
+    sal = B.stepkv_score([TL.bf16_dev(K)], [TL.bf16_dev(Q)], T, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    g = sal[0].cpu().numpy()
+    TL.assert_close(g, O.window_attention_saliency(K, Q), f"sal W={W}")
+    assert np.allclose(g.sum(axis=1), W, rtol=1e-4)
+
+
+def test_compress_observation_window(B):
+    """The fused pass with a 1024-token window (fixed-point accumulation over 16 row groups per pair)."""
+    import torch
+    tr = wl.custom(61, L=3, Hq=8, Hkv=2, d=128, T=3000, W=1024, n_steps=3, budget=wl.Budget.ratio(1, 4))
+    assert tr.step_id[-1] == tr.n_steps - 1 and (tr.step_id[-tr.shape.W:] == tr.n_steps - 1).all()
+    g = TL.GpuTraj(tr)
+    prob = g.problem()
+    st = B.stepkv_compress([prob], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    TL.check_select_outputs(g, TL.run_oracle(tr, O.Params()))
+
+
+@pytest.mark.slow
+def test_score_observation_prefill_full_size_sampled(B):
+    """The 32K Llama-shaped trajectory with its whole last Observation (2048 tokens, 8192 query rows per
+    KV head) as the window, in the launch the fused pass makes (all 3 saliency layers): one sampled
+    (layer, KV head) pair is computed by the oracle and compared over all 32768 keys; every pair's
+    masses must sum to W (each query row's softmax sums to one)."""
+    import torch
+    tr = wl.observation_prefill("llama8b_32k", 2048)
+    s = tr.shape
+    Ks = [tr.keys(l) for l in tr.sal_layer_ids()]
+    Qs = [tr.queries(l) for l in tr.sal_layer_ids()]
+    st = B.new_status()
+    sal = B.stepkv_score([TL.bf16_dev(k) for k in Ks], [TL.bf16_dev(q) for q in Qs], s.T, status=st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    g = sal.cpu().numpy()
+    assert np.allclose(g.sum(axis=2), s.W, rtol=1e-4)
+    li, h = 1, 5
+    ref = O.window_attention_saliency(Ks[li][h:h + 1], Qs[li][h * s.G:(h + 1) * s.G])[0]
+    TL.assert_close(g[li, h], ref, "sal full-size observation window, layer 1 head 5")
+
+
+# Table 2 and Table 3 ablations as oracle-checked modes of the fused pass: no redundancy penalty (lambda = 0),
+# no reuse credit (eta = 0), step utility alone (alpha = 0) and token saliency alone (beta = 0), plus the
+# un-normalised saliency.
+ABLATIONS = [
+    {"lam": 0.0}, {"eta": 0.0}, {"alpha": 0.0, "beta": 1.0}, {"alpha": 1.0, "beta": 0.0},
+    {"alpha": 0.5, "beta": 0.5, "sal_norm": 1},
+]
+
+
+@pytest.mark.parametrize("ablation", ABLATIONS, ids=lambda a: "-".join(f"{k}{v}" for k, v in a.items()))
+def test_compress_ablation_modes(B, ablation):
+    import torch
+    tr = wl.custom(81, L=4, Hq=16, Hkv=4, d=128, T=5000, W=64, n_steps=12, budget=wl.Budget.ratio(1, 8))
+    p = B.Params()
+    for k, v in ablation.items():
+        setattr(p, k, v)
+    g = TL.GpuTraj(tr)
+    prob = g.problem()
+    st = B.stepkv_compress([prob], p)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    out = TL.run_oracle(tr, TL.oracle_params(p))
+    TL.check_select_outputs(g, out)
+    n = int(g.out.n_kept.item())
+    kt = g.out.kept_idx[:n].long()
+    for l in range(tr.shape.L):
+        assert torch.equal(g.K_out[l][:, :n], g.K[l].index_select(1, kt))
+        assert torch.equal(g.V_out[l][:, :n], g.V[l].index_select(1, kt))
+
+
 def test_score_capacity_head_stride(B):
     """K rows live in a larger capacity buffer ([Hkv, cap, d] with cap > T)."""
     import torch

@@ -390,6 +390,75 @@ def test_decode_bruteforce():
     check_decode_bruteforce(REAL)
 
 
+# ------------------------------------------------------------------ accumulated decode attention (H2O-style)
+def check_mass_single_query_softmax(O):
+    """One KV head, one query head: the mass is the textbook softmax of the scaled logits (scipy)."""
+    rng = np.random.default_rng(31)
+    q, K = _bits(rng.standard_normal((1, 16))), _bits(rng.standard_normal((1, 37, 16)))
+    A = O.decode_attention_mass(q, K)
+    ref = softmax(REAL.bf16_to_f64(K)[0] @ REAL.bf16_to_f64(q)[0] / 4.0)
+    assert np.allclose(A[0], ref, rtol=1e-12, atol=0)
+
+
+def check_mass_sums(O):
+    """Every KV head receives a total of exactly one per read (each query head's softmax sums to one, and
+    the group's heads are averaged); summed over reads, the masses total the number of reads."""
+    rng = np.random.default_rng(32)
+    Hkv, G, n, d = 3, 4, 50, 32
+    tot = np.zeros((Hkv, n))
+    for r in range(5):
+        A = O.decode_attention_mass(_bits(rng.standard_normal((Hkv * G, d))), _bits(rng.standard_normal((Hkv, n, d))))
+        assert np.allclose(A.sum(axis=1), 1.0, rtol=0, atol=1e-12)
+        assert (A >= 0).all()
+        tot += A
+    assert np.allclose(tot.sum(axis=1), 5.0, rtol=0, atol=1e-11)
+
+
+def check_mass_two_key_analytic(O):
+    """Two keys: the first key's weight is the logistic function of the scaled logit difference."""
+    q = _bits(np.full((1, 16), 0.5))
+    K = _bits(np.stack([np.full(16, 1.0), np.full(16, -0.5)])[None])
+    A = O.decode_attention_mass(q, K)
+    s0, s1 = 16 * 0.5 * 1.0 / 4.0, 16 * 0.5 * -0.5 / 4.0
+    assert abs(A[0, 0] - expit(s0 - s1)) < 1e-14 and abs(A[0, 1] - expit(s1 - s0)) < 1e-14
+
+
+def check_mass_gqa(O):
+    """Query head g reads KV head g // G: a group whose heads all match key 0 puts its mass there."""
+    d, n = 16, 4
+    K = np.zeros((2, n, d), np.float32)
+    K[0, 0, 0] = K[0, 1, 1] = 8.0   # KV head 0: key 0 along e0, key 1 along e1
+    K[1, 2, 0] = K[1, 3, 1] = 8.0   # KV head 1: key 2 along e0, key 3 along e1
+    q = np.zeros((4, d), np.float32)  # G = 2: heads 0, 1 -> KV head 0; heads 2, 3 -> KV head 1
+    q[0, 0] = q[1, 0] = 8.0           # group of KV head 0 looks along e0
+    q[2, 1] = q[3, 1] = 8.0           # group of KV head 1 looks along e1
+    A = O.decode_attention_mass(_bits(q), _bits(K))
+    assert A[0, 0] > 0.99 and A[1, 3] > 0.99
+
+
+def check_mass_bruteforce(O):
+    """Plain loops over heads and keys, exponentials and sums written out, on a tiny case."""
+    rng = np.random.default_rng(33)
+    Hkv, G, n, d = 2, 2, 5, 4
+    q, K = _bits(rng.standard_normal((Hkv * G, d))), _bits(rng.standard_normal((Hkv, n, d)))
+    qf, Kf = REAL.bf16_to_f64(q), REAL.bf16_to_f64(K)
+    ref = np.zeros((Hkv, n))
+    for g in range(Hkv * G):
+        h = g // G
+        logits = [sum(qf[g, e] * Kf[h, j, e] for e in range(d)) / math.sqrt(d) for j in range(n)]
+        ex = [math.exp(x) for x in logits]
+        tot = sum(ex)
+        for j in range(n):
+            ref[h, j] += ex[j] / tot / G
+    assert np.allclose(O.decode_attention_mass(q, K), ref, rtol=1e-12, atol=0)
+
+
+@pytest.mark.parametrize("chk", [check_mass_single_query_softmax, check_mass_sums, check_mass_two_key_analytic,
+                                 check_mass_gqa, check_mass_bruteforce])
+def test_decode_mass_pins(chk):
+    chk(REAL)
+
+
 # ------------------------------------------------------------------ end-to-end invariants
 def test_boundary_invariants_tiny():
     tr = wl.tiny(0)
@@ -625,6 +694,28 @@ def _boundary_stats_on_raw(A_layers, step_id, prot, valid, gain, red, obs_sim, r
     return out
 
 
+def _mass_sum_over_group(q, K):
+    # sum over the GQA group instead of the mean
+    return REAL.decode_attention_mass(q, K) * (q.shape[0] // K.shape[0])
+
+
+def _mass_no_scale(q, K):
+    qf, Kf = REAL.bf16_to_f64(q), REAL.bf16_to_f64(K)
+    G = qf.shape[0] // Kf.shape[0]
+    A = np.zeros(Kf.shape[:2])
+    for g in range(qf.shape[0]):
+        A[g // G] += softmax(Kf[g // G] @ qf[g]) / G
+    return A
+
+
+def _mass_interleaved(q, K):
+    # wrong GQA convention: q head g reads KV head g % Hkv
+    Hkv = K.shape[0]
+    G = q.shape[0] // Hkv
+    perm = np.array([h + Hkv * g for h in range(Hkv) for g in range(G)])
+    return REAL.decode_attention_mass(q[perm], K)
+
+
 @pytest.mark.parametrize("check, mutant", [
     (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
     (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
@@ -644,6 +735,10 @@ def _boundary_stats_on_raw(A_layers, step_id, prot, valid, gain, red, obs_sim, r
     (check_step_statistics_table, _mutant(step_statistics=_stats_max_over_all)),
     (check_step_statistics_table, _mutant(step_statistics=_stats_count_protected)),
     (check_boundary_step_statistics, _mutant(stepkv_boundary=_boundary_stats_on_raw)),
+    (check_mass_sums, _mutant(decode_attention_mass=_mass_sum_over_group)),
+    (check_mass_two_key_analytic, _mutant(decode_attention_mass=_mass_no_scale)),
+    (check_mass_bruteforce, _mutant(decode_attention_mass=_mass_no_scale)),
+    (check_mass_gqa, _mutant(decode_attention_mass=_mass_interleaved)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

@@ -336,6 +336,30 @@ STEPKV_API stepkv_status_t stepkv_decode_h2o(int32_t n_layers, const void* const
                                   float* const* out, float* const* mass, int64_t mass_head_stride,
                                   void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
 
+/* ---------------------------------------------------------------------------------------------
+ * Step signals from evidence cues (Sec. 4.1: observation validity, evidence gain, action redundancy of
+ * Eq. 2 and the similarity that drives Eq. 3).  Every field of a step (0 Thought, 1 Action,
+ * 2 Observation) is given as up to STEPKV_MAX_CUES evidence cues: distinct 32-bit ids in strictly
+ * increasing order (how cues are drawn from text is the caller's; the paper caps them at 64 per field).
+ * sim(a, b) = |A n B| / |A u B| over cue sets (0 when both are empty); a concatenation of fields is the
+ * union of their cues.  For every target step k in [k0, n_steps):
+ *   gain[k] = 1 - max_{u<k} sim(Th_k || Obs_k, Th_u || Obs_u)     (1 for the first step)
+ *   red[k]  = max_{u<k} sim(Act_k, Act_u)                          (0 for the first step)
+ * and, when obs_sim is not NULL, for the newest step t = n_steps - 1:
+ *   obs_sim[k] = sim(Obs_t, Obs_k) for k < t, obs_sim[t] = 0      (the input of Eq. 3)
+ *  cues     [n_steps][3][STEPKV_MAX_CUES] uint32 (entries past a field's count are ignored)
+ *  n_cues   [n_steps][3] int32 in [0, STEPKV_MAX_CUES]
+ *  gain/red [n_steps] float32 or NULL (only entries k >= k0 are written); obs_sim [n_steps] or NULL.
+ *  A count outside [0, 64] or a list that is not strictly increasing sets STEPKV_EDATA and the values
+ *  that depend on it are not written.  1 <= n_steps <= 65535, 0 <= k0 <= n_steps.
+ *  The outputs can be passed straight to stepkv_steps_t (valid stays the caller's: an empty or
+ *  error-returning Observation is unusable).
+ */
+#define STEPKV_MAX_CUES 64
+STEPKV_API stepkv_status_t stepkv_step_signals(const uint32_t* cues, const int32_t* n_cues, int32_t n_steps,
+                                               int32_t k0, float* gain, float* red, float* obs_sim,
+                                               int32_t* dev_status, void* stream);
+
 /* Failure-detection self-test (no counterpart in the paper).  Runs the saliency kernel of stepkv_score
  * on the same arguments, except that the wait of its second pass (for every CTA's first-pass flag)
  * looks for a value no CTA ever publishes, so every CTA's wait runs out after wait_limit_ns

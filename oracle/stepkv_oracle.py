@@ -135,6 +135,36 @@ def reuse_update(c_prev, obs_sim, eta: float) -> np.ndarray:
     return c
 
 
+def cue_similarity(a, b) -> float:
+    """sim(a, b) of Sec. 4.1, "overlap-based textual similarity" over evidence cues (at most 64 per field,
+    Table H).  Reading: the overlap of the two cue sets relative to their union, |A n B| / |A u B|, and 0
+    when both are empty."""
+    A, B = set(int(x) for x in a), set(int(x) for x in b)
+    union = len(A | B)
+    return len(A & B) / union if union else 0.0
+
+
+def step_signals(th, act, obs, k0=None):
+    """Sec. 4.1 field signals from per-step cue sets th[k], act[k], obs[k] (k = 0 .. t, t the newest step):
+      gain_k = 1 - max_{u<k} sim(Th_k || Obs_k, Th_u || Obs_u)  (gain = 1 for the first step)
+      red_k  = max_{u<k} sim(Act_k, Act_u)                       (red = 0 for the first step)
+    for k >= k0 (default: the newest step only), and Eq. 3's obs_sim[k] = sim(Obs_t, Obs_k) for k < t
+    (obs_sim[t] = 0).  The concatenation of two fields is the union of their cues (reading)."""
+    n = len(obs)
+    t = n - 1
+    k0 = t if k0 is None else k0
+    gain = np.full(n, np.nan)
+    red = np.full(n, np.nan)
+    for k in range(k0, n):
+        cur = set(th[k]) | set(obs[k])
+        gain[k] = 1.0 - max([cue_similarity(cur, set(th[u]) | set(obs[u])) for u in range(k)], default=0.0)
+        red[k] = max([cue_similarity(act[k], act[u]) for u in range(k)], default=0.0)
+    obs_sim = np.zeros(n)
+    for k in range(t):
+        obs_sim[k] = cue_similarity(obs[t], obs[k])
+    return gain, red, obs_sim
+
+
 def clip(z, a, b):
     """clip(z, a, b) truncates z to [a, b] (Sec. 4.1)."""
     return np.minimum(np.maximum(z, a), b)

@@ -91,6 +91,7 @@ SIGNATURES = {
                               _VP, _VP, _VP, _VP]),
     "stepkv_decode_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
     "stepkv_decode_h2o_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
+    "stepkv_step_signals": (_I32, [_VP, _VP, _I32, _I32, _VP, _VP, _VP, _VP, _VP]),
     "stepkv_decode_h2o": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _I64, _VP,
                                  _SZ, _VP, _VP]),
     "stepkv_decode": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _SZ, _VP,
@@ -468,6 +469,33 @@ def stepkv_decode_h2o(q: Sequence, K: Sequence, V: Sequence, n, mass: Sequence, 
                                  _stream_handle(stream))
     _check(code, "stepkv_decode_h2o")
     return out
+
+
+def stepkv_step_signals(cues, n_cues, k0: Optional[int] = None, gain=None, red=None, obs_sim=None, status=None,
+                        stream=None):
+    """Sec. 4.1 field signals from evidence cues: cues [n_steps, 3, 64] (int32 or uint32 bits of the sorted cue
+    ids of Thought / Action / Observation), n_cues [n_steps, 3] int32.  Writes gain/red for steps >= k0 (default
+    the newest) and obs_sim of the newest step against every earlier one; returns (gain, red, obs_sim)."""
+    torch = _torch()
+    lib = load_library()
+    if cues.dim() != 3 or cues.shape[1] != 3 or cues.shape[2] != 64 or cues.element_size() != 4:
+        raise ValueError("cues must be [n_steps, 3, 64] 32-bit")
+    _need(n_cues, torch.int32, "n_cues", 2)
+    if not cues.is_contiguous() or not n_cues.is_contiguous() or n_cues.shape != cues.shape[:2]:
+        raise ValueError("cues and n_cues must be contiguous, n_cues [n_steps, 3]")
+    n = cues.shape[0]
+    k0 = n - 1 if k0 is None else k0
+    dev = cues.device
+    gain = gain if gain is not None else torch.full((n,), float("nan"), dtype=torch.float32, device=dev)
+    red = red if red is not None else torch.full((n,), float("nan"), dtype=torch.float32, device=dev)
+    obs_sim = obs_sim if obs_sim is not None else torch.empty(n, dtype=torch.float32, device=dev)
+    for t, nm in ((gain, "gain"), (red, "red"), (obs_sim, "obs_sim")):
+        _need(t, torch.float32, nm, 1)
+    status = status if status is not None else new_status(dev)
+    code = lib.stepkv_step_signals(cues.data_ptr(), n_cues.data_ptr(), n, k0, gain.data_ptr(), red.data_ptr(),
+                                   obs_sim.data_ptr(), status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_step_signals")
+    return gain, red, obs_sim
 
 
 # Limits of the fixed scratch compiled into the library (STEPKV_STATIC_SCRATCH_MAX_* in the header).

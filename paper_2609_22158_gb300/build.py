@@ -26,7 +26,7 @@ ROOT = os.path.dirname(PKG_DIR)
 BUILD_DIR = os.path.join(PKG_DIR, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libstepkv.so")
 
-SOURCES = ["api.cu", "score.cu", "select.cu", "compact.cu", "decode.cu"]
+SOURCES = ["api.cu", "score.cu", "select.cu", "compact.cu", "decode.cu", "signals.cu"]
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
                 "-I" + os.path.join(ROOT, "include"), "--expt-relaxed-constexpr"]

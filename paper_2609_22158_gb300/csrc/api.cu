@@ -375,6 +375,14 @@ stepkv_status_t stepkv_decode(int32_t n_layers, const void* const* q, const void
                     static_cast<cudaStream_t>(stream));
 }
 
+stepkv_status_t stepkv_step_signals(const uint32_t* cues, const int32_t* n_cues, int32_t n_steps, int32_t k0,
+                                    float* gain, float* red, float* obs_sim, int32_t* dev_status, void* stream) {
+  if (!cues || !n_cues || n_steps < 1 || n_steps > 65535 || k0 < 0 || k0 > n_steps) return STEPKV_EINVAL;
+  if (k0 < n_steps && (!gain || !red)) return STEPKV_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(cues) & 3u) || (reinterpret_cast<uintptr_t>(n_cues) & 3u)) return STEPKV_EUNSUPPORTED;
+  return signals_run(cues, n_cues, n_steps, k0, gain, red, obs_sim, dev_status, static_cast<cudaStream_t>(stream));
+}
+
 size_t stepkv_decode_h2o_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, int32_t d, int32_t n_cap) {
   if (stepkv_decode_workspace_size(n_layers, Hkv, Hq, d, n_cap) == 0) return 0;
   return decode_mass_ws_bytes(std::min(n_layers, kMaxDecodeLayers), Hkv, Hq, d, n_cap);

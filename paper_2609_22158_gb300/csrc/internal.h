@@ -90,6 +90,10 @@ stepkv_status_t decode_run(int n_layers, const void* const* q, const void* const
                            float* const* out, void* ws, int32_t* status, cudaStream_t stream,
                            float* const* mass = nullptr, int64_t mass_stride = 0);
 
+// ---- step signals from evidence cues (signals.cu)
+stepkv_status_t signals_run(const uint32_t* cues, const int32_t* n_cues, int n_steps, int k0, float* gain, float* red,
+                            float* obs_sim, int32_t* status, cudaStream_t stream);
+
 // ---- score (score.cu)
 int score_row_groups(int Hkv, int Hq, int W);
 size_t score_partial_bytes(int n_layers, int Hkv, int Hq, int W, int n_traj = 1);

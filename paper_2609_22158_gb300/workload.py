@@ -447,3 +447,29 @@ def decode_queries(seed: int, n_layers: int, Hq: int, d: int, n: int) -> np.ndar
     """Single-token decode queries [n, n_layers, Hq, d] bf16 bits."""
     g = _rng(seed, _K_QUERIES, 77_777)
     return f32_to_bf16_bits(g.standard_normal((n, n_layers, Hq, d), dtype=np.float32))
+
+
+def synthetic_cues(seed: int, n_steps: int, vocab: int = 4000, reuse: float = 0.3, repeat_action: float = 0.25):
+    """Evidence cues of every step's fields (Thought, Action, Observation) for the Sec. 4.1 signals: each
+    field draws 8-64 distinct ids from a vocabulary; a fraction ``reuse`` of an Observation's and Thought's
+    cues repeats cues of a random earlier Observation (later steps reusing earlier evidence), and with
+    probability ``repeat_action`` an Action repeats an earlier Action's cues (a redundant tool call).
+    Returns [(th, act, obs)] of sorted uint32 arrays."""
+    g = _rng(seed, _K_SIGNALS, 123_456)
+    steps = []
+    for k in range(n_steps):
+        fields = []
+        for f in range(3):
+            n = int(g.integers(8, 65))
+            if f == 1 and k > 0 and g.random() < repeat_action:
+                fields.append(steps[int(g.integers(0, k))][1].copy())
+                continue
+            own = g.integers(0, vocab, n)
+            if f != 1 and k > 0:
+                src = steps[int(g.integers(0, k))][2]
+                m = min(len(src), int(reuse * n))
+                if m:
+                    own[:m] = g.choice(src, m, replace=False)
+            fields.append(np.unique(own.astype(np.uint32))[:64])
+        steps.append(tuple(fields))
+    return steps

@@ -459,6 +459,57 @@ def test_decode_mass_pins(chk):
     chk(REAL)
 
 
+# ------------------------------------------------------------------ step signals from evidence cues (Sec. 4.1)
+def _signal_table():
+    rows = _load_table("step_signals.txt")
+    parse = lambda x: [] if x == "-" else [int(v) for v in x.split(",")]
+    steps = [r[1:] for r in rows if r[0] == "step"]
+    sig = np.array([[float(v) for v in r[2:]] for r in rows if r[0] == "sig"])
+    return [parse(r[1]) for r in steps], [parse(r[2]) for r in steps], [parse(r[3]) for r in steps], sig
+
+
+def check_step_signals_table(O):
+    th, act, obs, sig = _signal_table()
+    gain, red, obs_sim = O.step_signals(th, act, obs, k0=0)
+    assert np.allclose(gain, sig[:, 0], rtol=0, atol=1e-15), gain
+    assert np.allclose(red, sig[:, 1], rtol=0, atol=1e-15), red
+    assert np.allclose(obs_sim, sig[:, 2], rtol=0, atol=1e-15), obs_sim
+
+
+def check_cue_similarity_cases(O):
+    """Identical non-empty sets give 1, disjoint or empty sets 0, the value is symmetric, and it equals
+    a count written out with loops on random small sets."""
+    assert O.cue_similarity([3, 5, 9], [3, 5, 9]) == 1.0
+    assert O.cue_similarity([3, 5], [4, 6]) == 0.0
+    assert O.cue_similarity([], []) == 0.0 and O.cue_similarity([1], []) == 0.0
+    rng = np.random.default_rng(9)
+    for _ in range(50):
+        a = sorted(set(rng.integers(0, 30, rng.integers(0, 12)).tolist()))
+        b = sorted(set(rng.integers(0, 30, rng.integers(0, 12)).tolist()))
+        inter = sum(1 for x in a if x in b)
+        union = len(a) + sum(1 for x in b if x not in a)
+        ref = inter / union if union else 0.0
+        assert O.cue_similarity(a, b) == ref and O.cue_similarity(b, a) == ref
+
+
+def test_step_signals_table():
+    check_step_signals_table(REAL)
+
+
+def test_cue_similarity_cases():
+    check_cue_similarity_cases(REAL)
+
+
+def test_step_signals_ranges():
+    rng = np.random.default_rng(10)
+    draw = lambda: sorted(set(rng.integers(0, 200, rng.integers(0, 64)).tolist()))
+    th, act, obs = [draw() for _ in range(30)], [draw() for _ in range(30)], [draw() for _ in range(30)]
+    gain, red, obs_sim = REAL.step_signals(th, act, obs, k0=0)
+    assert gain[0] == 1.0 and red[0] == 0.0 and obs_sim[-1] == 0.0
+    assert ((gain >= 0) & (gain <= 1)).all() and ((red >= 0) & (red <= 1)).all()
+    assert ((obs_sim >= 0) & (obs_sim <= 1)).all()
+
+
 # ------------------------------------------------------------------ end-to-end invariants
 def test_boundary_invariants_tiny():
     tr = wl.tiny(0)
@@ -716,6 +767,37 @@ def _mass_interleaved(q, K):
     return REAL.decode_attention_mass(q[perm], K)
 
 
+def _sim_dice(a, b):
+    A, B = set(a), set(b)
+    return 2 * len(A & B) / (len(A) + len(B)) if (A or B) else 0.0
+
+
+def _signals_with(sim):
+    def f(th, act, obs, k0=None):
+        saved = REAL.cue_similarity
+        REAL.cue_similarity = sim
+        try:
+            return saved.__globals__["step_signals"](th, act, obs, k0)
+        finally:
+            REAL.cue_similarity = saved
+    return f
+
+
+def _signals_mean_redundancy(th, act, obs, k0=None):
+    gain, red, obs_sim = REAL.step_signals(th, act, obs, k0)
+    n = len(obs)
+    for k in range(0 if k0 is None else k0, n):
+        red[k] = np.mean([REAL.cue_similarity(act[k], act[u]) for u in range(k)]) if k else 0.0
+    return gain, red, obs_sim
+
+
+def _signals_obs_only_gain(th, act, obs, k0=None):
+    gain, red, obs_sim = REAL.step_signals(th, act, obs, k0)
+    for k in range(0 if k0 is None else k0, len(obs)):
+        gain[k] = 1.0 - max([REAL.cue_similarity(obs[k], obs[u]) for u in range(k)], default=0.0)
+    return gain, red, obs_sim
+
+
 @pytest.mark.parametrize("check, mutant", [
     (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
     (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
@@ -739,6 +821,10 @@ def _mass_interleaved(q, K):
     (check_mass_two_key_analytic, _mutant(decode_attention_mass=_mass_no_scale)),
     (check_mass_bruteforce, _mutant(decode_attention_mass=_mass_no_scale)),
     (check_mass_gqa, _mutant(decode_attention_mass=_mass_interleaved)),
+    (check_cue_similarity_cases, _mutant(cue_similarity=_sim_dice)),
+    (check_step_signals_table, _mutant(step_signals=_signals_with(_sim_dice))),
+    (check_step_signals_table, _mutant(step_signals=_signals_mean_redundancy)),
+    (check_step_signals_table, _mutant(step_signals=_signals_obs_only_gain)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

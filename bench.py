@@ -47,11 +47,11 @@ UNIT = "tokens/s"
 # 152 SMs at 1.95 GHz); the peak below uses the maximum SM clock.
 MUFU_PER_CLK_SM = 32
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch from single-pass, full-size ncu captures of the
-# current kernels (profiles/compact_kernel_llama8b_32k.md, profiles/score_kernel_llama8b_32k.md):
+# dram__bytes_read.sum + dram__bytes_write.sum per launch from one single-pass, full-size ncu capture of the
+# current kernels on the 32K workload (profiles/launches_llama8b_32k.md, steady-state launches):
 # {config: {kernel: bytes}}.  A kernel absent here reports traffic null.
 NCU_TRAFFIC = {
-    2: {"compact_kernel": 438.94e6 + 388.77e6},
+    2: {"score_kernel": 319.0e6 + 1.4e6, "select_kernel": 0.5e6, "compact_kernel": 438.9e6 + 388.1e6},
 }
 
 

@@ -67,9 +67,14 @@ def _peaks():
 
 
 # ---------------------------------------------------------------------------------- workloads
-def make_trajs(cfg: int, seed=None, window: int = 2048):
-    """The trajectories of one bench configuration (config 5 is the incremental loop: see run_incremental)."""
+def make_trajs(cfg: int, seed=None, window: int = 2048, layers=None):
+    """The trajectories of one bench configuration (config 5 is the incremental loop: see run_incremental).
+    ``layers`` replaces the model's layer count (configs 2 and 4): the saliency work, which reads only the
+    last 3 layers, is unchanged, and the compaction covers fewer layers (small profiling captures)."""
     from paper_2609_22158_gb300 import workload as wl
+    if layers is not None and cfg in (2, 4):
+        return [wl.llama8b_32k(seed=1 if seed is None else seed, L=layers) if cfg == 2 else
+                wl.qwen32b_64k(seed=3 if seed is None else seed, L=layers)]
     if cfg == 6:
         return [wl.observation_prefill("llama8b_32k", window, seed)]
     if cfg == 7:
@@ -700,7 +705,8 @@ def run_ours(args):
     stream = torch.cuda.current_stream(dev)
     flush = torch.empty(512 * 1024 * 1024, dtype=torch.uint8, device=dev)
     params = B.Params()
-    trs = make_trajs(args.config, None if world == 1 else MR.rank_seed(args.config, rank), window=args.window)
+    trs = make_trajs(args.config, None if world == 1 else MR.rank_seed(args.config, rank), window=args.window,
+                     layers=args.layers)
     status = B.new_status(dev)
     dts = []
     for i, tr in enumerate(trs):
@@ -974,6 +980,8 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--config", type=int, choices=[1, 2, 3, 4, 5, 6, 7], default=2)
     ap.add_argument("--window", type=int, default=2048, help="observation length for configs 6 and 7")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="model layers for configs 2 and 4 (profiling captures; the line is then not the headline)")
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)

@@ -389,6 +389,18 @@ STEPKV_API stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_
                                 const stepkv_params_t* params, void* ws, size_t ws_bytes,
                                 int32_t* dev_status, void* stream);
 
+/* ---------------------------------------------------------------------------------------------
+ * Stage timing of the fused pass (profiling; the paper has no counterpart).  Sets, for the calling
+ * thread, three caller-owned CUDA events (cudaEvent_t passed as void*, NULL = not recorded) that every
+ * later stepkv_compress call of this thread records on its stream: `before` ahead of its first launch,
+ * `after_select` between the selection and the compaction launches, `after` behind its last launch.
+ * cudaEventElapsedTime between them gives the saliency + selection time and the compaction time of a
+ * pass without changing its launches (the compaction follows the selection in plain stream order; no
+ * event separates the saliency and selection kernels, which overlap by programmatic dependent
+ * launch).  Call with three NULLs to stop.  The events must outlive the calls that record them.
+ */
+STEPKV_API void stepkv_set_stage_events(void* before, void* after_select, void* after);
+
 #ifdef __cplusplus
 }
 #endif

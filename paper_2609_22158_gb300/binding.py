@@ -92,6 +92,7 @@ SIGNATURES = {
     "stepkv_decode_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
     "stepkv_decode_h2o_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
     "stepkv_step_signals": (_I32, [_VP, _VP, _I32, _I32, _VP, _VP, _VP, _VP, _VP]),
+    "stepkv_set_stage_events": (None, [_VP, _VP, _VP]),
     "stepkv_decode_h2o": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _I64, _VP,
                                  _SZ, _VP, _VP]),
     "stepkv_decode": (_I32, [_I32, _VP, _VP, _VP, _I64, _I32, _I32, _I32, _VP, _I32, _I32, _VP, _VP, _SZ, _VP,
@@ -496,6 +497,14 @@ def stepkv_step_signals(cues, n_cues, k0: Optional[int] = None, gain=None, red=N
                                    obs_sim.data_ptr(), status.data_ptr(), _stream_handle(stream))
     _check(code, "stepkv_step_signals")
     return gain, red, obs_sim
+
+
+def set_stage_events(before=None, after_select=None, after=None):
+    """Events (torch.cuda.Event, created with enable_timing) that later stepkv_compress calls of this thread
+    record before their first launch, between selection and compaction, and after their last launch;
+    no arguments stop the recording."""
+    h = lambda e: None if e is None else ctypes.c_void_p(e.cuda_event)
+    load_library().stepkv_set_stage_events(h(before), h(after_select), h(after))
 
 
 # Limits of the fixed scratch compiled into the library (STEPKV_STATIC_SCRATCH_MAX_* in the header).

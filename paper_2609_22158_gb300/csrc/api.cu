@@ -16,6 +16,12 @@ namespace stepkv {
 
 static thread_local char g_last_error[256] = {0};
 
+// Caller-owned CUDA events stepkv_compress records on its stream (stepkv_set_stage_events), per thread.
+struct StageEvents {
+  cudaEvent_t e[3];
+};
+static thread_local StageEvents t_stage_events = {{nullptr, nullptr, nullptr}};
+
 void set_last_cuda_error(cudaError_t e) {
   snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e), cudaGetErrorString(e));
 }
@@ -536,6 +542,12 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
                           *params, p.budget, p.sel, sel_ws, dev_status};
   }
+  // optional stage timing (profiling): caller-owned events recorded on the stream of this call
+  const StageEvents ev = t_stage_events;
+  if (ev.e[0]) {
+    const cudaError_t er = cudaEventRecord(ev.e[0], s);
+    if (er != cudaSuccess) { set_last_cuda_error(er); return STEPKV_ECUDA; }
+  }
   // stage 1: one cooperative launch per saliency batch
   for (const SalBatch& b : batches) {
     const stepkv_problem_t& p = probs[b.first];
@@ -547,6 +559,10 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   // stages 2-4 for all trajectories in one launch (one cluster per trajectory)
   stepkv_status_t st = select_run_batch(specs.data(), n_traj, s);
   if (st != STEPKV_OK) return st;
+  if (ev.e[1]) {
+    const cudaError_t er = cudaEventRecord(ev.e[1], s);  // the compaction is launched plainly after it
+    if (er != cudaSuccess) { set_last_cuda_error(er); return STEPKV_ECUDA; }
+  }
   // stage 5: in place by hole filling where the outputs are the inputs (one plan and one move launch per
   // trajectory), the rest out of place, sharing launches
   std::vector<CompactSpec> outs;
@@ -567,8 +583,20 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
                                p.sel.n_kept, p.sel.kept_cap, c.K_out.data(), c.V_out.data(), p.out_head_stride,
                                p.step_id, p.pos_in, p.step_id_out, p.pos_out});
   }
-  if (!outs.empty()) return compact_run_batch(outs.data(), (int)outs.size(), dev_status, s);
+  if (!outs.empty()) {
+    st = compact_run_batch(outs.data(), (int)outs.size(), dev_status, s);
+    if (st != STEPKV_OK) return st;
+  }
+  if (ev.e[2]) {
+    const cudaError_t er = cudaEventRecord(ev.e[2], s);
+    if (er != cudaSuccess) { set_last_cuda_error(er); return STEPKV_ECUDA; }
+  }
   return STEPKV_OK;
+}
+
+void stepkv_set_stage_events(void* before, void* after_select, void* after) {
+  t_stage_events = StageEvents{{static_cast<cudaEvent_t>(before), static_cast<cudaEvent_t>(after_select),
+                                static_cast<cudaEvent_t>(after)}};
 }
 
 }  // extern "C"

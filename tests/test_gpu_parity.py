@@ -634,3 +634,30 @@ def test_compress_batched_short_trajectories(B):
         for l in range(tr.shape.L):
             assert np.array_equal(TL.bits_of(g.K_out[l])[:, :n], O.compact_rows(tr.keys(l), gk))
             assert np.array_equal(TL.bits_of(g.V_out[l])[:, :n], O.compact_rows(tr.values(l), gk))
+
+
+def test_compress_stage_events(B):
+    """stepkv_set_stage_events: a pass records the caller's three events around its stages and its
+    results equal those of a pass without them; clearing the events stops the recording."""
+    import torch
+    tr = wl.custom(95, L=4, Hq=16, Hkv=4, d=128, T=6000, W=64, n_steps=10, budget=wl.Budget.ratio(1, 10))
+    g1, g2 = TL.GpuTraj(tr), TL.GpuTraj(tr)
+    p1, p2 = g1.problem(), g2.problem()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    for e in ev:
+        e.record()
+    torch.cuda.synchronize()
+    B.set_stage_events(*ev)
+    B.stepkv_compress([p1], B.Params())
+    B.set_stage_events()
+    after = torch.cuda.Event(enable_timing=True)
+    B.stepkv_compress([p2], B.Params())
+    after.record()
+    torch.cuda.synchronize()
+    t_sal_sel, t_compact = ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])
+    assert t_sal_sel > 0 and t_compact > 0
+    assert ev[2].elapsed_time(after) > 0  # the second pass recorded nothing into the events
+    n = int(g1.out.n_kept.item())
+    assert torch.equal(g1.out.kept_idx[:n], g2.out.kept_idx[:n])
+    for l in range(tr.shape.L):
+        assert torch.equal(g1.K_out[l][:, :n], g2.K_out[l][:, :n])

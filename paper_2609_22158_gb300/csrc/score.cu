@@ -25,6 +25,7 @@
 #include <chrono>
 
 #include "common.cuh"
+#include "fastdiv.h"
 #include "internal.h"
 
 namespace stepkv {
@@ -48,12 +49,17 @@ struct ScoreGeom {
   int n_tiles;       // ceil(T / 128)
   float c;           // log2(e) / sqrt(d)
   float inv_G;
+  // the divisors of the per-tile bookkeeping, as multiply-and-shift dividers
+  FastDiv rg_div;    // n_rg
+  FastDiv hkv_div;   // Hkv
+  FastDiv rph_div;   // rph
 };
 
 // One trajectory of a batched launch: its items are [item_off, item_off + units_per * n_tiles).
 struct ScoreTraj {
   int T;
   int n_tiles;                 // ceil(T / 128)
+  FastDiv nt_div;              // n_tiles
   int item_off;
   unsigned long long* t_acc;   // pass 2: per-token fixed-point sum (when the launch accumulates)
 };
@@ -69,6 +75,8 @@ struct ScoreLaunch {
   int units_per;      // units per trajectory = n_layers x Hkv x n_rg
   int n_items;        // items of all trajectories
   int tpc;            // tiles per CTA (contiguous range)
+  FastDiv tpc_div;    // tpc
+  FastDiv units_div;  // units_per
   float2* part;       // pass-1 partials: slot (unit + cta) x 256 rows
   float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when not accumulating)
   int64_t out_stride;
@@ -101,9 +109,10 @@ __host__ __device__ inline RowGroup row_group(const ScoreGeom& g, int rg) {
     r.blk_rows = g.W_pad;
     r.w0 = 0;
   } else {
-    r.g_first = rg / g.rph;
+    int w_blk;
+    r.g_first = fdivmod(rg, g.rph_div, w_blk);
     r.n_blk = 1;
-    r.w0 = (rg % g.rph) * kMaxRows;
+    r.w0 = w_blk * kMaxRows;
     r.blk_rows = min(kMaxRows, g.W_pad - r.w0);
   }
   r.rows = r.n_blk * r.blk_rows;
@@ -119,17 +128,16 @@ __device__ __forceinline__ ItemLoc locate(const ScoreLaunch& p, int t) {
   int b = 0;
   while (b + 1 < p.n_traj && p.traj[b + 1].item_off <= t) ++b;
   const int local = t - p.traj[b].item_off;
-  const int nt = p.traj[b].n_tiles;
   ItemLoc r;
   r.b = b;
-  r.ul = local / nt;
-  r.tile = local - r.ul * nt;
+  r.ul = fdivmod(local, p.traj[b].nt_div, r.tile);
   r.u = b * p.units_per + r.ul;
   return r;
 }
 // First item of global unit u.
 __device__ __forceinline__ int unit_first_item(const ScoreLaunch& p, int u) {
-  const int b = u / p.units_per, ul = u - b * p.units_per;
+  int ul;
+  const int b = fdivmod(u, p.units_div, ul);
   return p.traj[b].item_off + ul * p.traj[b].n_tiles;
 }
 
@@ -396,8 +404,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       auto load_tile = [&](int gt, int st) -> bool {
         const ItemLoc il = locate(p, gt);
         const int u = il.u, tile = il.tile;
-        const int pair = p.pair0 + il.ul / g.n_rg, rg = il.ul % g.n_rg;
-        const int layer = pair / g.Hkv, h = pair - layer * g.Hkv;
+        int rg, h;
+        const int pair = p.pair0 + fdivmod(il.ul, g.rg_div, rg);
+        const int layer = fdivmod(pair, g.hkv_div, h);
         const int map = il.b * p.n_layers + layer;
         if (u != cur) {
           if (cur >= 0) {
@@ -473,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         const ItemLoc il = locate(p, t);
         const int nt = item_tiles(il, t);
         const int u = il.u;
-        const RowGroup r = row_group(g, u % g.n_rg);
+        const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
         if (!(ok = new_unit(u))) break;
         for (int i = 0; i < nt && ok; ++i) {
           const int st = 2 * slot + i;
@@ -507,7 +516,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       // pass 2: S^T = K Q^T, the tile's keys on M, the query rows on N
       for (int k = 0; k < n1 && ok; ++k) {
         const int u = locate(p, t_hi - 1 - k).u;
-        const RowGroup r = row_group(g, u % g.n_rg);
+        const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
         if (!(ok = new_unit(u))) break;
         int b;
         if (!(ok = take_buffer(b))) break;
@@ -596,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           // Every warp flushes every unit the CTA touches (an untouched share flushes m = -inf, Z = 0),
           // so each of the unit's partial entries is written.
           if (cur >= 0) flush_partial(cur);
-          const RowGroup r = row_group(g, u % g.n_rg);
+          const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
           two = r.rows > 128;
           // Above 128 rows every item has two halves, query tile mt in buffer (h0 + mt) & 1 (h0 = halves
           // before the item, of fixed parity within the unit), so group g drains tile (g + h0) & 1 of
@@ -679,8 +688,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         if (u != cur) {
           // The CTAs whose pass-1 ranges cover unit u: their partials are combined below.
           const int f0 = unit_first_item(p, u);
-          const int c0 = f0 / p.tpc;
-          const int c1 = (f0 + p.traj[il.b].n_tiles - 1) / p.tpc;
+          const int c0 = fdiv(f0, p.tpc_div);
+          const int c1 = fdiv(f0 + p.traj[il.b].n_tiles - 1, p.tpc_div);
           // Wait until those CTAs have published their pass-1 partials (and, before the first addition,
           // every CTA its zeroed accumulators): the unit starts as soon as its own producers are done.
           if (leader) {
@@ -707,8 +716,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           // Combine the pass-1 partials of unit u into this group's per-row offsets, in contributing-CTA
           // order (the group no longer reads the previous unit's offsets once all its warps arrive).
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
-          r = row_group(g, u % g.n_rg);
+          r = row_group(g, fmodulo(u, g.rg_div));
           const int n_e = r.rows > 128 ? 2 : kPartEntries;  // entries written per row in pass 1
+          const int n_e_log2 = r.rows > 128 ? 1 : 2;
           const int row = (ew & 7) * 32 + lane;             // 256 threads of the group, one row each
           const int w = r.w0 + row % r.blk_rows;
           const bool valid = row < r.rows && w < g.W;
@@ -724,7 +734,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
 #pragma unroll
               for (int t8 = 0; t8 < 16; ++t8) {
                 const int i = i0 + t8;
-                const int ci = c0 + i / n_e, e = i - (i / n_e) * n_e;
+                const int ci = c0 + (i >> n_e_log2), e = i & (n_e - 1);
                 pz[t8] = i < n_ent ? __ldcg(&p.part[((size_t)(u + ci) * kPartEntries + e) * kMaxRows + row])
                                    : make_float2(-INFINITY, 0.f);
               }
@@ -800,7 +810,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           if (!(ok = epi_sync(&epi_bar[grp], eb_phase, abort_flag))) break;
           if (s2 == 0 && j < Tb) {
             const float val = (acc + comb[q * 32 + lk]) * g.inv_G;
-            const int pair = p.pair0 + il.ul / g.n_rg, rg = il.ul % g.n_rg;
+            int rg;
+            const int pair = p.pair0 + fdivmod(il.ul, g.rg_div, rg);
             p.out[(size_t)(pair * g.n_rg + rg) * p.out_stride + j] = val;
           }
         }
@@ -875,6 +886,9 @@ static ScoreGeom make_geom(int Hkv, int Hq, int d, int T, int W) {
   g.n_tiles = (T + kKeyTile - 1) / kKeyTile;
   g.c = (float)(1.4426950408889634 / sqrt((double)d));
   g.inv_G = 1.0f / (float)g.G;
+  g.rg_div = make_fastdiv(g.n_rg);
+  g.hkv_div = make_fastdiv(g.Hkv);
+  g.rph_div = make_fastdiv(g.rph);
   return g;
 }
 
@@ -983,6 +997,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.n_traj = n_traj;
   L.n_layers = n_layers;
   L.units_per = n_layers * Hkv * g.n_rg;
+  L.units_div = make_fastdiv(L.units_per);
   L.part = part;
   L.flags = reinterpret_cast<unsigned long long*>(reinterpret_cast<uint8_t*>(part) +
                                                   score_partial_slots_bytes(n_traj, n_layers, Hkv, Hq, W));
@@ -1004,6 +1019,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
     }
     L.traj[b].T = t.T;
     L.traj[b].n_tiles = (t.T + kKeyTile - 1) / kKeyTile;
+    L.traj[b].nt_div = make_fastdiv(L.traj[b].n_tiles);
     L.traj[b].item_off = items;
     L.traj[b].t_acc = t.t_acc;
     items += L.units_per * L.traj[b].n_tiles;
@@ -1017,6 +1033,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.n_items = items;
   const int grid0 = std::min(grid_cap, items);
   L.tpc = (items + grid0 - 1) / grid0;
+  L.tpc_div = make_fastdiv(L.tpc);
   const int grid = (items + L.tpc - 1) / L.tpc;
   L.token = next_launch_token();
   // Self-test of the failure path: the pass-2 wait looks for a value no CTA ever publishes, so every

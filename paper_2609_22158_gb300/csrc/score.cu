@@ -679,8 +679,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       float* negoff = sNegOff + grp * kMaxRows;  // this group's per-row offsets and causal limits
       int* pw_tab = sPw + grp * kMaxRows;
       float* combf = sComb + grp * (2 * 128);     // rows output: [2 parity][128]
-      for (int k = 0; k < n1 && ok; ++k, ++hh) {
-        if ((hh & 1u) != (uint32_t)grp) continue;
+      // pass-2 item k is half hh + k: this group drains every other item, starting with the first of its parity
+      const int k_first = (int)(((uint32_t)grp - hh) & 1u);
+      for (int k = k_first; k < n1 && ok; k += 2) {
         const int gt = t_hi - 1 - k;
         const ItemLoc il = locate(p, gt);
         const int u = il.u, tile = il.tile;

@@ -80,7 +80,9 @@ __device__ __forceinline__ void merge_state(float& m, float& l, float (&acc)[E],
   m = mn;
 }
 
-template <int D, int G>
+// MASS: the accumulated-attention variant, which also stores every key's logits (a separate
+// instantiation, so the plain decode keeps its register budget).
+template <int D, int G, bool MASS>
 __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __grid_constant__ DecodeArgs a) {
   constexpr int LPK = D / 8;          // lanes per key row
   constexpr int KPS = 32 / LPK;       // keys per warp step
@@ -172,7 +174,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
         }
       }
     }
-    if (a.logits != nullptr && hl == 0) {
+    if (MASS && hl == 0) {
       // every lane of a key row holds the row's logits of all G heads: the first one stores them
 #pragma unroll
       for (int t = 0; t < kDecBlockSteps; ++t) {
@@ -349,10 +351,15 @@ size_t decode_mass_ws_bytes(int n_layers, int Hkv, int Hq, int d, int n_cap) {
 
 template <int D, int G>
 static cudaError_t decode_launch(const DecodeArgs& a, int pairs, cudaStream_t stream) {
-  cudaError_t e = launch_kernel(decode_partial_kernel<D, G>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
+  if (a.logits != nullptr) {
+    cudaError_t e = launch_kernel(decode_partial_kernel<D, G, true>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
+                                  stream, a);
+    if (e != cudaSuccess) return e;
+    return launch_kernel(decode_merge_mass_kernel<D, G>, dim3(pairs), dim3(128), 0, stream, a);
+  }
+  cudaError_t e = launch_kernel(decode_partial_kernel<D, G, false>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
                                 stream, a);
   if (e != cudaSuccess) return e;
-  if (a.logits != nullptr) return launch_kernel(decode_merge_mass_kernel<D, G>, dim3(pairs), dim3(128), 0, stream, a);
   const int items = pairs * G;
   return launch_kernel(decode_merge_kernel<D, G>, dim3((items + 3) / 4), dim3(128), 0, stream, a, items);
 }

@@ -692,13 +692,31 @@ def decode_report(s, dev, stream, flush, status, hbm):
     torch.cuda.synchronize()
     us = d0.elapsed_time(d1) * 1e3 / n_tok
     dbytes = 2 * s.L * s.Hkv * dec_rows * s.d * 2
+    # the same reads with the H2O-style accumulated attention (stepkv_decode_h2o): every key's logits are
+    # stored per head and re-read by the merge, which adds the group-mean softmax into the mass rows
+    mass = [torch.zeros((s.Hkv, dec_rows), dtype=torch.float32, device=dev) for _ in range(s.L)]
+    ws_h = torch.empty(B.load_library().stepkv_decode_h2o_workspace_size(s.L, s.Hkv, s.Hq, s.d, dec_rows) + 512,
+                       dtype=torch.uint8, device=dev)
+    for _ in range(3):
+        B.stepkv_decode_h2o(qd, Kd, Vd, dec_rows, mass, out=outd, ws=ws_h, status=status, stream=stream)
+    flush.fill_(8)
+    torch.cuda.synchronize()
+    d0.record(stream)
+    for _ in range(n_tok):
+        B.stepkv_decode_h2o(qd, Kd, Vd, dec_rows, mass, out=outd, ws=ws_h, status=status, stream=stream)
+    d1.record(stream)
+    torch.cuda.synchronize()
+    us_h = d0.elapsed_time(d1) * 1e3 / n_tok
+    hbytes = dbytes + s.L * dec_rows * (2 * s.Hq * 4 + 2 * s.Hkv * 4)  # + logits written and read, mass RMW
     if int(status.item()) != 0:
         raise RuntimeError(f"device status {int(status.item())} after decode")
     return {"workload": f"decode attention, {n_tok} single-token reads over a compacted cache of {dec_rows} "
                         f"rows x {s.L} layers x {s.Hkv} KV heads (Hq={s.Hq}, d={s.d})",
             "us_per_token": round(us, 2), "algorithmic_bytes_per_token": dbytes,
             "achieved_gbs": round(dbytes / (us * 1e-6) / 1e9, 1),
-            "frac_of_measured_hbm": round(dbytes / (us * 1e-6) / 1e9 / hbm, 4), "launches_per_token": 2}
+            "frac_of_measured_hbm": round(dbytes / (us * 1e-6) / 1e9 / hbm, 4), "launches_per_token": 2,
+            "h2o": {"us_per_token": round(us_h, 2), "algorithmic_bytes_per_token": hbytes,
+                    "frac_of_measured_hbm": round(hbytes / (us_h * 1e-6) / 1e9 / hbm, 4)}}
 
 
 # ---------------------------------------------------------------------------------- ours

@@ -206,6 +206,21 @@ __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
+// L2 eviction-priority hints for small, hot global data that large streams would otherwise push out of
+// L2 (the saliency kernel's per-token fixed-point sums: zeroed, then hit by an atomic per key and KV head).
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ void st_u64_hint(unsigned long long* p, unsigned long long v, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.u64 [%0], %1, %2;" ::"l"(p), "l"(v), "l"(pol) : "memory");
+}
+// atomicAdd without a return value (relaxed, GPU scope), with an L2 cache policy
+__device__ __forceinline__ void red_add_u64_hint(unsigned long long* p, unsigned long long v, uint64_t pol) {
+  asm volatile("red.relaxed.gpu.global.add.L2::cache_hint.u64 [%0], %1, %2;" ::"l"(p), "l"(v), "l"(pol) : "memory");
+}
+
 // Exact fixed-point conversion of a non-negative float: round(x * 2^shift) as uint64, with integer
 // instructions only (the float -> 64-bit conversion instructions run on the slow FP64 pipe).  Requires
 // x * 2^shift < 2^63.  Rounds half away from zero.

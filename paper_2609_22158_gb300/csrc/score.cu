@@ -21,6 +21,7 @@
 #include <math.h>
 
 #include <algorithm>
+#include <vector>
 #include <atomic>
 #include <chrono>
 
@@ -74,8 +75,7 @@ struct ScoreLaunch {
   int pair0;          // first (layer*Hkv + head) pair of this launch (rows output)
   int units_per;      // units per trajectory = n_layers x Hkv x n_rg
   int n_items;        // items of all trajectories
-  int tpc;            // tiles per CTA (contiguous range)
-  FastDiv tpc_div;    // tpc
+  int cta_first[kMaxGrid + 1];  // CTA b owns items [cta_first[b], cta_first[b + 1])
   FastDiv units_div;  // units_per
   float2* part;       // pass-1 partials: slot (unit + cta) x 256 rows
   float* out;         // pass-2 output rows: row (pair*n_rg + rg), stride out_stride (when not accumulating)
@@ -139,6 +139,17 @@ __device__ __forceinline__ int unit_first_item(const ScoreLaunch& p, int u) {
   int ul;
   const int b = fdivmod(u, p.units_div, ul);
   return p.traj[b].item_off + ul * p.traj[b].n_tiles;
+}
+
+// The CTA whose item range holds item t (binary search over the ranges' first items).
+__device__ __forceinline__ int cta_of_item(const ScoreLaunch& p, int t) {
+  int lo = 0, hi = (int)gridDim.x - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.cta_first[mid] <= t) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
 }
 
 // Shared memory of the kernel.
@@ -349,8 +360,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
   const ScoreGeom& g = p.g;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int U = p.n_items;
-  const int t_lo = blockIdx.x * p.tpc;
-  const int t_hi = min(U, t_lo + p.tpc);
+  const int t_lo = p.cta_first[blockIdx.x];
+  const int t_hi = min(U, p.cta_first[blockIdx.x + 1]);
   const int n1 = max(0, t_hi - t_lo);  // tiles of the CTA (each is streamed once per pass)
   // Pass-1 items: two consecutive tiles of one unit where possible, else one.
   auto item_tiles = [&](const ItemLoc& l, int t) {
@@ -693,8 +704,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         if (u != cur) {
           // The CTAs whose pass-1 ranges cover unit u: their partials are combined below.
           const int f0 = unit_first_item(p, u);
-          const int c0 = fdiv(f0, p.tpc_div);
-          const int c1 = fdiv(f0 + p.traj[il.b].n_tiles - 1, p.tpc_div);
+          const int c0 = cta_of_item(p, f0);
+          const int c1 = cta_of_item(p, f0 + p.traj[il.b].n_tiles - 1);
           // Wait until those CTAs have published their pass-1 partials (and, before the first addition,
           // every CTA its zeroed accumulators): the unit starts as soon as its own producers are done.
           if (leader) {
@@ -867,6 +878,55 @@ __global__ void sum_row_groups_kernel(const float* __restrict__ rows, int n_pair
 
 // -------------------------------------------------------------------------------------------------
 // Host side
+// Contiguous item ranges for the persistent grid, balanced by cost rather than by tile count.  A key tile
+// costs 1; a range that switches to another unit costs kUnitSwitchCost more, since the switch stages
+// another Q block (the MMAs wait for it), flushes a pass-1 partial, and in pass 2 combines another
+// unit's partials after another cross-CTA wait.  With equal tile counts the CTAs whose ranges cross a unit
+// boundary finished pass 1 last, and every CTA sharing their units waited for them at the change of pass.
+constexpr int kUnitSwitchCost = 3;
+
+// Greedy split under a per-CTA cost cap: returns the number of ranges (max_ranges + 1 if they do not fit)
+// and, with `first`, their first items (first[ranges] = the item count).
+static int greedy_split(const std::vector<int>& unit_tiles, int cap, int max_ranges, int* first) {
+  int ranges = 0, item = 0, cost = 0;
+  bool open = false;
+  for (const int n : unit_tiles) {
+    int left = n;
+    bool in_unit = false;  // the open range already holds tiles of this unit
+    while (left > 0) {
+      if (open && !in_unit && cost + kUnitSwitchCost + 1 > cap) open = false;  // switch would overflow
+      if (!open || cost >= cap) {
+        if (ranges == max_ranges) return max_ranges + 1;
+        if (first) first[ranges] = item;
+        ++ranges;
+        open = true;
+        cost = 0;
+        in_unit = false;
+      }
+      if (!in_unit && cost > 0) cost += kUnitSwitchCost;
+      in_unit = true;
+      const int take = std::min(left, std::max(1, cap - cost));
+      cost += take;
+      left -= take;
+      item += take;
+    }
+  }
+  if (first) first[ranges] = item;
+  return ranges;
+}
+
+// The smallest cap whose greedy split fits max_ranges CTAs; writes the ranges and returns their count.
+static int split_items(const std::vector<int>& unit_tiles, int items, int max_ranges, int* first) {
+  int lo = std::max(1, (items + max_ranges - 1) / max_ranges);
+  int hi = items + kUnitSwitchCost * (int)unit_tiles.size();
+  while (lo < hi) {
+    const int mid = lo + (hi - lo) / 2;
+    if (greedy_split(unit_tiles, mid, max_ranges, nullptr) <= max_ranges) hi = mid;
+    else lo = mid + 1;
+  }
+  return greedy_split(unit_tiles, lo, max_ranges, first);
+}
+
 static ScoreGeom make_geom(int Hkv, int Hq, int d, int T, int W) {
   ScoreGeom g;
   memset(&g, 0, sizeof(g));
@@ -1036,10 +1096,10 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   // all (trajectory, layer, KV head) pairs in one launch: every CTA gets a contiguous range of items
   L.pair0 = 0;
   L.n_items = items;
-  const int grid0 = std::min(grid_cap, items);
-  L.tpc = (items + grid0 - 1) / grid0;
-  L.tpc_div = make_fastdiv(L.tpc);
-  const int grid = (items + L.tpc - 1) / L.tpc;
+  std::vector<int> unit_tiles;
+  unit_tiles.reserve((size_t)n_traj * L.units_per);
+  for (int b = 0; b < n_traj; ++b) unit_tiles.insert(unit_tiles.end(), L.units_per, L.traj[b].n_tiles);
+  const int grid = split_items(unit_tiles, items, grid_cap, L.cta_first);
   L.token = next_launch_token();
   // Self-test of the failure path: the pass-2 wait looks for a value no CTA ever publishes, so every
   // CTA's wait runs out after selftest_wait_ns and the kernel takes its abort path.

@@ -260,11 +260,13 @@ def test_select_budgets(B, budget):
     TL.check_select_outputs(g, out)
 
 
-@pytest.mark.parametrize("levels", [2, 7, 1000])
+@pytest.mark.parametrize("levels", [2, 7, 150, 200, 1000])
 def test_select_exact_on_shared_fp32_priorities(B, levels):
     """alpha=1, beta=0, no normalisation, one saliency row: the kernel ranks exactly the fp32 values
     it is given, so its retained set must equal the oracle's ranking of the same values bit for bit,
-    ties (few distinct levels) included."""
+    ties (few distinct levels) included.  ~100-130 tokens per level (150 and 200 levels over 20000
+    tokens) put the threshold bin on both sides of the 128 candidates the value-bin path resolves
+    directly; 2 and 7 levels take the radix fallback."""
     import torch
     T = 20000
     tr = wl.custom(9, L=1, Hq=1, Hkv=1, d=64, T=T, W=8, n_steps=12, budget=wl.Budget.ratio(3, 10))

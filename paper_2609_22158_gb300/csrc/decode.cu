@@ -14,10 +14,12 @@
 //
 // Accumulated attention (the H2O-style token saliency, Sec. 4.2: T_i may come from an existing
 // token-level importance estimator): with mass rows given, the partial kernel also stores every key's
-// logits per head, and the merge runs one CTA per (layer, KV head): its warps merge the heads' splits
-// (same order as the plain merge, so the outputs are bit-identical) and record each head's log-sum-exp,
-// then its threads add (1/G) sum_g softmax_j(q_g . k_j / sqrt(d)) to mass[j] for every key (one writer
-// per element and call, fixed order over g: deterministic).
+// logits per head, and the merge runs up to 8 CTAs per (layer, KV head), each over a contiguous share of
+// the keys.  Every CTA merges the heads' (m, l) split states in split order into each head's
+// log-sum-exp (the first CTA also merges the value rows, in the same order as the plain merge, so the
+// outputs are bit-identical).  Then its threads add (1/G) sum_g softmax_j(q_g . k_j / sqrt(d)) to
+// mass[j] for each of its keys: one writer per element and call, a fixed order over g, so the result is
+// deterministic.
 #include <math.h>
 
 #include <algorithm>
@@ -181,8 +183,14 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
         const int j = kb + t * KPS + kslot;
         if (ok[t]) {
           float* dst = a.logits + ((size_t)pair * a.n_cap + j) * G;
+          if constexpr (G % 4 == 0) {
 #pragma unroll
-          for (int g = 0; g < G; ++g) dst[g] = s[t][g];
+            for (int g = 0; g < G; g += 4)
+              *reinterpret_cast<float4*>(dst + g) = make_float4(s[t][g], s[t][g + 1], s[t][g + 2], s[t][g + 3]);
+          } else {
+#pragma unroll
+            for (int g = 0; g < G; ++g) dst[g] = s[t][g];
+          }
         }
       }
     }
@@ -297,31 +305,43 @@ __global__ void __launch_bounds__(128) decode_merge_kernel(const __grid_constant
 // decode_merge_kernel does (bit-identical outputs) and keeps each head's log-sum-exp; then every thread adds
 // the group-mean softmax mass of its keys to the pair's mass row.
 template <int D, int G>
-__global__ void __launch_bounds__(128) decode_merge_mass_kernel(const __grid_constant__ DecodeArgs a) {
+__global__ void __launch_bounds__(128) decode_merge_mass_kernel(const __grid_constant__ DecodeArgs a, int chunks) {
   constexpr int PER = D / 32;
   __shared__ float s_lse[G];
   pdl_wait();
   pdl_launch_dependents();
-  const int pair = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int pair = blockIdx.x / chunks, chunk = blockIdx.x - pair * chunks;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int layer = pair / a.Hkv, h = pair - layer * a.Hkv;
   const int n = max(0, min(decode_n(a), a.n_cap));
   const int used = max(0, min(a.n_splits, (n + kDecSplitKeys - 1) / kDecSplitKeys));
   for (int g = warp; g < G; g += 4) {
-    float mm = -INFINITY, ll = 0.f, aa[PER];
+    if (chunk == 0) {
+      // the pair's outputs: the splits merged in order, as decode_merge_kernel
+      float mm = -INFINITY, ll = 0.f, aa[PER];
 #pragma unroll
-    for (int e = 0; e < PER; ++e) aa[e] = 0.f;
-    for (int sp = 0; sp < used; ++sp) {
-      const float* src = a.part + ((size_t)(pair * a.n_splits + sp) * G + g) * (D + 4);
-      float a2[PER];
+      for (int e = 0; e < PER; ++e) aa[e] = 0.f;
+      for (int sp = 0; sp < used; ++sp) {
+        const float* src = a.part + ((size_t)(pair * a.n_splits + sp) * G + g) * (D + 4);
+        float a2[PER];
 #pragma unroll
-      for (int e = 0; e < PER; ++e) a2[e] = __ldcg(src + 4 + lane * PER + e);
-      merge_state<PER>(mm, ll, aa, __ldcg(src), __ldcg(src + 1), a2);
+        for (int e = 0; e < PER; ++e) a2[e] = __ldcg(src + 4 + lane * PER + e);
+        merge_state<PER>(mm, ll, aa, __ldcg(src), __ldcg(src + 1), a2);
+      }
+      const float inv = ll > 0.f ? 1.f / ll : 0.f;
+      float* o = a.out[layer] + (size_t)(h * G + g) * D + lane * PER;
+#pragma unroll
+      for (int e = 0; e < PER; ++e) o[e] = aa[e] * inv;
+      if (lane == 0) s_lse[g] = ll > 0.f ? mm + __log2f(ll) : INFINITY;
+    } else if (lane == 0) {
+      // the same (m, l) merge without the value rows: the same log-sum-exp in every chunk
+      float mm = -INFINITY, ll = 0.f, none[1] = {0.f};
+      for (int sp = 0; sp < used; ++sp) {
+        const float* src = a.part + ((size_t)(pair * a.n_splits + sp) * G + g) * (D + 4);
+        merge_state<1>(mm, ll, none, __ldcg(src), __ldcg(src + 1), none);
+      }
+      s_lse[g] = ll > 0.f ? mm + __log2f(ll) : INFINITY;
     }
-    const float inv = ll > 0.f ? 1.f / ll : 0.f;
-    float* o = a.out[layer] + (size_t)(h * G + g) * D + lane * PER;
-#pragma unroll
-    for (int e = 0; e < PER; ++e) o[e] = aa[e] * inv;
-    if (lane == 0) s_lse[g] = ll > 0.f ? mm + __log2f(ll) : INFINITY;
   }
   __syncthreads();
   float lse[G];
@@ -330,10 +350,22 @@ __global__ void __launch_bounds__(128) decode_merge_mass_kernel(const __grid_con
   const float inv_G = 1.f / (float)G;
   float* mrow = a.mass[layer] + (size_t)h * a.mass_stride;
   const float* lg = a.logits + (size_t)pair * a.n_cap * G;
-  for (int j = threadIdx.x; j < n; j += 128) {
+  // this chunk's keys (one writer per key: the additions are ordered across calls by the stream)
+  const int per = (n + chunks - 1) / chunks;
+  const int j0 = chunk * per, j1 = min(n, j0 + per);
+  for (int j = j0 + threadIdx.x; j < j1; j += 128) {
     float sum = 0.f;
+    if constexpr (G % 4 == 0) {
 #pragma unroll
-    for (int g = 0; g < G; ++g) sum += ex2_approx(__ldcg(lg + (size_t)j * G + g) - lse[g]);
+      for (int g4 = 0; g4 < G; g4 += 4) {
+        const float4 v = __ldcg(reinterpret_cast<const float4*>(lg + (size_t)j * G + g4));
+        sum += ex2_approx(v.x - lse[g4]) + ex2_approx(v.y - lse[g4 + 1]) + ex2_approx(v.z - lse[g4 + 2]) +
+               ex2_approx(v.w - lse[g4 + 3]);
+      }
+    } else {
+#pragma unroll
+      for (int g = 0; g < G; ++g) sum += ex2_approx(__ldcg(lg + (size_t)j * G + g) - lse[g]);
+    }
     mrow[j] += sum * inv_G;
   }
 }
@@ -355,7 +387,9 @@ static cudaError_t decode_launch(const DecodeArgs& a, int pairs, cudaStream_t st
     cudaError_t e = launch_kernel(decode_partial_kernel<D, G, true>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
                                   stream, a);
     if (e != cudaSuccess) return e;
-    return launch_kernel(decode_merge_mass_kernel<D, G>, dim3(pairs), dim3(128), 0, stream, a);
+    // several CTAs per pair over the keys' mass updates (a pair's ~n keys are too few per SM otherwise)
+    const int chunks = std::max(1, std::min(8, (a.n_cap + 1023) / 1024));
+    return launch_kernel(decode_merge_mass_kernel<D, G>, dim3(pairs * chunks), dim3(128), 0, stream, a, chunks);
   }
   cudaError_t e = launch_kernel(decode_partial_kernel<D, G, false>, dim3(pairs * a.n_splits), dim3(kDecThreads), 0,
                                 stream, a);

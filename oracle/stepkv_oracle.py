@@ -17,7 +17,8 @@ at the function (the readings are listed together in the design notes).
 Precision: all floating point is fp64.  bf16 inputs are widened exactly.
 
 Library primitives used as single steps: ``numpy.matmul`` (the Q.K^T dot
-products), ``numpy.exp``/``numpy.log1p``, ``numpy.lexsort`` (the global ranking).
+products), ``numpy.exp``/``numpy.log1p``, ``numpy.lexsort`` (the global ranking),
+``numpy.lib.stride_tricks.sliding_window_view`` (the pooling windows).
 No blocking, fusion or reordering beyond the definitions.
 
 Pinning status (see tests/test_oracle_pins.py): every function below is pinned
@@ -48,6 +49,8 @@ class Params:
     alpha: float = 0.2    # token-saliency weight (Eq. 5)
     beta: float = 0.8     # step-utility weight (Eq. 5)
     sal_norm: str = "max"  # "max": T_i / max over prunable tokens (appendix, H_i in [0, H_max]); "none"
+    pool: int = 1          # SnapKV-style pooling width k along the token axis (odd; 1 = none)
+    pool_mode: str = "max"  # "max" or "avg" pooling
 
 
 def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
@@ -95,9 +98,27 @@ def window_attention_saliency(K: np.ndarray, Q: np.ndarray, row_chunk: int = 256
     return A
 
 
-def token_saliency(A_layers: Sequence[np.ndarray]) -> np.ndarray:
-    """T_i = mean over (saliency layer, KV head) of A[l, h, i]  (reading: mean pooling)."""
+def pool_tokens(a: np.ndarray, k: int, mode: str = "max") -> np.ndarray:
+    """SnapKV-style pooling of one saliency row along the token axis (Sec. 4.2 names SnapKV as an
+    interchangeable T_i estimator; reading: a 1-D pool of odd width k, stride 1, the window
+    [i - k//2, i + k//2] clipped to [0, T), so padding never enters a maximum or an average).
+    out[i] = max (or mean) of a[j] over the window."""
+    a = np.asarray(a, dtype=np.float64)
+    h = k // 2
+    if h == 0:
+        return a.copy()
+    fill = -np.inf if mode == "max" else np.nan
+    padded = np.concatenate([np.full(h, fill), a, np.full(h, fill)])
+    windows = np.lib.stride_tricks.sliding_window_view(padded, 2 * h + 1)  # [T, k], window i centred on i
+    return windows.max(axis=1) if mode == "max" else np.nanmean(windows, axis=1)
+
+
+def token_saliency(A_layers: Sequence[np.ndarray], pool: int = 1, pool_mode: str = "max") -> np.ndarray:
+    """T_i = mean over (saliency layer, KV head) of A[l, h, i]  (reading: mean pooling); with pool > 1
+    each (layer, KV head) row is first pooled along the token axis (pool_tokens)."""
     A = np.stack([np.asarray(a, dtype=np.float64) for a in A_layers])  # [Ls, Hkv, T]
+    if pool > 1:
+        A = np.stack([[pool_tokens(row, pool, pool_mode) for row in layer] for layer in A])
     return A.mean(axis=(0, 1))
 
 
@@ -268,7 +289,7 @@ def stepkv_boundary(A_layers: Sequence[np.ndarray], step_id: np.ndarray, prot: n
     c = reuse_update(reuse_prev, obs_sim, p.eta)
     S = step_utility(r, c, p)
     # Phase 3
-    T_raw = token_saliency(A_layers)
+    T_raw = token_saliency(A_layers, p.pool, p.pool_mode)
     T_hat = normalise_saliency(T_raw, prunable, p.sal_norm)
     N = int(prunable.sum())
     B = budget_tokens(N, budget_mode, num, den, count)

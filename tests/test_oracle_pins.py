@@ -587,6 +587,65 @@ def test_boundary_step_statistics():
     check_boundary_step_statistics(REAL)
 
 
+# ------------------------------------------------------------------ SnapKV-style pooling (Sec. 4.2)
+def check_pool_table(O):
+    """The hand table of tests/golden/snapkv_pooling.txt."""
+    a = np.array([0.1, 0.5, 0.2, 0.0, 0.9, 0.3])
+    for row in _load_table("snapkv_pooling.txt"):
+        k, mode, exp = int(row[0]), row[1], np.array([float(x) for x in row[2:]])
+        np.testing.assert_allclose(O.pool_tokens(a, k, mode), exp, rtol=0, atol=1e-12)
+
+
+def check_pool_max_library(O):
+    """Max pooling with the window clipped at the ends equals scipy's maximum filter with edge
+    replication (a replicated edge value lies inside the clipped window)."""
+    from scipy.ndimage import maximum_filter1d
+    rng = np.random.default_rng(5)
+    for T, k in ((1, 3), (2, 5), (7, 3), (50, 7), (33, 9)):
+        a = rng.random(T)
+        np.testing.assert_array_equal(O.pool_tokens(a, k, "max"), maximum_filter1d(a, size=k, mode="nearest"))
+
+
+def check_pool_avg_convolution(O):
+    """Average pooling: a k-tap box convolution where the whole window fits, the mean of the in-range
+    values at the ends."""
+    rng = np.random.default_rng(6)
+    T, k = 40, 7
+    h = k // 2
+    a = rng.random(T)
+    out = O.pool_tokens(a, k, "avg")
+    np.testing.assert_allclose(out[h:T - h], np.convolve(a, np.ones(k) / k, mode="valid"), rtol=1e-12)
+    for i in list(range(h)) + list(range(T - h, T)):
+        assert abs(out[i] - a[max(0, i - h):min(T, i + h + 1)].mean()) < 1e-12
+
+
+def check_pool_before_mean(O):
+    """Each (layer, KV head) row is pooled before the mean over rows: for a maximum the two orders
+    differ."""
+    rows = [np.array([[1.0, 0.0, 0.0], [0.0, 0.0, 1.0]])]  # one layer, two KV heads
+    np.testing.assert_allclose(O.token_saliency(rows, 3, "max"), [0.5, 1.0, 0.5])
+    np.testing.assert_allclose(O.token_saliency(rows, 1, "max"), [0.5, 0.0, 0.5])
+
+
+def test_snapkv_pooling_pins():
+    for chk in (check_pool_table, check_pool_max_library, check_pool_avg_convolution, check_pool_before_mean):
+        chk(REAL)
+
+
+def test_boundary_uses_pooling():
+    rng = np.random.default_rng(7)
+    T, n_steps = 60, 4
+    A = [rng.random((2, T)) for _ in range(2)]
+    step_id = np.repeat(np.arange(n_steps), T // n_steps).astype(np.int32)
+    prot = np.zeros(T, dtype=np.uint8)
+    sig = [rng.random(n_steps) for _ in range(4)]
+    p = REAL.Params(pool=5, pool_mode="avg")
+    out = REAL.stepkv_boundary(A, step_id, prot, sig[0] > 0.5, sig[1], sig[2], sig[3], np.zeros(n_steps), p,
+                               "ratio", 1, 4)
+    np.testing.assert_allclose(out["T"], REAL.token_saliency(A, 5, "avg"))
+    assert not np.allclose(out["T"], REAL.token_saliency(A))
+
+
 # ------------------------------------------------------------------ planted mistakes
 def _mutant(**overrides):
     ns = types.SimpleNamespace(**{k: getattr(REAL, k) for k in dir(REAL) if not k.startswith("__")})
@@ -798,6 +857,26 @@ def _signals_obs_only_gain(th, act, obs, k0=None):
     return gain, red, obs_sim
 
 
+def _pool_window_shifted(a, k, mode="max"):
+    # window [i - k//2 + 1, i + k//2 + 1]: off by one to the right
+    b = np.concatenate([np.asarray(a, dtype=np.float64)[1:], [-np.inf if mode == "max" else np.nan]])
+    return REAL.pool_tokens(b, k, mode)
+
+
+def _pool_avg_counts_padding(a, k, mode="max"):
+    out = REAL.pool_tokens(a, k, mode)
+    if mode != "avg":
+        return out
+    a = np.asarray(a, dtype=np.float64)
+    padded = np.concatenate([np.zeros(k // 2), a, np.zeros(k // 2)])
+    return np.convolve(padded, np.ones(k) / k, mode="valid")
+
+
+def _token_saliency_pool_after_mean(A_layers, pool=1, pool_mode="max"):
+    T = REAL.token_saliency(A_layers)
+    return REAL.pool_tokens(T, pool, pool_mode) if pool > 1 else T
+
+
 @pytest.mark.parametrize("check, mutant", [
     (check_gqa_grouping, _mutant(window_attention_saliency=_sal_interleaved_groups)),
     (check_zero_keys_closed_form, _mutant(window_attention_saliency=_sal_no_causal)),
@@ -825,6 +904,11 @@ def _signals_obs_only_gain(th, act, obs, k0=None):
     (check_step_signals_table, _mutant(step_signals=_signals_with(_sim_dice))),
     (check_step_signals_table, _mutant(step_signals=_signals_mean_redundancy)),
     (check_step_signals_table, _mutant(step_signals=_signals_obs_only_gain)),
+    (check_pool_table, _mutant(pool_tokens=_pool_window_shifted)),
+    (check_pool_max_library, _mutant(pool_tokens=_pool_window_shifted)),
+    (check_pool_table, _mutant(pool_tokens=_pool_avg_counts_padding)),
+    (check_pool_avg_convolution, _mutant(pool_tokens=_pool_avg_counts_padding)),
+    (check_pool_before_mean, _mutant(token_saliency=_token_saliency_pool_after_mean)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

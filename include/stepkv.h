@@ -72,6 +72,8 @@ typedef enum {
 } stepkv_status_t;
 
 enum { STEPKV_NORM_MAX = 0, STEPKV_NORM_NONE = 1 };
+enum { STEPKV_POOL_MAX = 0, STEPKV_POOL_AVG = 1 };
+#define STEPKV_MAX_POOL 63
 enum { STEPKV_BUDGET_RATIO = 0, STEPKV_BUDGET_COUNT = 1 };
 
 /* Hyper-parameters of Eqs. 2-5 (Table H defaults from stepkv_default_params). */
@@ -87,6 +89,14 @@ typedef struct {
   float beta;     /* step-utility weight (Eq. 5) */
   int32_t sal_norm; /* STEPKV_NORM_MAX: T_i divided by its maximum over prunable tokens (appendix,
                        "H_i normalised to [0, H_max]"); STEPKV_NORM_NONE: T_i used as is */
+  int32_t sal_pool; /* SnapKV-style token-axis pooling of each saliency row before the mean over rows
+                       (Sec. 4.2: T_i from an existing estimator such as SnapKV): odd width k in
+                       [1, STEPKV_MAX_POOL], 1 = none.  Window [i - k/2, i + k/2] clipped to [0, T).
+                       Taken by stepkv_select; stepkv_compress rejects k > 1 (EUNSUPPORTED): its
+                       saliency pass sums the rows on the fly, so pool through stepkv_score rows and
+                       stepkv_select instead */
+  int32_t sal_pool_mode; /* STEPKV_POOL_MAX: maximum over the window; STEPKV_POOL_AVG: mean of the
+                            window's in-range values */
 } stepkv_params_t;
 
 /* KV budget (Eq. 1).  RATIO: B_t = max(1, floor(ratio_num * N_t / ratio_den)) of the N_t
@@ -213,7 +223,8 @@ STEPKV_API stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, 
  * Stages 2-4: step reduction, fusion and selection (Eqs. 1-5, Algorithm 1 Phases 1-3).
  *
  *  sal       [n_sal][T] float32: saliency rows (e.g. stepkv_score's n_layers*Hkv rows);
- *            T_i = mean over the n_sal rows, then normalised per params->sal_norm.
+ *            T_i = mean over the n_sal rows (each row first pooled over params->sal_pool tokens when
+ *            that is > 1), then normalised per params->sal_norm.
  *  step_id   [T] int32: step of each token (must lie in [0, n_steps) for prunable tokens; a
  *            violation sets STEPKV_EDATA and no selection is written).
  *  prot      [T] uint8: 1 = protected.

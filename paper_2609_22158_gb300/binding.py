@@ -17,6 +17,7 @@ LIB_PATH = os.path.join(_PKG_DIR, "libstepkv.so")
 
 STEPKV_OK, STEPKV_EINVAL, STEPKV_ECUDA, STEPKV_ENOSPACE, STEPKV_EUNSUPPORTED, STEPKV_EDATA, STEPKV_ETIMEOUT = range(7)
 NORM_MAX, NORM_NONE = 0, 1
+POOL_MAX, POOL_AVG = 0, 1
 BUDGET_RATIO, BUDGET_COUNT = 0, 1
 
 
@@ -31,7 +32,7 @@ class CParams(ctypes.Structure):
     _fields_ = [("lambda_", ctypes.c_float), ("w_r", ctypes.c_float), ("w_c", ctypes.c_float),
                 ("r_min", ctypes.c_float), ("r_max", ctypes.c_float), ("s_max", ctypes.c_float),
                 ("eta", ctypes.c_float), ("alpha", ctypes.c_float), ("beta", ctypes.c_float),
-                ("sal_norm", ctypes.c_int32)]
+                ("sal_norm", ctypes.c_int32), ("sal_pool", ctypes.c_int32), ("sal_pool_mode", ctypes.c_int32)]
 
 
 class CBudget(ctypes.Structure):
@@ -141,16 +142,19 @@ class Params:
     alpha: float = 0.2
     beta: float = 0.8
     sal_norm: int = NORM_MAX
+    sal_pool: int = 1  # SnapKV-style token-axis pooling width (odd; 1 = none), taken by stepkv_select
+    sal_pool_mode: int = POOL_MAX
 
     def c(self) -> CParams:
         return CParams(self.lam, self.w_r, self.w_c, self.r_min, self.r_max, self.s_max, self.eta, self.alpha,
-                       self.beta, self.sal_norm)
+                       self.beta, self.sal_norm, self.sal_pool, self.sal_pool_mode)
 
 
 def default_params() -> Params:
     cp = CParams()
     load_library().stepkv_default_params(ctypes.byref(cp))
-    return Params(cp.lambda_, cp.w_r, cp.w_c, cp.r_min, cp.r_max, cp.s_max, cp.eta, cp.alpha, cp.beta, cp.sal_norm)
+    return Params(cp.lambda_, cp.w_r, cp.w_c, cp.r_min, cp.r_max, cp.s_max, cp.eta, cp.alpha, cp.beta, cp.sal_norm,
+                  cp.sal_pool, cp.sal_pool_mode)
 
 
 # ----------------------------------------------------------------------------- helpers

@@ -128,6 +128,8 @@ static stepkv_status_t check_select_args(int n_sal, int T, const int32_t* step_i
   if (!steps->valid || !steps->gain || !steps->red || !steps->reuse_in) return STEPKV_EINVAL;
   if (!out->kept_idx || !out->n_kept || out->kept_cap < 0) return STEPKV_EINVAL;
   if (params->sal_norm != STEPKV_NORM_MAX && params->sal_norm != STEPKV_NORM_NONE) return STEPKV_EINVAL;
+  if (params->sal_pool < 1 || params->sal_pool > STEPKV_MAX_POOL || (params->sal_pool & 1) == 0) return STEPKV_EINVAL;
+  if (params->sal_pool_mode != STEPKV_POOL_MAX && params->sal_pool_mode != STEPKV_POOL_AVG) return STEPKV_EINVAL;
   if (budget->mode == STEPKV_BUDGET_RATIO) {
     if (budget->ratio_num < 0 || budget->ratio_den < 1) return STEPKV_EINVAL;
   } else if (budget->mode == STEPKV_BUDGET_COUNT) {
@@ -202,6 +204,18 @@ void stepkv_default_params(stepkv_params_t* p) {
   p->alpha = 0.2f;
   p->beta = 0.8f;
   p->sal_norm = STEPKV_NORM_MAX;
+  p->sal_pool = 1;
+  p->sal_pool_mode = STEPKV_POOL_MAX;
+}
+
+// T_i from the saliency rows: their mean, each row first pooled over params->sal_pool tokens when
+// that is > 1 (the SnapKV-style estimator).
+static stepkv_status_t token_saliency_run(const float* sal, int n_sal, int T, const stepkv_params_t& params,
+                                          float* Tbuf, cudaStream_t s) {
+  if (params.sal_pool > 1)
+    return pool_mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, params.sal_pool / 2,
+                              params.sal_pool_mode == STEPKV_POOL_MAX, Tbuf, s);
+  return mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, Tbuf, s);
 }
 
 const char* stepkv_status_string(int32_t status) {
@@ -281,7 +295,7 @@ stepkv_status_t stepkv_select(const float* sal, int32_t n_sal, int32_t T, const 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* Tbuf = static_cast<float*>(ws);
   void* sel_ws = static_cast<uint8_t*>(ws) + align256((size_t)T * sizeof(float));
-  st = mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, Tbuf, s);
+  st = token_saliency_run(sal, n_sal, T, *params, Tbuf, s);
   if (st != STEPKV_OK) return st;
   return select_run(Tbuf, nullptr, 0.0, T, step_id, prot, *steps, *params, *budget, *out, sel_ws, dev_status, s);
 }
@@ -336,7 +350,7 @@ stepkv_status_t stepkv_select_static_scratch(const float* sal, int32_t n_sal, in
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   float* Tbuf = static_cast<float*>(scratch);
   void* sel_ws = static_cast<uint8_t*>(scratch) + t_bytes;
-  st = mean_rows_run(sal, n_sal, T, 1.0f / (float)n_sal, T, Tbuf, s);
+  st = token_saliency_run(sal, n_sal, T, *params, Tbuf, s);
   if (st != STEPKV_OK) return st;
   return select_run(Tbuf, nullptr, 0.0, T, step_id, prot, *steps, *params, *budget, *out, sel_ws, dev_status, s);
 }
@@ -507,6 +521,8 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     if (st != STEPKV_OK) return st;
     st = check_select_args(Ls * p.Hkv, p.T, p.step_id, p.prot, &p.steps, params, &p.budget, &p.sel);
     if (st != STEPKV_OK) return st;
+    // the fused saliency pass sums the rows as it goes: pooling needs the rows (stepkv_score + stepkv_select)
+    if (params->sal_pool > 1) return STEPKV_EUNSUPPORTED;
     bool inplace = false;
     st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
                             p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);

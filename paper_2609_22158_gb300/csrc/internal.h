@@ -147,6 +147,10 @@ stepkv_status_t select_run(const float* T_in, const unsigned long long* t_acc, d
 // T_out[j] = inv_div * sum_r rows[r * row_stride + j] (fixed order over r).
 stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, float* T_out,
                               cudaStream_t stream);
+// The same mean after a token-axis pooling of each row over [j - h, j + h] clipped to [0, T): the
+// maximum (is_max) or the mean of the in-range values.
+stepkv_status_t pool_mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, int h,
+                                   bool is_max, float* T_out, cudaStream_t stream);
 
 // ---- compact (compact.cu)
 // One out-of-place compaction (as stepkv_compact's arguments).

@@ -678,6 +678,58 @@ __global__ void mean_rows_kernel(const float* __restrict__ rows, int n_rows, int
   }
 }
 
+// SnapKV-style estimator (Sec. 4.2: T_i from an existing token-level estimator): each row pooled along the
+// token axis over the window [j - h, j + h] clipped to [0, T) -- its maximum, or the mean of its in-range
+// values -- then T_out[j] = inv_div * the sum over rows in row order.  A CTA takes 256 tokens and stages
+// each row's 256 + 2h values (the tile and its halo) in shared memory, one row at a time.
+constexpr int kPoolTile = 256;
+
+template <bool IS_MAX>
+__global__ void __launch_bounds__(kPoolTile) pool_mean_rows_kernel(const float* __restrict__ rows, int n_rows,
+                                                                   int64_t row_stride, float inv_div, int T, int h,
+                                                                   float* __restrict__ T_out) {
+  extern __shared__ float tile[];  // [kPoolTile + 2h]
+  pdl_wait();
+  pdl_launch_dependents();
+  const int j0 = blockIdx.x * kPoolTile, j = j0 + (int)threadIdx.x;
+  const int span = kPoolTile + 2 * h;
+  // this token's window as tile indices (tile index x holds token j0 - h + x)
+  const int lo = max(0, j - h) - (j0 - h), hi = min(T - 1, j + h) - (j0 - h);
+  float acc = 0.f;
+  for (int r = 0; r < n_rows; ++r) {
+    const float* row = rows + (int64_t)r * row_stride;
+    __syncthreads();  // the previous row's tile has been read
+    for (int x = (int)threadIdx.x; x < span; x += kPoolTile) {
+      const int src = j0 - h + x;
+      tile[x] = (src >= 0 && src < T) ? __ldg(row + src) : 0.f;
+    }
+    __syncthreads();
+    if (j < T) {
+      float v = tile[lo];
+      for (int x = lo + 1; x <= hi; ++x) v = IS_MAX ? fmaxf(v, tile[x]) : v + tile[x];
+      if (!IS_MAX) v = v / (float)(hi - lo + 1);
+      acc += v;
+    }
+  }
+  if (j < T) T_out[j] = acc * inv_div;
+}
+
+stepkv_status_t pool_mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, int h,
+                                   bool is_max, float* T_out, cudaStream_t stream) {
+  const int blocks = (T + kPoolTile - 1) / kPoolTile;
+  const size_t smem = (size_t)(kPoolTile + 2 * h) * sizeof(float);
+  const cudaError_t e =
+      is_max ? launch_kernel(pool_mean_rows_kernel<true>, dim3(blocks), dim3(kPoolTile), smem, stream, rows, n_rows,
+                             row_stride, inv_div, T, h, T_out)
+             : launch_kernel(pool_mean_rows_kernel<false>, dim3(blocks), dim3(kPoolTile), smem, stream, rows, n_rows,
+                             row_stride, inv_div, T, h, T_out);
+  if (e != cudaSuccess) {
+    set_last_cuda_error(e);
+    return STEPKV_ECUDA;
+  }
+  return STEPKV_OK;
+}
+
 stepkv_status_t mean_rows_run(const float* rows, int n_rows, int64_t row_stride, float inv_div, int T, float* T_out,
                               cudaStream_t stream) {
   const int blocks = std::max(1, std::min((T + 255) / 256, 4096));

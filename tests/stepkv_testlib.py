@@ -33,7 +33,8 @@ def bits_of(x) -> np.ndarray:
 
 def oracle_params(p) -> "O.Params":
     return O.Params(lam=p.lam, w_r=p.w_r, w_c=p.w_c, r_min=p.r_min, r_max=p.r_max, s_max=p.s_max, eta=p.eta,
-                    alpha=p.alpha, beta=p.beta, sal_norm="max" if p.sal_norm == 0 else "none")
+                    alpha=p.alpha, beta=p.beta, sal_norm="max" if p.sal_norm == 0 else "none",
+                    pool=getattr(p, "sal_pool", 1), pool_mode="max" if getattr(p, "sal_pool_mode", 0) == 0 else "avg")
 
 
 def max_rel_err(g, o, floor: float = 0.0) -> float:

@@ -43,6 +43,7 @@ def test_default_params_are_table_h(lib):
     assert abs(p.lam - 0.3) < 1e-7 and abs(p.w_r - 0.85) < 1e-7 and abs(p.w_c - 0.15) < 1e-7
     assert p.r_min == -1.0 and p.r_max == 2.0 and p.s_max == 8.0
     assert p.eta == 1.5 and abs(p.alpha - 0.2) < 1e-7 and abs(p.beta - 0.8) < 1e-7 and p.sal_norm == 0
+    assert p.sal_pool == 1 and p.sal_pool_mode == binding.POOL_MAX  # no pooling by default
 
 
 def test_status_strings(lib):
@@ -90,6 +91,8 @@ def test_select_rejects_bad_arguments_on_host(lib):
     assert args(steps, params, bad, out) == B.STEPKV_EINVAL          # zero denominator
     bad_norm = B.Params(sal_norm=7).c()
     assert args(steps, bad_norm, bud, out) == B.STEPKV_EINVAL
+    for pool, mode in ((0, B.POOL_MAX), (4, B.POOL_MAX), (65, B.POOL_MAX), (3, 2)):  # even, too wide, bad mode
+        assert args(steps, B.Params(sal_pool=pool, sal_pool_mode=mode).c(), bud, out) == B.STEPKV_EINVAL
     out.kept_idx = None
     assert args(steps, params, bud, out) == B.STEPKV_EINVAL
 

@@ -284,6 +284,30 @@ def test_select_exact_on_shared_fp32_priorities(B, levels):
     assert np.array_equal(g.out.step_kept.cpu().numpy(), out["step_kept"])
 
 
+@pytest.mark.parametrize("pool, mode, T", [(3, 0, 9000), (7, 0, 9000), (7, 1, 9000), (63, 1, 9000), (31, 0, 9000),
+                                           (5, 1, 1500)])
+def test_select_snapkv_pooling(B, pool, mode, T):
+    """SnapKV-style estimator: every saliency row pooled over `pool` tokens (max or in-range mean) before
+    the mean over rows, then Eqs. 2-5 and the selection, against the oracle (windows clipped at both ends;
+    T = 1500 takes the single-CTA selection)."""
+    tr = wl.custom(11 + pool, L=1, Hq=8, Hkv=2, d=64, T=T, W=16, n_steps=10, budget=wl.Budget.ratio(1, 5))
+    rng = np.random.default_rng(pool * 10 + mode)
+    sal = (rng.random((6, tr.T)) ** 3).astype(np.float32)
+    p = B.Params(sal_pool=pool, sal_pool_mode=mode)
+    g, out, st = _select_case(B, tr, p, sal)
+    assert st == 0
+    TL.check_select_outputs(g, out)
+
+
+def test_compress_rejects_pooling(B):
+    """The fused pass sums the saliency rows as it goes, so it refuses a pooling width (EUNSUPPORTED)."""
+    tr = wl.custom(5, L=2, Hq=8, Hkv=2, d=64, T=1200, W=16, n_steps=6, budget=wl.Budget.ratio(1, 4))
+    g = TL.GpuTraj(tr)
+    with pytest.raises(B.StepKVError) as e:
+        B.stepkv_compress([g.problem()], B.Params(sal_pool=3))
+    assert e.value.code == B.STEPKV_EUNSUPPORTED
+
+
 def test_select_large_T(B):
     """T = 200000 (beyond 8 x 16K): every CTA of the cluster holds ~25K tokens."""
     T = 200000

@@ -113,6 +113,27 @@ def pool_tokens(a: np.ndarray, k: int, mode: str = "max") -> np.ndarray:
     return windows.max(axis=1) if mode == "max" else np.nanmean(windows, axis=1)
 
 
+def window_row_lse(K: np.ndarray, Q: np.ndarray) -> np.ndarray:
+    """Natural-log log-sum-exp of every observation query's causal attention row (what a prefill
+    attention kernel reports beside its output): lse[g, w] = log sum_{j <= p_w} exp(q_{g,w} . k_j / sqrt(d)),
+    p_w = T-W+w, with the query heads mapped to KV heads as in window_attention_saliency.
+    K: [Hkv, T, d] and Q: [Hq, W, d] bf16 bits; returns [Hq, W] float64."""
+    K = bf16_to_f64(K)
+    Q = bf16_to_f64(Q)
+    Hkv, T, d = K.shape
+    Hq, W, _ = Q.shape
+    G = Hq // Hkv
+    scale = 1.0 / math.sqrt(d)
+    lse = np.empty((Hq, W), dtype=np.float64)
+    for g in range(Hq):
+        s = (Q[g] @ K[g // G].T) * scale                           # [W, T] logits
+        visible = np.arange(T)[None, :] <= (T - W + np.arange(W))[:, None]
+        s = np.where(visible, s, -np.inf)
+        m = s.max(axis=1, keepdims=True)
+        lse[g] = (m + np.log(np.where(visible, np.exp(s - m), 0.0).sum(axis=1, keepdims=True)))[:, 0]
+    return lse
+
+
 def token_saliency(A_layers: Sequence[np.ndarray], pool: int = 1, pool_mode: str = "max") -> np.ndarray:
     """T_i = mean over (saliency layer, KV head) of A[l, h, i]  (reading: mean pooling); with pool > 1
     each (layer, KV head) row is first pooled along the token axis (pool_tokens)."""

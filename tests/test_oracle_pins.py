@@ -587,6 +587,51 @@ def test_boundary_step_statistics():
     check_boundary_step_statistics(REAL)
 
 
+# ------------------------------------------------------------------ prefill row log-sum-exp
+def check_lse_zero_keys(O):
+    """All logits 0: each row's log-sum-exp is log(number of visible keys) = log(T - W + w + 1)."""
+    Hkv, G, T, W, d = 2, 2, 40, 6, 16
+    K = _bits(np.zeros((Hkv, T, d)))
+    Q = _bits(np.random.default_rng(1).standard_normal((Hkv * G, W, d)))
+    lse = O.window_row_lse(K, Q)
+    np.testing.assert_allclose(lse, np.log(T - W + np.arange(W) + 1.0)[None, :].repeat(Hkv * G, 0), rtol=1e-12)
+
+
+def check_lse_logsumexp(O):
+    """Brute force: scipy's logsumexp over each row's visible scaled dot products, key by key."""
+    from scipy.special import logsumexp
+    rng = np.random.default_rng(2)
+    Hkv, G, T, W, d = 2, 3, 30, 4, 8
+    K, Q = _rand_qk(rng, Hkv, G, T, W, d)
+    Kf, Qf = wl.bf16_bits_to_f32(K).astype(np.float64), wl.bf16_bits_to_f32(Q).astype(np.float64)
+    lse = O.window_row_lse(K, Q)
+    for g in range(Hkv * G):
+        for w in range(W):
+            logits = [float(Qf[g, w] @ Kf[g // G, j]) / math.sqrt(d) for j in range(T - W + w + 1)]
+            assert abs(lse[g, w] - logsumexp(logits)) < 1e-10
+
+
+def check_lse_rebuilds_saliency(O):
+    """exp(s - lse) summed over a KV head's query rows and averaged over its group is the saliency."""
+    rng = np.random.default_rng(3)
+    Hkv, G, T, W, d = 2, 2, 25, 5, 8
+    K, Q = _rand_qk(rng, Hkv, G, T, W, d)
+    Kf, Qf = wl.bf16_bits_to_f32(K).astype(np.float64), wl.bf16_bits_to_f32(Q).astype(np.float64)
+    lse = O.window_row_lse(K, Q)
+    A = np.zeros((Hkv, T))
+    for g in range(Hkv * G):
+        for w in range(W):
+            vis = T - W + w + 1
+            s = Qf[g, w] @ Kf[g // G, :vis].T / math.sqrt(d)
+            A[g // G, :vis] += np.exp(s - lse[g, w]) / G
+    np.testing.assert_allclose(A, O.window_attention_saliency(K, Q), rtol=1e-10, atol=1e-14)
+
+
+def test_prefill_lse_pins():
+    for chk in (check_lse_zero_keys, check_lse_logsumexp, check_lse_rebuilds_saliency):
+        chk(REAL)
+
+
 # ------------------------------------------------------------------ SnapKV-style pooling (Sec. 4.2)
 def check_pool_table(O):
     """The hand table of tests/golden/snapkv_pooling.txt."""
@@ -857,6 +902,23 @@ def _signals_obs_only_gain(th, act, obs, k0=None):
     return gain, red, obs_sim
 
 
+def _lse_interleaved_groups(K, Q):
+    # wrong GQA convention: q head g reads KV head g % Hkv
+    Hkv = K.shape[0]
+    order = np.concatenate([np.arange(g, Q.shape[0], Hkv) for g in range(Hkv)])
+    out = np.empty((Q.shape[0], Q.shape[1]))
+    out[order] = REAL.window_row_lse(K, Q[order])
+    return out
+
+
+def _lse_not_causal(K, Q):
+    # every query row sees all T keys
+    from scipy.special import logsumexp
+    Kf, Qf = wl.bf16_bits_to_f32(K).astype(np.float64), wl.bf16_bits_to_f32(Q).astype(np.float64)
+    G = Q.shape[0] // K.shape[0]
+    return np.stack([logsumexp(Qf[g] @ Kf[g // G].T / math.sqrt(K.shape[2]), axis=1) for g in range(Q.shape[0])])
+
+
 def _pool_window_shifted(a, k, mode="max"):
     # window [i - k//2 + 1, i + k//2 + 1]: off by one to the right
     b = np.concatenate([np.asarray(a, dtype=np.float64)[1:], [-np.inf if mode == "max" else np.nan]])
@@ -909,6 +971,9 @@ def _token_saliency_pool_after_mean(A_layers, pool=1, pool_mode="max"):
     (check_pool_table, _mutant(pool_tokens=_pool_avg_counts_padding)),
     (check_pool_avg_convolution, _mutant(pool_tokens=_pool_avg_counts_padding)),
     (check_pool_before_mean, _mutant(token_saliency=_token_saliency_pool_after_mean)),
+    (check_lse_logsumexp, _mutant(window_row_lse=_lse_interleaved_groups)),
+    (check_lse_rebuilds_saliency, _mutant(window_row_lse=_lse_interleaved_groups)),
+    (check_lse_zero_keys, _mutant(window_row_lse=_lse_not_causal)),
 ])
 def test_planted_mistake_is_caught(check, mutant):
     with pytest.raises(AssertionError):

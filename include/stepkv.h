@@ -179,6 +179,11 @@ typedef struct {
   const void* const* K_sal;        /* host [n_sal_layers] of device pointers, required when kv_location is
                                       HOST: layer L-n_sal_layers+i's K in device memory, same layout and
                                       head stride as K; ignored otherwise */
+  const float* const* sal_lse;     /* host [n_sal_layers] of device pointers, or NULL: each window query's
+                                      natural-log log-sum-exp over its causal row, [Hq][W] float32 (what the
+                                      Observation prefill's attention reports; Sec. 4.2 collects T_i during
+                                      that prefill).  Given, the saliency stage skips its first pass; see
+                                      stepkv_score_lse */
 } stepkv_problem_t;
 
 #define STEPKV_MEM_DEVICE 0
@@ -218,6 +223,21 @@ STEPKV_API stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, 
                              const void* const* Q, int64_t q_head_stride,
                              int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
                              float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
+
+/* stepkv_score with the rows' statistics supplied (Sec. 4.2: T_i "collected during the existing
+ * observation prefill"): the prefill's attention already computes, for every window query, the
+ * log-sum-exp of its causal row, so only the second pass (the per-key softmax mass) runs.
+ *
+ *  lse[l]  host array of device pointers, [Hq][W] float32: lse[g][w] = ln sum_{j <= T-W+w}
+ *          exp(q_{l,g,w} . k_{l,g/G,j} / sqrt(d)), natural log, as flash-attention kernels report it.
+ *  Everything else as stepkv_score (same workspace size).  The result equals stepkv_score's when lse is
+ *  the exact log-sum-exp; an lse off by delta for one query row scales that row's contribution by
+ *  exp(-delta).
+ */
+STEPKV_API stepkv_status_t stepkv_score_lse(int32_t n_layers, const void* const* K, int64_t k_head_stride,
+                                 const void* const* Q, int64_t q_head_stride, const float* const* lse,
+                                 int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
+                                 float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream);
 
 /* ---------------------------------------------------------------------------------------------
  * Stages 2-4: step reduction, fusion and selection (Eqs. 1-5, Algorithm 1 Phases 1-3).

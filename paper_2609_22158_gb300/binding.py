@@ -62,7 +62,8 @@ class CProblem(ctypes.Structure):
                 ("steps", CSteps), ("budget", CBudget),
                 ("K_out", ctypes.c_void_p), ("V_out", ctypes.c_void_p), ("out_head_stride", ctypes.c_int64),
                 ("step_id_out", ctypes.c_void_p), ("pos_out", ctypes.c_void_p), ("sel", CSelOut),
-                ("kv_location", ctypes.c_int32), ("out_location", ctypes.c_int32), ("K_sal", ctypes.c_void_p)]
+                ("kv_location", ctypes.c_int32), ("out_location", ctypes.c_int32), ("K_sal", ctypes.c_void_p),
+                ("sal_lse", ctypes.c_void_p)]
 
 
 STEPKV_MEM_DEVICE = 0
@@ -80,6 +81,8 @@ SIGNATURES = {
     "stepkv_last_cuda_error": (ctypes.c_char_p, []),
     "stepkv_score_workspace_size": (_SZ, [_I32, _I32, _I32, _I32, _I32]),
     "stepkv_score": (_I32, [_I32, _VP, _I64, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ, _VP, _VP]),
+    "stepkv_score_lse": (_I32, [_I32, _VP, _I64, _VP, _I64, _VP, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ, _VP,
+                                _VP]),
     "stepkv_selftest_score_timeout": (_I32, [_I32, _VP, _I64, _VP, _I64, _I32, _I32, _I32, _I32, _I32, _VP, _VP, _SZ,
                                              ctypes.c_uint64, _VP, _VP]),
     "stepkv_select_workspace_size": (_SZ, [_I32, _I32, _I32]),
@@ -242,9 +245,11 @@ def _aligned_ws(ws):
 
 # ----------------------------------------------------------------------------- stage 1
 def stepkv_score(K: Sequence, Q: Sequence, T: int, W: Optional[int] = None, sal=None, ws=None, status=None,
-                 stream=None):
+                 stream=None, lse: Optional[Sequence] = None):
     """Window-attention saliency of len(K) layers: returns sal [n_layers, Hkv, T] float32.
-    K[l]: [Hkv, rows >= T, d] bf16; Q[l]: [Hq, W, d] bf16 (query w at slot T-W+w)."""
+    K[l]: [Hkv, rows >= T, d] bf16; Q[l]: [Hq, W, d] bf16 (query w at slot T-W+w).  With lse (per layer
+    [Hq, W] float32, each query's natural-log causal log-sum-exp, as a prefill attention reports it) the
+    row statistics are taken from it and only the second pass runs (stepkv_score_lse)."""
     torch = _torch()
     lib = load_library()
     n = len(K)
@@ -266,9 +271,22 @@ def stepkv_score(K: Sequence, Q: Sequence, T: int, W: Optional[int] = None, sal=
     wp, wn = _aligned_ws(ws)
     status = status if status is not None else new_status(dev)
     kp, qp = _ptr_array(K), _ptr_array(Q)
-    code = lib.stepkv_score(n, ctypes.cast(kp, ctypes.c_void_p), ks, ctypes.cast(qp, ctypes.c_void_p), qs, Hkv, Hq, d,
-                            T, W, sal.data_ptr(), wp, wn, status.data_ptr(), _stream_handle(stream))
-    _check(code, "stepkv_score")
+    if lse is None:
+        code = lib.stepkv_score(n, ctypes.cast(kp, ctypes.c_void_p), ks, ctypes.cast(qp, ctypes.c_void_p), qs, Hkv, Hq,
+                                d, T, W, sal.data_ptr(), wp, wn, status.data_ptr(), _stream_handle(stream))
+        _check(code, "stepkv_score")
+        return sal
+    if len(lse) != n:
+        raise ValueError("lse needs one tensor per layer")
+    for i, t in enumerate(lse):
+        _need(t, torch.float32, f"lse[{i}]", 2)
+        if tuple(t.shape) != (Hq, W) or not t.is_contiguous():
+            raise ValueError(f"lse[{i}] must be a contiguous [Hq, W] float32 tensor")
+    lp = _ptr_array(lse)
+    code = lib.stepkv_score_lse(n, ctypes.cast(kp, ctypes.c_void_p), ks, ctypes.cast(qp, ctypes.c_void_p), qs,
+                                ctypes.cast(lp, ctypes.c_void_p), Hkv, Hq, d, T, W, sal.data_ptr(), wp, wn,
+                                status.data_ptr(), _stream_handle(stream))
+    _check(code, "stepkv_score_lse")
     return sal
 
 
@@ -597,6 +615,9 @@ class Problem:
     kv_location: int = STEPKV_MEM_DEVICE
     out_location: int = STEPKV_MEM_DEVICE
     K_sal: Optional[List] = None
+    # n_sal_layers x [Hq, W] float32: each window query's natural-log causal log-sum-exp from the
+    # Observation prefill; given, the saliency stage runs its second pass only
+    sal_lse: Optional[List] = None
     _keep: list = field(default_factory=list, repr=False)
     _c: object = field(default=None, repr=False)
 
@@ -629,14 +650,22 @@ class Problem:
         Hq, W, _ = self.Q[0].shape
         _need(self.step_id, torch.int32, "step_id", 1)
         _need(self.prot, torch.uint8, "prot", 1)
+        if self.sal_lse is not None:
+            if len(self.sal_lse) != Ls:
+                raise ValueError("sal_lse needs one [Hq, W] tensor per saliency layer")
+            for i, t in enumerate(self.sal_lse):
+                _need(t, torch.float32, f"sal_lse[{i}]", 2)
+                if tuple(t.shape) != (Hq, W) or not t.is_contiguous():
+                    raise ValueError(f"sal_lse[{i}] must be a contiguous [Hq, W] float32 tensor")
         arrs = [_ptr_array(self.K), _ptr_array(self.V), _ptr_array(self.Q), _ptr_array(self.K_out),
-                _ptr_array(self.V_out), _ptr_array(self.K_sal or [])]
+                _ptr_array(self.V_out), _ptr_array(self.K_sal or []), _ptr_array(self.sal_lse or [])]
         self._keep = arrs
         cv = lambda a: ctypes.cast(a, ctypes.c_void_p)
         return CProblem(L, Hkv, Hq, d, self.T, W, Ls, cv(arrs[0]), cv(arrs[1]), ks, cv(arrs[2]), qs,
                         _ptr(self.step_id), _ptr(self.prot), _ptr(self.pos_in), self.steps.c(), self.budget,
                         cv(arrs[3]), cv(arrs[4]), outs, _ptr(self.step_id_out), _ptr(self.pos_out), self.out.c(),
-                        self.kv_location, self.out_location, cv(arrs[5]) if kv_host else None)
+                        self.kv_location, self.out_location, cv(arrs[5]) if kv_host else None,
+                        cv(arrs[6]) if self.sal_lse is not None else None)
 
 
 def stepkv_workspace_size(problems: Sequence[Problem]) -> int:

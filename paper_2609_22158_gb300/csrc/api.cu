@@ -240,11 +240,16 @@ size_t stepkv_score_workspace_size(int32_t n_layers, int32_t Hkv, int32_t Hq, in
   return score_ws(n_layers, Hkv, Hq, T, W, score_row_groups(Hkv, Hq, W) > 1);
 }
 
-stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
-                             int64_t q_head_stride, int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
-                             float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
+static stepkv_status_t score_entry(int32_t n_layers, const void* const* K, int64_t k_head_stride,
+                                   const void* const* Q, int64_t q_head_stride, const float* const* lse, int32_t Hkv,
+                                   int32_t Hq, int32_t d, int32_t T, int32_t W, float* sal, void* ws, size_t ws_bytes,
+                                   int32_t* dev_status, void* stream) {
   stepkv_status_t st = check_score_args(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W);
   if (st != STEPKV_OK) return st;
+  if (lse) {
+    for (int l = 0; l < n_layers; ++l)
+      if (!lse[l] || (reinterpret_cast<uintptr_t>(lse[l]) & 3u) != 0) return STEPKV_EINVAL;
+  }
   if (!sal || !ws) return STEPKV_EINVAL;
   const int n_rg = score_row_groups(Hkv, Hq, W);
   const size_t need = score_ws(n_layers, Hkv, Hq, T, W, n_rg > 1);
@@ -256,10 +261,26 @@ stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_h
   if (n_rg > 1)
     rows = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + align256(score_partial_bytes(n_layers, Hkv, Hq, W)));
   st = score_run(n_layers, K, k_head_stride, Q, q_head_stride, Hkv, Hq, d, T, W, rows, T, nullptr, 0, part,
-                 dev_status, s);
+                 dev_status, s, 0, lse);
   if (st != STEPKV_OK) return st;
   if (n_rg > 1) st = score_sum_row_groups(rows, n_layers * Hkv, n_rg, T, sal, s);
   return st;
+}
+
+stepkv_status_t stepkv_score(int32_t n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                             int64_t q_head_stride, int32_t Hkv, int32_t Hq, int32_t d, int32_t T, int32_t W,
+                             float* sal, void* ws, size_t ws_bytes, int32_t* dev_status, void* stream) {
+  return score_entry(n_layers, K, k_head_stride, Q, q_head_stride, nullptr, Hkv, Hq, d, T, W, sal, ws, ws_bytes,
+                     dev_status, stream);
+}
+
+stepkv_status_t stepkv_score_lse(int32_t n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
+                                 int64_t q_head_stride, const float* const* lse, int32_t Hkv, int32_t Hq, int32_t d,
+                                 int32_t T, int32_t W, float* sal, void* ws, size_t ws_bytes, int32_t* dev_status,
+                                 void* stream) {
+  if (!lse) return STEPKV_EINVAL;
+  return score_entry(n_layers, K, k_head_stride, Q, q_head_stride, lse, Hkv, Hq, d, T, W, sal, ws, ws_bytes,
+                     dev_status, stream);
 }
 
 stepkv_status_t stepkv_selftest_score_timeout(int32_t n_layers, const void* const* K, int64_t k_head_stride,
@@ -460,7 +481,7 @@ static std::vector<SalBatch> saliency_batches(const stepkv_problem_t* probs, int
   std::vector<SalBatch> out;
   auto same = [](const stepkv_problem_t& a, const stepkv_problem_t& b) {
     return std::min(a.n_sal_layers, a.L) == std::min(b.n_sal_layers, b.L) && a.Hkv == b.Hkv && a.Hq == b.Hq &&
-           a.d == b.d && a.W == b.W;
+           a.d == b.d && a.W == b.W && (a.sal_lse != nullptr) == (b.sal_lse != nullptr);
   };
   for (int i = 0; i < n_traj;) {
     const int Ls = std::max(1, std::min(probs[i].n_sal_layers, probs[i].L));
@@ -523,6 +544,10 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     if (st != STEPKV_OK) return st;
     // the fused saliency pass sums the rows as it goes: pooling needs the rows (stepkv_score + stepkv_select)
     if (params->sal_pool > 1) return STEPKV_EUNSUPPORTED;
+    if (p.sal_lse) {
+      for (int l = 0; l < Ls; ++l)
+        if (!p.sal_lse[l] || (reinterpret_cast<uintptr_t>(p.sal_lse[l]) & 3u) != 0) return STEPKV_EINVAL;
+    }
     bool inplace = false;
     st = check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
                             p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
@@ -554,7 +579,7 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     w += compress_traj_bytes(p);
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
-    sal[i] = ScoreTrajSpec{sal_keys(p), p.Q, p.T, t_acc, p.kv_head_stride, p.q_head_stride};
+    sal[i] = ScoreTrajSpec{sal_keys(p), p.Q, p.T, t_acc, p.kv_head_stride, p.q_head_stride, p.sal_lse};
     specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
                           *params, p.budget, p.sel, sel_ws, dev_status};
   }

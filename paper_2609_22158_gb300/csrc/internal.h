@@ -108,6 +108,7 @@ struct ScoreTrajSpec {
   int T;
   unsigned long long* t_acc;
   int64_t k_head_stride, q_head_stride;
+  const float* const* lse = nullptr;  // per layer [Hq][W] natural-log row log-sum-exp (skips pass 1), or NULL
 };
 // Saliency of n_traj trajectories of one head shape in one cooperative launch (n_traj <= kMaxScoreBatch,
 // n_traj * n_layers <= kMaxScoreMaps); rows output only for n_traj == 1.
@@ -118,7 +119,8 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
                           int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
-                          cudaStream_t stream, unsigned long long selftest_wait_ns = 0);
+                          cudaStream_t stream, unsigned long long selftest_wait_ns = 0,
+                          const float* const* lse = nullptr);
 stepkv_status_t score_sum_row_groups(const float* rows, int n_pairs, int n_rg, int T, float* sal, cudaStream_t stream);
 
 // ---- select (select.cu)

@@ -87,6 +87,8 @@ struct ScoreLaunch {
   unsigned long long* epoch;  // per-workspace launch counter, advanced by CTA 0 at the end of every launch
   unsigned long long token;   // host value, unique per call; mixed with the epoch into the launch token
   int selftest;               // 1: the pass-2 wait looks for a value no CTA publishes (failure-path self-test)
+  int pass2_only;             // 1: the row statistics come from the caller (lse), pass 1 is skipped
+  const float* lse[kMaxScoreMaps];  // [traj * n_layers + layer]: [Hq][W] natural-log row log-sum-exp
   unsigned long long wait_limit_ns;  // the pass-2 wait gives up (STEPKV_ETIMEOUT) after this long
   int32_t* status;
 };
@@ -444,7 +446,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         return true;
       };
       int slot = 0;
-      for (int t = t_lo; t < t_hi && ok;) {
+      for (int t = p.pass2_only ? t_hi : t_lo; t < t_hi && ok;) {
         const int nt = item_tiles(locate(p, t), t);
         for (int i = 0; i < nt && ok; ++i) ok = load_tile(t + i, 2 * slot + i);
         t += nt;
@@ -489,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       };
       // pass 1: S = Q K^T, one half per 128-row query tile, N = the item's keys (256 or 128)
       int slot = 0;
-      for (int t = t_lo; t < t_hi && ok;) {
+      for (int t = p.pass2_only ? t_hi : t_lo; t < t_hi && ok;) {
         const ItemLoc il = locate(p, t);
         const int nt = item_tiles(il, t);
         const int u = il.u;
@@ -600,8 +602,9 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       }
     }
 
-    // ---- pass 1: per-row running (m, Z) over the keys this warp sees
-    {
+    // ---- pass 1: per-row running (m, Z) over the keys this warp sees (skipped when the caller gives the
+    // rows' log-sum-exp)
+    if (!p.pass2_only) {
       int cur = -1, Tb = 0;
       float m = -INFINITY, Z = 0.f;
       int my_row = 0, my_pw = 0, my_e = 0;
@@ -714,7 +717,8 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
             const uint64_t t0 = globaltimer_ns();
             for (uint32_t it = 0; !all; ++it) {
               bool mine = true;
-              for (int b = c0 + lane; b <= c1; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == wait_tok;
+              if (!p.pass2_only)  // no pass-1 partials to wait for when the caller gives the row statistics
+                for (int b = c0 + lane; b <= c1; b += 32) mine &= ld_relaxed_u64(&p.flags[b]) == wait_tok;
               if (!zeros_seen) {
 #pragma unroll 4
                 for (int b = lane; b < (int)gridDim.x; b += 32) mine &= ld_relaxed_u64(&p.zflags[b]) == wait_tok;
@@ -739,7 +743,14 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
           const int w = r.w0 + row % r.blk_rows;
           const bool valid = row < r.rows && w < g.W;
           float off = INFINITY;
-          if (valid) {
+          if (valid && p.pass2_only) {
+            // the caller's natural-log row log-sum-exp, in the kernel's log2 units
+            int rg_x, h_x;
+            const int pair_x = p.pair0 + fdivmod(il.ul, g.rg_div, rg_x);
+            const int layer_x = fdivmod(pair_x, g.hkv_div, h_x);
+            const int q_head = h_x * g.G + r.g_first + row / r.blk_rows;
+            off = __ldg(p.lse[il.b * p.n_layers + layer_x] + (size_t)q_head * g.W + w) * 1.4426950408889634f;
+          } else if (valid) {
             // Log-sum-exp over the unit's entries in a fixed order.  Up to 16 entries (every unit spans
             // at most 8 CTAs for tile ranges of 32 or more) are loaded at once, so one L2 round trip
             // serves them all; longer lists continue in batches of 16.
@@ -1071,6 +1082,7 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   L.out = rows_out;
   L.out_stride = out_stride;
   L.accumulate = trajs[0].t_acc != nullptr ? 1 : 0;
+  L.pass2_only = trajs[0].lse != nullptr ? 1 : 0;
   L.acc_shift = acc_shift;
   L.status = status;
   const int box_rows = std::min(g.W_pad, kMaxRows);
@@ -1078,7 +1090,10 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
   for (int b = 0; b < n_traj; ++b) {
     const ScoreTrajSpec& t = trajs[b];
     if ((t.t_acc != nullptr) != (L.accumulate != 0)) return STEPKV_EINVAL;
+    if ((t.lse != nullptr) != (L.pass2_only != 0)) return STEPKV_EINVAL;
     for (int l = 0; l < n_layers; ++l) {
+      if (t.lse && !t.lse[l]) return STEPKV_EINVAL;
+      L.lse[b * n_layers + l] = t.lse ? t.lse[l] : nullptr;
       if (!encode_3d(&L.tmK[b * n_layers + l], t.K[l], d, t.T, Hkv, t.k_head_stride, kKeyTile)) return STEPKV_ECUDA;
       if (!encode_3d(&L.tmQ[b * n_layers + l], t.Q[l], d, W, Hq, t.q_head_stride, box_rows)) return STEPKV_ECUDA;
     }
@@ -1113,8 +1128,8 @@ stepkv_status_t score_run_batch(int n_layers, const ScoreTrajSpec* trajs, int n_
 stepkv_status_t score_run(int n_layers, const void* const* K, int64_t k_head_stride, const void* const* Q,
                           int64_t q_head_stride, int Hkv, int Hq, int d, int T, int W, float* rows_out,
                           int64_t out_stride, unsigned long long* t_acc, int acc_shift, float2* part, int32_t* status,
-                          cudaStream_t stream, unsigned long long selftest_wait_ns) {
-  const ScoreTrajSpec one{K, Q, T, t_acc, k_head_stride, q_head_stride};
+                          cudaStream_t stream, unsigned long long selftest_wait_ns, const float* const* lse) {
+  const ScoreTrajSpec one{K, Q, T, t_acc, k_head_stride, q_head_stride, lse};
   return score_run_batch(n_layers, &one, 1, Hkv, Hq, d, W, rows_out, out_stride, acc_shift, part, status, stream,
                          selftest_wait_ns);
 }

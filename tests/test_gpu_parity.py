@@ -60,6 +60,71 @@ def test_score_matches_oracle(B, Hkv, G, d, T, W, nl):
         assert np.allclose(g[l].sum(axis=1), W, rtol=1e-4)
 
 
+@pytest.mark.parametrize("Hkv,G,d,T,W,nl", SCORE_CASES + [(1, 4, 128, 2500, 512, 1), (1, 5, 128, 3000, 1024, 1)])
+def test_score_with_prefill_lse_matches_oracle(B, Hkv, G, d, T, W, nl):
+    """stepkv_score_lse: the rows' log-sum-exp comes from the caller (the oracle's, rounded to fp32, as
+    a prefill attention kernel would report it) and only the second pass runs."""
+    import torch
+    rng = np.random.default_rng(2000 + T + W)
+    Ks = [_rand_bits(rng, (Hkv, T, d)) for _ in range(nl)]
+    Qs = [_rand_bits(rng, (Hkv * G, W, d)) for _ in range(nl)]
+    lse = [torch.from_numpy(O.window_row_lse(k, q).astype(np.float32)).cuda() for k, q in zip(Ks, Qs)]
+    st = B.new_status()
+    sal = B.stepkv_score([TL.bf16_dev(k) for k in Ks], [TL.bf16_dev(q) for q in Qs], T, status=st, lse=lse)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    g = sal.cpu().numpy()
+    for l in range(nl):
+        TL.assert_close(g[l], O.window_attention_saliency(Ks[l], Qs[l]), f"sal layer {l}")
+
+
+def test_compress_with_prefill_lse(B):
+    """The fused pass with each saliency layer's row log-sum-exp given (stepkv_problem_t.sal_lse): pass 1
+    is skipped and every output matches the oracle."""
+    import torch
+    tr = wl.custom(83, L=4, Hq=16, Hkv=4, d=128, T=6000, W=64, n_steps=12, budget=wl.Budget.ratio(1, 8))
+    g = TL.GpuTraj(tr)
+    prob = g.problem()
+    prob.sal_lse = [torch.from_numpy(O.window_row_lse(tr.keys(l), tr.queries(l)).astype(np.float32)).cuda()
+                    for l in tr.sal_layer_ids()]
+    prob.refresh()
+    p = B.Params()
+    st = B.stepkv_compress([prob], p)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(p)))
+    n = int(g.out.n_kept.item())
+    kt = g.out.kept_idx[:n].long()
+    for l in range(tr.shape.L):
+        assert torch.equal(g.K_out[l][:, :n], g.K[l].index_select(1, kt))
+
+
+def test_score_with_prefill_lse_uses_it(B):
+    """An lse raised by delta for one query head scales that head's share of the saliency by exp(-delta):
+    the kernel takes the caller's statistics instead of recomputing them."""
+    import torch
+    rng = np.random.default_rng(17)
+    Hkv, G, d, T, W = 2, 4, 128, 3000, 64
+    K, Q = _rand_bits(rng, (Hkv, T, d)), _rand_bits(rng, (Hkv * G, W, d))
+    lse = O.window_row_lse(K, Q)
+    delta = 0.7
+    lse_shift = lse.copy()
+    lse_shift[5] += delta  # query head 5 = KV head 1, group member 1
+    sal = B.stepkv_score([TL.bf16_dev(K)], [TL.bf16_dev(Q)], T,
+                         lse=[torch.from_numpy(lse_shift.astype(np.float32)).cuda()])
+    torch.cuda.synchronize()
+    # the reference: head 5's rows weighted by exp(-delta) (the saliency rebuilt from the oracle's rows)
+    Kf, Qf = wl.bf16_bits_to_f32(K).astype(np.float64), wl.bf16_bits_to_f32(Q).astype(np.float64)
+    ref = np.zeros((Hkv, T))
+    for gq in range(Hkv * G):
+        for w in range(W):
+            vis = T - W + w + 1
+            s = Qf[gq, w] @ Kf[gq // G, :vis].T / np.sqrt(d)
+            ref[gq // G, :vis] += np.exp(s - lse_shift[gq, w]) / G
+    TL.assert_close(sal.cpu().numpy()[0], ref, "sal with a shifted lse")
+    assert abs(ref[1].sum() - (W * (G - 1) + W * np.exp(-delta)) / G) < 1e-6 * W
+
+
 # Observation-length windows (the queries are a whole last Observation, hundreds to 4096 tokens): the
 # window is split over up to 16 row groups per query head, GQA 4 and 5.
 LONG_WINDOW_CASES = [

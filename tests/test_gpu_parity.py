@@ -541,6 +541,26 @@ def test_compress_batched_ragged(B):
         assert np.array_equal(TL.bits_of(g.K_out[0])[:, :n], O.compact_rows(tr.keys(0), gk))
 
 
+def test_compress_batched_mixed_prefill_lse(B):
+    """Four ragged trajectories in one call, two with the prefill's row log-sum-exp and two without: the
+    saliency batches split by mode (one launch may not mix them) and every trajectory matches the oracle."""
+    import torch
+    trs = [wl.custom(120 + i, L=3, Hq=8, Hkv=2, d=128, T=T, W=32, n_steps=5 + i, budget=wl.Budget.ratio(1, 5))
+           for i, T in enumerate((1700, 2600, 999, 3100))]
+    gs = [TL.GpuTraj(tr) for tr in trs]
+    probs = [g.problem() for g in gs]
+    for i in (0, 1):
+        tr = trs[i]
+        probs[i].sal_lse = [torch.from_numpy(O.window_row_lse(tr.keys(l), tr.queries(l)).astype(np.float32)).cuda()
+                            for l in tr.sal_layer_ids()]
+        probs[i].refresh()
+    st = B.stepkv_compress(probs, B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    for g, tr in zip(gs, trs):
+        TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(B.Params())))
+
+
 @pytest.mark.parametrize("Hq,Hkv,W", [(10, 2, 128), (4, 2, 300)])
 def test_compress_batched_row_groups(B, Hq, Hkv, W):
     """Short trajectories whose query rows need several row groups (GQA 5 x W 128 = 640 rows; a

@@ -92,9 +92,8 @@ typedef struct {
   int32_t sal_pool; /* SnapKV-style token-axis pooling of each saliency row before the mean over rows
                        (Sec. 4.2: T_i from an existing estimator such as SnapKV): odd width k in
                        [1, STEPKV_MAX_POOL], 1 = none.  Window [i - k/2, i + k/2] clipped to [0, T).
-                       Taken by stepkv_select; stepkv_compress rejects k > 1 (EUNSUPPORTED): its
-                       saliency pass sums the rows on the fly, so pool through stepkv_score rows and
-                       stepkv_select instead */
+                       In stepkv_compress a width > 1 makes the saliency stage write its rows (one
+                       launch per trajectory) and pool them, instead of summing them on the fly */
   int32_t sal_pool_mode; /* STEPKV_POOL_MAX: maximum over the window; STEPKV_POOL_AVG: mean of the
                             window's in-range values */
 } stepkv_params_t;

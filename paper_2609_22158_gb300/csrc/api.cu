@@ -510,19 +510,28 @@ static size_t compress_traj_bytes(const stepkv_problem_t& p) {
   return align256((size_t)p.T * sizeof(unsigned long long)) + align256(select_ws_bytes(p.T, p.steps.n_steps)) +
          align256(compact_inplace_ws_bytes(p.T));
 }
+// Saliency rows of one trajectory, for a pooled token saliency (params.sal_pool > 1), which needs every
+// (layer, KV head) row before the mean: the row groups' rows, then (when there are several row groups)
+// their per-(layer, KV head) sums.  One region, reused trajectory after trajectory.
+static size_t compress_rows_bytes(const stepkv_problem_t& p) {
+  const int Ls = std::min(p.n_sal_layers, p.L);
+  const int n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
+  return align256((size_t)Ls * p.Hkv * (n_rg + (n_rg > 1 ? 1 : 0)) * p.T * sizeof(float));
+}
 
 size_t stepkv_compress_workspace_size(const stepkv_problem_t* probs, int32_t n_traj) {
   if (!probs || n_traj < 1) return 0;
-  size_t part = 0, per = 0;
+  size_t part = 0, per = 0, rows = 0;
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     if (p.L < 1 || p.Hkv < 1 || p.Hq < p.Hkv || p.T < 1 || p.W < 1 || p.n_sal_layers < 1 || p.steps.n_steps < 1)
       return 0;
     per += compress_traj_bytes(p);
+    rows = std::max(rows, compress_rows_bytes(p));
   }
   for (const SalBatch& b : saliency_batches(probs, n_traj))
     part = std::max(part, compress_part_bytes(probs[b.first], b.n));
-  return part + per;
+  return part + per + rows;
 }
 
 stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, const stepkv_params_t* params,
@@ -542,8 +551,6 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     if (st != STEPKV_OK) return st;
     st = check_select_args(Ls * p.Hkv, p.T, p.step_id, p.prot, &p.steps, params, &p.budget, &p.sel);
     if (st != STEPKV_OK) return st;
-    // the fused saliency pass sums the rows as it goes: pooling needs the rows (stepkv_score + stepkv_select)
-    if (params->sal_pool > 1) return STEPKV_EUNSUPPORTED;
     if (p.sal_lse) {
       for (int l = 0; l < Ls; ++l)
         if (!p.sal_lse[l] || (reinterpret_cast<uintptr_t>(p.sal_lse[l]) & 3u) != 0) return STEPKV_EINVAL;
@@ -570,6 +577,11 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   std::vector<SelectSpec> specs((size_t)n_traj);
   std::vector<void*> plan_ws((size_t)n_traj);
   std::vector<ScoreTrajSpec> sal((size_t)n_traj);
+  // a pooled token saliency (SnapKV-style) needs every (layer, KV head) row before the mean, so the
+  // saliency stage writes rows per trajectory and a pooling launch forms T; the fixed-point token sums of
+  // the fused saliency pass are not used then (their region holds the float T instead)
+  const bool pooled = params->sal_pool > 1;
+  std::vector<float*> t_float((size_t)n_traj);
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     const int Ls = std::min(p.n_sal_layers, p.L);
@@ -580,21 +592,38 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     const int n_pairs = Ls * p.Hkv;
     const int shift = score_acc_shift(n_pairs, p.W);
     sal[i] = ScoreTrajSpec{sal_keys(p), p.Q, p.T, t_acc, p.kv_head_stride, p.q_head_stride, p.sal_lse};
-    specs[i] = SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot, p.steps,
-                          *params, p.budget, p.sel, sel_ws, dev_status};
+    t_float[i] = reinterpret_cast<float*>(t_acc);
+    specs[i] = pooled ? SelectSpec{t_float[i], nullptr, 0.0, p.T, p.step_id, p.prot, p.steps, *params, p.budget,
+                                   p.sel, sel_ws, dev_status}
+                      : SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot,
+                                   p.steps, *params, p.budget, p.sel, sel_ws, dev_status};
   }
+  float* rows_ws = reinterpret_cast<float*>(w);  // compress_rows_bytes of the largest trajectory
   // optional stage timing (profiling): caller-owned events recorded on the stream of this call
   const StageEvents ev = t_stage_events;
   if (ev.e[0]) {
     const cudaError_t er = cudaEventRecord(ev.e[0], s);
     if (er != cudaSuccess) { set_last_cuda_error(er); return STEPKV_ECUDA; }
   }
-  // stage 1: one cooperative launch per saliency batch
-  for (const SalBatch& b : batches) {
+  // stage 1: one cooperative launch per saliency batch (pooled: per trajectory, rows then the pooled mean)
+  for (const SalBatch& b : (pooled ? std::vector<SalBatch>{} : batches)) {
     const stepkv_problem_t& p = probs[b.first];
     const int Ls = std::min(p.n_sal_layers, p.L);
     stepkv_status_t st = score_run_batch(Ls, &sal[b.first], b.n, p.Hkv, p.Hq, p.d, p.W, nullptr, 0,
                                          score_acc_shift(Ls * p.Hkv, p.W), part, dev_status, s);
+    if (st != STEPKV_OK) return st;
+  }
+  for (int i = 0; pooled && i < n_traj; ++i) {
+    const stepkv_problem_t& p = probs[i];
+    const int Ls = std::min(p.n_sal_layers, p.L);
+    const int n_pairs = Ls * p.Hkv, n_rg = score_row_groups(p.Hkv, p.Hq, p.W);
+    float* sal_rows = n_rg > 1 ? rows_ws + (size_t)n_pairs * n_rg * p.T : rows_ws;
+    stepkv_status_t st = score_run(Ls, sal_keys(p), p.kv_head_stride, p.Q, p.q_head_stride, p.Hkv, p.Hq, p.d, p.T,
+                                   p.W, rows_ws, p.T, nullptr, 0, part, dev_status, s, 0, p.sal_lse);
+    if (st == STEPKV_OK && n_rg > 1) st = score_sum_row_groups(rows_ws, n_pairs, n_rg, p.T, sal_rows, s);
+    if (st == STEPKV_OK)
+      st = pool_mean_rows_run(sal_rows, n_pairs, p.T, 1.0f / (float)n_pairs, p.T, params->sal_pool / 2,
+                              params->sal_pool_mode == STEPKV_POOL_MAX, t_float[i], s);
     if (st != STEPKV_OK) return st;
   }
   // stages 2-4 for all trajectories in one launch (one cluster per trajectory)

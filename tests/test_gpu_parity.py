@@ -364,13 +364,26 @@ def test_select_snapkv_pooling(B, pool, mode, T):
     TL.check_select_outputs(g, out)
 
 
-def test_compress_rejects_pooling(B):
-    """The fused pass sums the saliency rows as it goes, so it refuses a pooling width (EUNSUPPORTED)."""
-    tr = wl.custom(5, L=2, Hq=8, Hkv=2, d=64, T=1200, W=16, n_steps=6, budget=wl.Budget.ratio(1, 4))
+@pytest.mark.parametrize("pool, mode, W, lse", [(7, 0, 64, False), (5, 1, 64, True), (3, 0, 128, False)])
+def test_compress_with_snapkv_pooling(B, pool, mode, W, lse):
+    """The fused pass with a pooled token saliency: the saliency rows are written and pooled per
+    trajectory (with and without the prefill's row statistics; W = 128 at GQA 4 takes two row groups)."""
+    import torch
+    tr = wl.custom(60 + pool, L=4, Hq=16, Hkv=4, d=128, T=5000, W=W, n_steps=12, budget=wl.Budget.ratio(1, 8))
     g = TL.GpuTraj(tr)
-    with pytest.raises(B.StepKVError) as e:
-        B.stepkv_compress([g.problem()], B.Params(sal_pool=3))
-    assert e.value.code == B.STEPKV_EUNSUPPORTED
+    prob = g.problem()
+    if lse:
+        prob.sal_lse = [torch.from_numpy(O.window_row_lse(tr.keys(l), tr.queries(l)).astype(np.float32)).cuda()
+                        for l in tr.sal_layer_ids()]
+        prob.refresh()
+    p = B.Params(sal_pool=pool, sal_pool_mode=mode)
+    st = B.stepkv_compress([prob], p)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(p)))
+    n = int(g.out.n_kept.item())
+    kt = g.out.kept_idx[:n].long()
+    assert torch.equal(g.K_out[0][:, :n], g.K[0].index_select(1, kt))
 
 
 def test_select_large_T(B):

@@ -410,7 +410,9 @@ STEPKV_API stepkv_status_t stepkv_selftest_score_timeout(int32_t n_layers, const
  * the saliency of each trajectory (one launch each), then the selections of all trajectories in one
  * launch (one 8-CTA cluster per trajectory, up to 16 per launch), then each compaction.  `ws` (size
  * from stepkv_compress_workspace_size over the same array) holds one shared region for the saliency
- * partials and a private region per trajectory.  Caches in host memory (kv_location / out_location
+ * partials, a private region per trajectory, and one shared region for the saliency rows of a pooled
+ * token saliency (params->sal_pool > 1: the rows of each trajectory are written, then pooled; the
+ * region is sized for the largest trajectory whatever the params).  Caches in host memory (kv_location / out_location
  * STEPKV_MEM_HOST) are read and written in place over the CPU-GPU link by the compaction kernels;
  * their pointers are checked on the host before anything is enqueued.
  */

@@ -915,12 +915,15 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4096, n_dec=64, seed=5):
+def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4096, n_dec=64, seed=5,
+                    stage_events=False):
     """Boundaries of the incremental loop on device-random K/V/Q (layout and signals from the seeded
     generator).  The cache lives in one capacity buffer per layer and is compacted in place (hole filling);
     each new step is appended after the retained rows.  Events time each compression and each group of
     n_dec decode reads.  With growth_total, the new steps' lengths are rescaled to add that many tokens
-    over the loop."""
+    over the loop.  With stage_events, stepkv_compress also records events between its selection and its
+    compaction (which keeps the compaction from starting early under programmatic dependent launch), and
+    the loop reports the time of each stage instead of timing the plain call."""
     import numpy as np
     import torch
     from paper_2609_22158_gb300 import binding as B, workload as wl
@@ -938,7 +941,10 @@ def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4
     reuse = np.zeros(n_steps, np.float32)
     params = B.Params()
     status = B.new_status(dev)
-    comp_us, dec_us, rows, moved = [], [], [], []
+    comp_us, dec_us, rows, moved, sel_us, cpt_us = [], [], [], [], [], []
+    sev = tuple(torch.cuda.Event(enable_timing=True) for _ in range(3))  # stage split inside each compression
+    for e_ in sev:
+        e_.record(stream)  # torch creates an event at its first record
     ws = torch.empty(64 << 20, dtype=torch.uint8, device=dev)
     ws_d = torch.empty(B.load_library().stepkv_decode_workspace_size(s.L, s.Hkv, s.Hq, s.d, cap) + 512,
                        dtype=torch.uint8, device=dev)
@@ -978,9 +984,13 @@ def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4
         torch.cuda.synchronize()
         torch.cuda._sleep(300_000)  # the device stays busy while the host prepares the call
         e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        if stage_events:
+            B.set_stage_events(*sev)
         e[0].record(stream)
         B.stepkv_compress([prob], params, ws=ws, status=status, stream=stream)
         e[1].record(stream)
+        if stage_events:
+            B.set_stage_events()
         for _ in range(n_dec):
             B.stepkv_decode(qd, live_K, live_V, out.n_kept, out=outd, ws=ws_d, status=status, stream=stream)
         e[2].record(stream)
@@ -992,6 +1002,9 @@ def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4
         rows.append(T)
         moved.append(int((kept >= n).sum()))
         comp_us.append(e[0].elapsed_time(e[1]) * 1e3)
+        if stage_events:
+            sel_us.append(sev[0].elapsed_time(sev[1]) * 1e3)
+            cpt_us.append(sev[1].elapsed_time(sev[2]) * 1e3)
         dec_us.append(e[1].elapsed_time(e[2]) * 1e3 / n_dec)
         step_id = sid_out[:n].cpu().numpy()
         pos = pos_out[:n].cpu().numpy()
@@ -1015,6 +1028,8 @@ def run_incremental(n_boundaries, s, dev, stream, peaks, growth_total=None, t0=4
             "cache_rows_mean": round(mean(rows), 1), "rows_moved_mean": round(mean(moved), 1),
             "compress_us_mean": round(mean(comp_us), 2),
             "compress_us_p50_p90": [round(float(np.percentile([comp_us[i] for i in pick], q)), 2) for q in (50, 90)],
+            "compress_stage_us_mean": ({"score_select": round(mean(sel_us), 2), "compact_in_place": round(mean(cpt_us), 2)}
+                                       if stage_events else None),
             "compress_algorithmic_bytes_mean": int(mean(alg)),
             "compress_achieved_gbs": round(gbs, 1), "compress_frac_of_measured_hbm": round(gbs / peaks["hbm"], 4),
             "decode_us_per_token_mean": round(mean(dec_us), 2),
@@ -1037,6 +1052,11 @@ def run_config5(args, world, rank, local, dist, dev, peaks):
     clocks = sampler.stop() if sampler else None
     if rank != 0:
         return
+    split = run_incremental(args.inc_boundaries_cfg5, s, dev, stream, peaks, growth_total=131072 - 4096, n_dec=4,
+                            stage_events=True)
+    inc["compress_stage_us_mean"] = split["compress_stage_us_mean"]
+    inc["compress_stage_note"] = ("a second run of the same loop (same seeds, 4 decode reads per boundary) with "
+                                  "events between selection and compaction, outside the timed loop")
     value = inc["tokens_compressed"] / (inc["compress_us_total"] * 1e-6)
     ms = inc["compress_us_total"] / inc["boundaries"] / 1e3
     roof = {"kernel": "fused in-place boundary (score + select + hole-filling compaction)", "bound": "hbm",

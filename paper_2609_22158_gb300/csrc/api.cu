@@ -539,6 +539,7 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
   if (!probs || n_traj < 1 || !params || !ws) return STEPKV_EINVAL;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return STEPKV_EINVAL;
   // validate everything before enqueueing anything
+  std::vector<char> in_place((size_t)n_traj, 0);
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
     if (p.L < 1 || p.n_sal_layers < 1) return STEPKV_EINVAL;
@@ -560,6 +561,7 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
                             p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
     if (st != STEPKV_OK) return st;
     if (inplace && p.kv_location != p.out_location) return STEPKV_EINVAL;
+    in_place[i] = inplace ? 1 : 0;
   }
   // cache pointers as the kernels see them (host-resident caches: checked and translated here)
   std::vector<CachePtrs> caches((size_t)n_traj);
@@ -597,6 +599,12 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
                                    p.sel, sel_ws, dev_status}
                       : SelectSpec{nullptr, t_acc, ldexp(1.0, -shift) / (double)n_pairs, p.T, p.step_id, p.prot,
                                    p.steps, *params, p.budget, p.sel, sel_ws, dev_status};
+    if (in_place[i]) {  // the selection also writes the hole-filling plan and the in-place rows' metadata
+      specs[i].plan = static_cast<int32_t*>(plan_ws[i]);
+      specs[i].pos_in = p.pos_in;
+      specs[i].step_id_out = p.step_id_out;
+      specs[i].pos_out = p.pos_out;
+    }
   }
   float* rows_ws = reinterpret_cast<float*>(w);  // compress_rows_bytes of the largest trajectory
   // optional stage timing (profiling): caller-owned events recorded on the stream of this call
@@ -633,16 +641,13 @@ stepkv_status_t stepkv_compress(const stepkv_problem_t* probs, int32_t n_traj, c
     const cudaError_t er = cudaEventRecord(ev.e[1], s);  // the compaction is launched plainly after it
     if (er != cudaSuccess) { set_last_cuda_error(er); return STEPKV_ECUDA; }
   }
-  // stage 5: in place by hole filling where the outputs are the inputs (one plan and one move launch per
-  // trajectory), the rest out of place, sharing launches
+  // stage 5: in place by hole filling where the outputs are the inputs (one move launch per trajectory,
+  // following the plan its selection wrote), the rest out of place, sharing launches
   std::vector<CompactSpec> outs;
   for (int i = 0; i < n_traj; ++i) {
     const stepkv_problem_t& p = probs[i];
-    bool inplace = false;
-    check_compact_args(p.L, p.K, p.V, p.kv_head_stride, p.Hkv, p.d, p.T, p.sel.kept_idx, p.sel.n_kept,
-                       p.sel.kept_cap, p.K_out, p.V_out, p.out_head_stride, &inplace);
     const CachePtrs& c = caches[i];
-    if (inplace) {
+    if (in_place[i]) {
       st = compact_inplace_run(p.L, c.K_out.data(), c.V_out.data(), p.kv_head_stride, p.Hkv, p.d, p.T,
                                p.sel.kept_idx, p.sel.n_kept, p.sel.kept_cap, p.step_id, p.pos_in, p.step_id_out,
                                p.pos_out, plan_ws[i], dev_status, s);

@@ -19,7 +19,8 @@ constexpr int kCompactCtasPerSm = 8;
 constexpr int kCompactUnroll = 4;
 constexpr int kCompactLayersPerLaunch = 96;
 
-// The in-place move kernel's arguments: the row sets of up to kCompactLayersPerLaunch layers.
+// The in-place move kernel's arguments: the row sets of up to kCompactLayersPerLaunch layers and the plan
+// the selection kernel wrote.
 struct CompactMoveArgs {
   uint8_t* dst[2 * kCompactLayersPerLaunch];  // per (layer, tensor): base of [Hkv][rows][d]
   int n_sets;               // n_layers_in_launch * n_tensors * Hkv
@@ -27,6 +28,16 @@ struct CompactMoveArgs {
   int row_bytes;            // d * 2
   int64_t out_head_bytes;
   int T;
+  int kept_cap;
+  const int32_t* plan;      // plan[0] = holes H, plan[1 + j] = hole j (ascending)
+  const int32_t* kept_idx;  // the j-th mover is kept_idx[n_kept - H + j]
+  const int32_t* n_kept;
+  const int32_t* step_id_in;  // metadata of the filled holes (first launch of a trajectory only)
+  const int32_t* pos_in;
+  int32_t* step_id_out;
+  int32_t* pos_out;
+  int meta;
+  int32_t* status;
 };
 
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
@@ -174,62 +185,33 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(const __grid_c
 // receives one retained row from a slot at or above n (a mover), the j-th hole the j-th mover.  Sources
 // (>= n) and destinations (< n) never overlap, so all moves run in parallel.  Rows [0, n) then hold the
 // retained set, no longer in slot order; step_id_out / pos_out record each row's step and original
-// position.  Only the movers are read and written, instead of every retained row.
+// position.  Only the movers are read and written, instead of every retained row.  The selection kernel
+// lays out the plan as it writes kept_idx (the number of a hole is its slot minus the retained slots below
+// it, which that pass counts anyway), so the moves need no launch of their own to find it.
 
-__device__ __forceinline__ int lower_bound_i32(const int32_t* a, int n, int x) {
-  int lo = 0, hi = n;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (__ldg(&a[mid]) < x) lo = mid + 1; else hi = mid;
-  }
-  return lo;
-}
-
-// Plan: plan[0] = number of moves; hole[j], mover[j]; and the step/position metadata of rows [0, n).
-__global__ void __launch_bounds__(kCompactThreads) compact_plan_kernel(
-    const int32_t* kept_idx, const int32_t* n_kept_p, int kept_cap, int T, const int32_t* step_id_in,
-    const int32_t* pos_in, int32_t* step_id_out, int32_t* pos_out, int32_t* plan, int32_t* status) {
+__global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __grid_constant__ CompactMoveArgs a) {
   pdl_wait();
   pdl_launch_dependents();
-  const int n = *n_kept_p;
-  if (n > kept_cap || n < 0 || n > T) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) {
-      record_status(status, STEPKV_ENOSPACE);
-      plan[0] = 0;
-    }
+  const int n = __ldcg(a.n_kept);
+  if (n < 0 || n > a.kept_cap || n > a.T) return;  // the selection has recorded the error; nothing moves
+  const int n_moves = __ldcg(a.plan);
+  if (n_moves < 0 || n_moves > n) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) record_status(a.status, STEPKV_EDATA);
     return;
   }
-  const int m0 = lower_bound_i32(kept_idx, n, n);  // retained slots below n: kept_idx[0..m0)
-  if (blockIdx.x == 0 && threadIdx.x == 0) plan[0] = n - m0;
-  int32_t* hole = plan + 1;
-  int32_t* mover = plan + 1 + T;
-  for (int r = blockIdx.x * kCompactThreads + threadIdx.x; r < n; r += gridDim.x * kCompactThreads) {
-    const int c = lower_bound_i32(kept_idx, m0, r);  // retained slots below r
-    int src;
-    if (c < m0 && __ldg(&kept_idx[c]) == r) {
-      src = r;
-    } else {
-      const int j = r - c;  // holes below r
-      src = __ldg(&kept_idx[m0 + j]);
-      if (src < n || src >= T) {
-        record_status(status, STEPKV_EDATA);
-        src = r;
+  const int m0 = n - n_moves;  // the movers are kept_idx[m0 .. n), the retained slots at or above n
+  const int32_t* hole = a.plan + 1;
+  if (a.meta) {
+    for (int j = blockIdx.x * kCompactThreads + threadIdx.x; j < n_moves; j += gridDim.x * kCompactThreads) {
+      const int r = __ldcg(&hole[j]), src = __ldcg(&a.kept_idx[m0 + j]);
+      if (r < 0 || r >= n || src < n || src >= a.T) {
+        record_status(a.status, STEPKV_EDATA);
+        continue;
       }
-      hole[j] = r;
-      mover[j] = src;
+      if (a.step_id_out) a.step_id_out[r] = a.step_id_in ? __ldg(&a.step_id_in[src]) : -1;
+      if (a.pos_out) a.pos_out[r] = a.pos_in ? __ldg(&a.pos_in[src]) : src;
     }
-    if (step_id_out) step_id_out[r] = step_id_in ? step_id_in[src] : -1;
-    if (pos_out) pos_out[r] = pos_in ? pos_in[src] : src;
   }
-}
-
-__global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __grid_constant__ CompactMoveArgs a,
-                                                                       const int32_t* plan) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int n_moves = *plan;
-  const int32_t* hole = plan + 1;
-  const int32_t* mover = plan + 1 + a.T;
   const int64_t total = (int64_t)a.n_sets * n_moves;
   const int64_t per_cta = (total + gridDim.x - 1) / gridDim.x;
   const int64_t lo = blockIdx.x * per_cta;
@@ -250,11 +232,14 @@ __global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __g
       if (lane_active && ri < hi) {
         const int set = (int)(ri / n_moves);
         const int j = (int)(ri - (int64_t)set * n_moves);
-        const int src_row = __ldg(&mover[j]), dst_row = __ldg(&hole[j]);
-        const int lt = set / a.Hkv, h = set - lt * a.Hkv;
-        uint8_t* head = a.dst[lt] + (int64_t)h * a.out_head_bytes;
-        buf[u] = ld_stream(reinterpret_cast<const uint4*>(head + (int64_t)src_row * a.row_bytes) + col);
-        dptr[u] = reinterpret_cast<uint4*>(head + (int64_t)dst_row * a.row_bytes) + col;
+        // written by the selection kernel (programmatic dependent launch): read through L2
+        const int src_row = __ldcg(&a.kept_idx[m0 + j]), dst_row = __ldcg(&hole[j]);
+        if (src_row >= n && src_row < a.T && dst_row >= 0 && dst_row < n) {
+          const int lt = set / a.Hkv, h = set - lt * a.Hkv;
+          uint8_t* head = a.dst[lt] + (int64_t)h * a.out_head_bytes;
+          buf[u] = ld_stream(reinterpret_cast<const uint4*>(head + (int64_t)src_row * a.row_bytes) + col);
+          dptr[u] = reinterpret_cast<uint4*>(head + (int64_t)dst_row * a.row_bytes) + col;
+        }
       }
     }
 #pragma unroll
@@ -263,19 +248,19 @@ __global__ void __launch_bounds__(kCompactThreads) compact_move_kernel(const __g
   }
 }
 
-size_t compact_inplace_ws_bytes(int T) { return (size_t)(1 + 2 * (size_t)T) * sizeof(int32_t); }
+size_t compact_inplace_ws_bytes(int T) { return (size_t)(1 + (size_t)T) * sizeof(int32_t); }
 
 stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V, int64_t head_stride, int Hkv, int d,
                                     int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,
                                     const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
                                     int32_t* pos_out, void* ws, int32_t* status, cudaStream_t stream) {
-  int32_t* plan = static_cast<int32_t*>(ws);
+  static int resident = 0;  // move-kernel CTAs resident per SM (registers bound it): one wave of them
   int n_sm = 0;
   cudaError_t e = device_sm_count(&n_sm);
-  if (e == cudaSuccess) {
-    const int blocks = std::max(1, std::min((std::max(kept_cap, 1) + kCompactThreads - 1) / kCompactThreads, n_sm * 4));
-    e = launch_kernel(compact_plan_kernel, dim3(blocks), dim3(kCompactThreads), 0, stream, kept_idx, n_kept, kept_cap,
-                      T, step_id_in, pos_in, step_id_out, pos_out, plan, status);
+  if (e == cudaSuccess && resident == 0) {
+    int r = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&r, compact_move_kernel, kCompactThreads, 0);
+    resident = std::max(1, std::min(r, kCompactCtasPerSm));
   }
   const int n_tensors = V ? 2 : 1;
   for (int l0 = 0; e == cudaSuccess && l0 < std::max(n_layers, 1); l0 += kCompactLayersPerLaunch) {
@@ -292,11 +277,21 @@ stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V
     a.row_bytes = d * 2;
     a.out_head_bytes = head_stride * 2;
     a.T = T;
-    const int64_t rows_max = (int64_t)a.n_sets * std::max(std::min(kept_cap, T - 1), 1);
+    a.kept_cap = kept_cap;
+    a.plan = static_cast<const int32_t*>(ws);
+    a.kept_idx = kept_idx;
+    a.n_kept = n_kept;
+    a.step_id_in = step_id_in;
+    a.pos_in = pos_in;
+    a.step_id_out = step_id_out;
+    a.pos_out = pos_out;
+    a.meta = l0 == 0;
+    a.status = status;
+    // moves: at most min(n_kept, T - n_kept) <= T / 2 rows per set
+    const int64_t rows_max = (int64_t)a.n_sets * std::max(std::min(kept_cap, T / 2), 1);
     const int64_t want = (rows_max + 31) / 32;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * kCompactCtasPerSm, want));
-    e = launch_kernel(compact_move_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a,
-                      static_cast<const int32_t*>(plan));
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)n_sm * resident, want));
+    e = launch_kernel(compact_move_kernel, dim3(grid), dim3(kCompactThreads), 0, stream, a, true);
   }
   if (e != cudaSuccess) {
     set_last_cuda_error(e);

@@ -139,6 +139,12 @@ struct SelectSpec {
   stepkv_select_out_t out;
   void* ws;          // select_ws_bytes(T, n_steps), 256-byte aligned, private to this trajectory
   int32_t* status;
+  // in-place compaction: the selection also writes the hole-filling plan (compact_inplace_ws_bytes(T))
+  // and the step id / position of the rows retained in place
+  int32_t* plan = nullptr;
+  const int32_t* pos_in = nullptr;
+  int32_t* step_id_out = nullptr;
+  int32_t* pos_out = nullptr;
 };
 // Independent trajectories in as few launches as possible (one cluster each).
 stepkv_status_t select_run_batch(const SelectSpec* specs, int n, cudaStream_t stream);
@@ -181,7 +187,9 @@ stepkv_status_t compact_run(int n_layers, const void* const* K_in, const void* c
                             const int32_t* step_id_in, const int32_t* pos_in, int32_t* step_id_out,
                             int32_t* pos_out, int32_t* status, cudaStream_t stream);
 
-// In place (K_out == K): hole filling; ws holds the move plan (compact_inplace_ws_bytes(T)).
+// In place (K_out == K): hole filling, following the plan the selection kernel wrote into ws
+// (compact_inplace_ws_bytes(T), SelectSpec::plan); the move kernel also writes the step id / position of
+// every filled hole.
 size_t compact_inplace_ws_bytes(int T);
 stepkv_status_t compact_inplace_run(int n_layers, void* const* K, void* const* V, int64_t head_stride, int Hkv, int d,
                                     int T, const int32_t* kept_idx, const int32_t* n_kept, int kept_cap,

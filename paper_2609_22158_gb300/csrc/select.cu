@@ -51,6 +51,14 @@ struct SelectArgs {
   uint32_t* acc_max;
   int32_t* acc_kept;
   int32_t* status;
+  // In-place compaction by hole filling (NULL plan: none).  The write pass also lays out the plan the move
+  // kernel follows: plan[0] = number of holes H (slots below n_kept that are not retained), plan[1 + j] =
+  // the j-th hole in slot order; the j-th mover is kept_idx[n_kept - H + j].  Rows retained in place get
+  // their step id / position here; the move kernel writes those of the filled holes.
+  int32_t* plan;
+  const int32_t* pos_in;
+  int32_t* step_id_out;
+  int32_t* pos_out;
 };
 
 // Exchange block shared by the cluster (read remotely through DSMEM).
@@ -278,6 +286,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       if (a.steps.reuse_out) a.steps.reuse_out[k] = c;
     }
   }
+  if (a.plan && rank == 0 && tid == 0) a.plan[0] = 0;  // hole count, summed after barrier (B)
   for (int k = rank * NT + tid; k < n_steps; k += NC * NT) {
     a.acc_cnt[k] = 0;
     a.acc_sum[k] = 0ull;
@@ -616,6 +625,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
     int tie_rank = ties_before + eq_before;                                 // cluster-wide tie rank
     int out_pos = out_off + strict_before + min(granted_cta, eq_before);   // next output slot
     int run_sid = -1, run_c = 0;
+    int holes = 0;  // in-place plan: holes among this lane's slots
     for (int i0 = s0; i0 < s1; i0 += 32) {
       const int i = i0 + lane;
       const bool in = i < s1;
@@ -627,7 +637,18 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       const unsigned em = __ballot_sync(0xffffffffu, is_eq);
       const bool keep = in && (pr || k > kth || (is_eq && tie_rank + __popc(em & lt) < need_eq));
       const unsigned km = __ballot_sync(0xffffffffu, keep);
-      if (keep) a.out.kept_idx[out_pos + __popc(km & lt)] = base + i;
+      const int kept_before = out_pos + __popc(km & lt);  // retained slots below this one, cluster-wide
+      if (keep) a.out.kept_idx[kept_before] = base + i;
+      if (a.plan && in && base + i < total_kept) {
+        const int gi = base + i;
+        if (keep) {  // retained in place
+          if (a.step_id_out) a.step_id_out[gi] = __ldg(&a.step_id[gi]);
+          if (a.pos_out) a.pos_out[gi] = a.pos_in ? __ldg(&a.pos_in[gi]) : gi;
+        } else {     // hole number gi - kept_before, filled by the mover of that number
+          a.plan[1 + gi - kept_before] = gi;
+          ++holes;
+        }
+      }
       out_pos += __popc(km);
       tie_rank += __popc(em);
       if (want_kept && keep && !pr) {
@@ -640,6 +661,10 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       }
     }
     step_stat_flush(run_c > 0, run_sid, run_c, 0ull, 0u, a.acc_kept, nullptr, nullptr);
+    if (a.plan) {
+      for (int o = 16; o > 0; o >>= 1) holes += __shfl_xor_sync(0xffffffffu, holes, o);
+      if (lane == 0 && holes) atomicAdd(&a.plan[0], holes);
+    }
   }
   if (want_stats || want_kept) {
     cl.sync();  // (C) all step accumulators final
@@ -775,6 +800,10 @@ static SelectArgs make_select_args(const SelectSpec& sp) {
   w += align256(n * 4);
   a.acc_kept = reinterpret_cast<int32_t*>(w);
   a.status = sp.status;
+  a.plan = sp.plan;
+  a.pos_in = sp.pos_in;
+  a.step_id_out = sp.step_id_out;
+  a.pos_out = sp.pos_out;
   return a;
 }
 

@@ -626,6 +626,44 @@ def test_compress_twenty_trajectories_mixed_in_place(B):
             assert np.array_equal(TL.bits_of(g.V[0])[:, :n], sv[1][0][:, srcs])
 
 
+@pytest.mark.parametrize("T,num,den,all_prot", [(20000, 1, 2, False), (9000, 9, 10, False), (5000, 1, 20, False),
+                                               (3000, 1, 4, True)])
+def test_compress_in_place_hole_filling(B, T, num, den, all_prot):
+    """In-place compaction by hole filling, with a retained set spanning several 4096-row plan chunks, few
+    holes, a short retained set and nothing to move: the retained set matches the oracle, every slot below
+    n_kept that is retained stays in place, the j-th hole receives the j-th retained slot at or above
+    n_kept, and every layer's K and V rows and the step / position metadata follow that plan exactly."""
+    import torch
+    tr = wl.custom(900 + T, L=3, Hq=4, Hkv=2, d=64, T=T, W=16, n_steps=14, budget=wl.Budget.ratio(num, den))
+    if all_prot:
+        tr.prot = np.ones(tr.T, np.uint8)
+    g = TL.GpuTraj(tr)
+    src = ([TL.bits_of(k) for k in g.K], [TL.bits_of(v) for v in g.V])
+    g.problem()
+    prob = B.Problem(g.K, g.V, g.Q, tr.T, g.step_id, g.prot, g.steps(), g.budget(), g.K, g.V, g.out,
+                     pos_in=g.pos, step_id_out=g.step_id_out, pos_out=g.pos_out)
+    st = B.stepkv_compress([prob], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    TL.check_select_outputs(g, TL.run_oracle(tr, TL.oracle_params(B.Params())))
+    n = int(g.out.n_kept.item())
+    gk = g.out.kept_idx[:n].cpu().numpy().astype(np.int64)
+    in_place = np.zeros(n, bool)
+    in_place[gk[gk < n]] = True
+    holes = np.flatnonzero(~in_place)
+    movers = gk[gk >= n]
+    assert len(holes) == len(movers)
+    if all_prot:
+        assert n == tr.T and len(holes) == 0
+    exp = np.arange(n)
+    exp[holes] = movers
+    assert np.array_equal(g.pos_out[:n].cpu().numpy(), tr.pos[exp])
+    assert np.array_equal(g.step_id_out[:n].cpu().numpy(), tr.step_id[exp])
+    for l in range(tr.shape.L):
+        assert np.array_equal(TL.bits_of(g.K[l])[:, :n], src[0][l][:, exp])
+        assert np.array_equal(TL.bits_of(g.V[l])[:, :n], src[1][l][:, exp])
+
+
 def test_compress_minimal_outputs_same_selection(B):
     """Without the optional outputs (per-step statistics, priorities) the kernel skips their work; the
     retained set and the compacted rows are the same as with every output requested."""

@@ -491,29 +491,41 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
       };
       // pass 1: S = Q K^T, one half per 128-row query tile, N = the item's keys (256 or 128)
       int slot = 0;
+      // This thread's work between two MMA groups is on the tensor pipe's critical path: it shares its
+      // scheduler with four epilogue warps that issue back to back.  So the unit, its rows and the
+      // instruction descriptors are worked out only where the unit changes, and every operand
+      // descriptor is one of two bases plus a constant offset (the 14-bit start-address field holds
+      // address / 16 of a shared-memory window below 256 KB, so adding offset / 16 never carries out).
+      const uint64_t dK0 = umma_desc_sw128(smem_u32(sK)), dQ0 = umma_desc_sw128(qst);
+      int t_unit_end = -1;  // pass 1: first item after the current unit
+      int n_mt = 1;
       for (int t = p.pass2_only ? t_hi : t_lo; t < t_hi && ok;) {
-        const ItemLoc il = locate(p, t);
-        const int nt = item_tiles(il, t);
-        const int u = il.u;
-        const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
-        if (!(ok = new_unit(u))) break;
+        if (t >= t_unit_end) {
+          const ItemLoc il = locate(p, t);
+          const RowGroup r = row_group(g, fmodulo(il.u, g.rg_div));
+          if (!(ok = new_unit(il.u))) break;
+          n_mt = r.rows > 128 ? 2 : 1;
+          t_unit_end = t - il.tile + p.traj[il.b].n_tiles;
+        }
+        const int nt = (t + 1 < t_hi && t + 1 < t_unit_end) ? 2 : 1;
         for (int i = 0; i < nt && ok; ++i) {
           const int st = 2 * slot + i;
           ok = mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag);
         }
         if (!ok) break;
         tc_fence_after();
-        const int n_mt = r.rows > 128 ? 2 : 1;
-        const uint32_t idesc = umma_idesc_bf16(128, nt * kKeyTile);
+        const uint32_t idesc = nt == 2 ? umma_idesc_bf16(128, 2 * kKeyTile) : umma_idesc_bf16(128, kKeyTile);
+        const uint64_t dK = dK0 + (uint64_t)(Cfg::chunk_off(2 * slot, 0) >> 4);
         for (int mt = 0; mt < n_mt && ok; ++mt) {
           int b;
           if (!(ok = take_buffer(b))) break;
           const uint32_t dcol = tmem_base + (uint32_t)(b * 256);
+          const uint64_t dQ = dQ0 + (uint64_t)((mt * 128 * 128) >> 4);
 #pragma unroll
           for (int kk = 0; kk < NCH * 4; ++kk) {
-            const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + mt * 128 * 128 + (kk & 3) * 32);
-            const uint32_t koff = (uint32_t)(Cfg::chunk_off(2 * slot, kk >> 2) + (kk & 3) * 32);
-            umma_bf16(dcol, umma_desc_sw128(qst + qoff), umma_desc_sw128(smem_u32(sK) + koff), idesc, kk > 0 ? 1u : 0u);
+            const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + (kk & 3) * 32);
+            const uint32_t koff = (uint32_t)((kk >> 2) * 2 * kKChunkBytes + (kk & 3) * 32);  // within the slot
+            umma_bf16(dcol, dQ + (qoff >> 4), dK + (koff >> 4), idesc, kk > 0 ? 1u : 0u);
           }
           give_buffer(b);
         }
@@ -527,23 +539,28 @@ __global__ void __launch_bounds__(kThreads, 1) score_kernel(const __grid_constan
         if (++slot == P1) slot = 0;
       }
       // pass 2: S^T = K Q^T, the tile's keys on M, the query rows on N
+      int k_unit_end = 0;  // pass 2: first item (in pass-2 order) after the current unit
+      uint32_t idesc2 = 0;
       for (int k = 0; k < n1 && ok; ++k) {
-        const int u = locate(p, t_hi - 1 - k).u;
-        const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
-        if (!(ok = new_unit(u))) break;
+        if (k == k_unit_end) {
+          const int u = locate(p, t_hi - 1 - k).u;
+          const RowGroup r = row_group(g, fmodulo(u, g.rg_div));
+          if (!(ok = new_unit(u))) break;
+          idesc2 = umma_idesc_bf16(128, (r.rows + 31) & ~31);  // every TMEM column the epilogue loads is written
+          k_unit_end = t_hi - unit_first_item(p, u);
+        }
         int b;
         if (!(ok = take_buffer(b))) break;
         const int st = k % S2;
         if (!(ok = mbar_wait(&k_full[st], (par >> st) & 1u, abort_flag))) break;
         tc_fence_after();
         const uint32_t dcol = tmem_base + (uint32_t)(b * 256);
-        const int n_mma = (r.rows + 31) & ~31;  // every TMEM column the epilogue loads is written
-        const uint32_t idesc = umma_idesc_bf16(128, n_mma);
+        const uint64_t dK = dK0 + (uint64_t)(Cfg::chunk_off(st, 0) >> 4);
 #pragma unroll
         for (int kk = 0; kk < NCH * 4; ++kk) {
           const uint32_t qoff = (uint32_t)((kk >> 2) * kQChunkBytes + (kk & 3) * 32);
-          const uint32_t koff = (uint32_t)(Cfg::chunk_off(st, kk >> 2) + (kk & 3) * 32);
-          umma_bf16(dcol, umma_desc_sw128(smem_u32(sK) + koff), umma_desc_sw128(qst + qoff), idesc, kk > 0 ? 1u : 0u);
+          const uint32_t koff = (uint32_t)((kk >> 2) * 2 * kKChunkBytes + (kk & 3) * 32);  // within the stage
+          umma_bf16(dcol, dK + (koff >> 4), dQ0 + (qoff >> 4), idesc2, kk > 0 ? 1u : 0u);
         }
         umma_commit(&k_empty[st]);
         par ^= 1u << st;

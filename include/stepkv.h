@@ -407,8 +407,10 @@ STEPKV_API stepkv_status_t stepkv_selftest_score_timeout(int32_t n_layers, const
 /* ---------------------------------------------------------------------------------------------
  * The fused pass (score -> reduce/fuse -> select -> compact) for n_traj independent trajectories
  * (one pruning boundary each, Algorithm 1).  probs is a host array; everything runs on `stream`:
- * the saliency of each trajectory (one launch each), then the selections of all trajectories in one
- * launch (one 8-CTA cluster per trajectory, up to 16 per launch), then each compaction.  `ws` (size
+ * the saliencies (consecutive trajectories of one head shape share a launch, up to 16), then the
+ * selections of all trajectories in one launch (one 8-CTA cluster per trajectory, up to 16 per
+ * launch), then the compactions (out-of-place ones share launches; an in-place one is a single move
+ * launch that follows the hole-filling plan its selection wrote).  `ws` (size
  * from stepkv_compress_workspace_size over the same array) holds one shared region for the saliency
  * partials, a private region per trajectory, and one shared region for the saliency rows of a pooled
  * token saliency (params->sal_pool > 1: the rows of each trajectory are written, then pooled; the

@@ -664,6 +664,29 @@ def test_compress_in_place_hole_filling(B, T, num, den, all_prot):
         assert np.array_equal(TL.bits_of(g.V[l])[:, :n], src[1][l][:, exp])
 
 
+def test_compress_in_place_overflow_moves_nothing(B):
+    """In place with kept_cap below the retained count (Eq. 1's protected + budget rows): the call records
+    STEPKV_ENOSPACE on the device, lays out no plan, and leaves every layer's cache rows and the step /
+    position outputs as they were."""
+    import torch
+    tr = wl.custom(77, L=2, Hq=4, Hkv=2, d=64, T=3000, W=16, n_steps=10, budget=wl.Budget.ratio(1, 2))
+    n_prot = int(tr.prot.sum())
+    n_exp = n_prot + max(1, (tr.T - n_prot) // 2)
+    g = TL.GpuTraj(tr, kept_cap=n_exp - 7)
+    src = ([TL.bits_of(k) for k in g.K], [TL.bits_of(v) for v in g.V])
+    g.problem()
+    prob = B.Problem(g.K, g.V, g.Q, tr.T, g.step_id, g.prot, g.steps(), g.budget(), g.K, g.V, g.out,
+                     pos_in=g.pos, step_id_out=g.step_id_out, pos_out=g.pos_out)
+    st = B.stepkv_compress([prob], B.Params())
+    torch.cuda.synchronize()
+    assert st.item() == B.STEPKV_ENOSPACE
+    assert int(g.out.n_kept.item()) == n_exp
+    for l in range(tr.shape.L):
+        assert np.array_equal(TL.bits_of(g.K[l]), src[0][l])
+        assert np.array_equal(TL.bits_of(g.V[l]), src[1][l])
+    assert bool((g.step_id_out == -7).all()) and bool((g.pos_out == -7).all())
+
+
 def test_compress_minimal_outputs_same_selection(B):
     """Without the optional outputs (per-step statistics, priorities) the kernel skips their work; the
     retained set and the compacted rows are the same as with every output requested."""

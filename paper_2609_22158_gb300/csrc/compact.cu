@@ -2,8 +2,9 @@
 //   out[l][h][r][:] = in[l][h][kept_idx[r]][:]  for every layer, KV head and tensor (K, V)
 //
 // GB300 design: a pure HBM copy (about 4/5 of the pass's bytes).  The work is the list of row items
-// (row set, retained row), row set = (layer, tensor, KV head); a persistent grid of 8 CTAs per SM splits
-// it into equal contiguous ranges, so every SM streams the same number of rows.  A row of d bf16 is
+// (row set, retained row), row set = (layer, tensor, KV head); a grid of 8 CTAs per SM (4 resident at
+// this kernel's registers, so two waves; one wave of 4 measured the same) splits it into equal
+// contiguous ranges, so every SM streams the same number of rows.  A row of d bf16 is
 // d/8 16-byte vectors handled by d/8 lanes, so a warp moves 32/(d/8) rows per instruction; four such
 // groups are loaded before the first store (8 rows, 2 KB per warp in flight at d = 128).  Loads and
 // stores are streaming (.cs): the data is touched once.  n_kept is read on the device.

@@ -236,7 +236,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int rank = cl.rank();
   extern __shared__ __align__(16) uint8_t smem_raw[];
   // layout: [chunk] float/uint32 keys | [chunk] u16 step id (0xFFFF = protected) | 2 x 2048 int hist |
-  //         SelShared (own) | SelShared[NC] (gathered) | scratch[64] | coarse[2][64] | S_k (when s_in_smem)
+  //         SelShared (own) | SelShared[NC] (gathered) | scratch[64] | coarse[2][NC][64] | S_k (when s_in_smem)
   uint32_t* sKey = reinterpret_cast<uint32_t*>(smem_raw);
   float* sT = reinterpret_cast<float*>(smem_raw);
   uint16_t* sSid = reinterpret_cast<uint16_t*>(smem_raw + (size_t)a.chunk * 4);
@@ -245,8 +245,8 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   SelShared* all = ex + 1;
   int* scratch = reinterpret_cast<int*>(all + NC);  // 64 ints
   int* bcast = scratch + 48;                        // radix decision
-  int* coarse = scratch + 64;                       // 2 x 64 coarse counts (alternate passes)
-  float* sS = reinterpret_cast<float*>(coarse + 128);
+  int* allc = scratch + 64;                         // [2 passes][NC ranks][64] every CTA's coarse counts
+  float* sS = reinterpret_cast<float*>(allc + 2 * NC * 64);
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int T = a.T;
@@ -499,14 +499,16 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         if (hit && (__ffs(peers) - 1) == lane) atomicAdd(&h[bin], __popc(peers));
       }
       __syncthreads();
-      // this CTA's coarse counts: sums of 32 consecutive bins (64 coarse bins for 11 bits, 32 for 10)
-      int* hc = coarse + (pass & 1) * 64;
+      // this CTA's coarse counts: sums of 32 consecutive bins (64 coarse bins for 11 bits, 32 for 10),
+      // pushed into every CTA's table before the barrier (lane r stores into rank r), so the coarse step
+      // below reads them from its own shared memory
+      int* ac = allc + (pass & 1) * NC * 64;
       const int ncoarse = nb >> 5;
       for (int c = warp; c < ncoarse; c += NW) {
         int v = h[c * 32 + lane];
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        if (lane == 0) hc[c] = v;
+        if (lane < NC) cl.peer(ac, lane)[rank * 64 + c] = v;
       }
       cl.sync();  // every CTA's histogram and coarse counts of this pass are complete
       if (warp == 0) {
@@ -516,9 +518,8 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         int clo = 0, chi = 0;
 #pragma unroll
         for (int r = 0; r < NC; ++r) {
-          const int* pc = cl.peer(hc, r);
-          clo += pc[lane];
-          if (ncoarse > 32) chi += pc[32 + lane];
+          clo += ac[r * 64 + lane];
+          if (ncoarse > 32) chi += ac[r * 64 + 32 + lane];
         }
         const int shi = warp_suffix_sum(chi, lane);                                    // keys in bins >= 32 + l
         const int slo = warp_suffix_sum(clo, lane) + __shfl_sync(0xffffffffu, shi, 0);  // keys in bins >= l
@@ -811,7 +812,7 @@ static SelectArgs make_select_args(const SelectSpec& sp) {
 // scratch, and S_k when it fits.
 static size_t select_smem(int chunk, int nc, int n_steps, int* s_in_smem) {
   const size_t fixed = (((size_t)chunk * 6 + 15) & ~size_t(15)) + 2 * 2048 * 4 + (1 + nc) * sizeof(SelShared) +
-                       (64 + 128) * 4;
+                       (64 + 2 * (size_t)nc * 64) * 4;
   const size_t budget_smem = 232448 - 1024;
   *s_in_smem = fixed + (size_t)n_steps * 4 <= budget_smem ? 1 : 0;
   return fixed + (*s_in_smem ? (size_t)n_steps * 4 : 0);

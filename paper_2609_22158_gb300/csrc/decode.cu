@@ -138,6 +138,14 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
       kr[t] = ok[t] ? __ldcs(reinterpret_cast<const uint4*>(Kh + (size_t)j * D) + hl) : make_uint4(0, 0, 0, 0);
       vr[t] = ok[t] ? __ldcs(reinterpret_cast<const uint4*>(Vh + (size_t)j * D) + hl) : make_uint4(0, 0, 0, 0);
     }
+    // The warp's next block is fetched into L2 while this one is computed: the loads above wait for
+    // DRAM only until the pipeline fills, and the prefetch holds no registers.
+    const int kn = kb + kDecWarps * BLK;
+    if (lane == 0 && kn < k_end) {
+      const uint32_t nbytes = (uint32_t)(min(BLK, k_end - kn) * D * 2);
+      bulk_prefetch_l2(Kh + (size_t)kn * D, nbytes);
+      bulk_prefetch_l2(Vh + (size_t)kn * D, nbytes);
+    }
     float s[kDecBlockSteps][G];
 #pragma unroll
     for (int t = 0; t < kDecBlockSteps; ++t) {

@@ -51,7 +51,7 @@ MUFU_PER_CLK_SM = 32
 # current kernels on the 32K workload (profiles/launches_llama8b_32k.md, steady-state launches):
 # {config: {kernel: bytes}}.  A kernel absent here reports traffic null.
 NCU_TRAFFIC = {
-    2: {"score_kernel": 318.8e6 + 1.3e6, "select_kernel": 0.5e6, "compact_kernel": 438.9e6 + 388.3e6},
+    2: {"score_kernel": 318.8e6 + 1.1e6, "select_kernel": 0.5e6, "compact_kernel": 438.9e6 + 388.2e6},
 }
 
 

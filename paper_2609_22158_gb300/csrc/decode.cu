@@ -116,13 +116,16 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
 #pragma unroll
     for (int e = 0; e < 8; ++e) q[g][e] *= a.c;
   }
-  float m[G], l[G], acc[G][8];
+  // Value accumulators as packed fp32 pairs: a bf16 word holds two neighbouring elements, so a value row
+  // converts straight into pairs and every value FMA and rescale is one f32x2 instruction for two elements.
+  float m[G], l[G];
+  uint64_t accp[G][4];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
     m[g] = -INFINITY;
     l[g] = 0.f;
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc[g][e] = 0.f;
+    for (int e = 0; e < 4; ++e) accp[g][e] = 0ull;
   }
 
   const uint16_t* Kh = a.K[layer] + (size_t)h * a.head_stride;
@@ -218,7 +221,7 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
       const float sc = ex2_approx(m[g] - mb);
       l[g] *= sc;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[g][e] *= sc;
+      for (int e = 0; e < 4; ++e) accp[g][e] = f2_mul(accp[g][e], f2_pack(sc, sc));
 #pragma unroll
       for (int t = 0; t < kDecBlockSteps; ++t) {
         p[t][g] = ex2_approx(s[t][g] - mb);
@@ -228,14 +231,23 @@ __global__ void __launch_bounds__(kDecThreads) decode_partial_kernel(const __gri
     }
 #pragma unroll
     for (int t = 0; t < kDecBlockSteps; ++t) {
-      float vf[8];
-      bf16x8_to_f32(vr[t], vf);
+      const uint32_t w[4] = {vr[t].x, vr[t].y, vr[t].z, vr[t].w};
+      uint64_t vp[4];
 #pragma unroll
-      for (int g = 0; g < G; ++g)
+      for (int e = 0; e < 4; ++e) vp[e] = f2_pack(__uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xFFFF0000u));
 #pragma unroll
-        for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p[t][g], vf[e], acc[g][e]);
+      for (int g = 0; g < G; ++g) {
+        const uint64_t pp = f2_pack(p[t][g], p[t][g]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) accp[g][e] = f2_fma(vp[e], pp, accp[g][e]);
+      }
     }
   }
+  float acc[G][8];
+#pragma unroll
+  for (int g = 0; g < G; ++g)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) f2_unpack(accp[g][e], acc[g][2 * e], acc[g][2 * e + 1]);
   // merge the key slots of the warp (lanes with the same hl), then the warps through shared memory
 #pragma unroll
   for (int o = LPK; o < 32; o <<= 1) {

@@ -77,6 +77,24 @@ def test_score_rejects_bad_arguments_on_host(lib):
     assert lib.stepkv_score(1, p, 128 * 99, p, 128 * 10, 2, 8, 128, 100, 10, 4096, ws, 1 << 30, None, None) == STEPKV_EINVAL
 
 
+def test_score_lse_rejects_bad_statistics_on_host(lib):
+    """stepkv_score_lse checks the per-layer row log-sum-exp pointers (present, 4-byte aligned) on the host,
+    after the arguments it shares with stepkv_score, before anything is enqueued."""
+    from paper_2609_22158_gb300.binding import STEPKV_EINVAL, STEPKV_EUNSUPPORTED
+    kq = (ctypes.c_void_p * 2)(256, 512)
+    p = ctypes.cast(kq, ctypes.c_void_p)
+    ws = ctypes.c_void_p(1 << 20)
+    sal = ctypes.c_void_p(4096)
+    call = lambda lse, n_layers=2, sal_=sal: lib.stepkv_score_lse(n_layers, p, 128 * 100, p, 128 * 10, lse, 2, 8, 128,
+                                                                   100, 10, sal_, ws, 1 << 30, None, None)
+    assert call(None) == STEPKV_EINVAL                                               # no statistics at all
+    assert call(ctypes.cast((ctypes.c_void_p * 2)(1024, None), ctypes.c_void_p)) == STEPKV_EINVAL   # layer 1 missing
+    assert call(ctypes.cast((ctypes.c_void_p * 2)(1024, 1026), ctypes.c_void_p)) == STEPKV_EINVAL   # misaligned
+    good = ctypes.cast((ctypes.c_void_p * 2)(1024, 2048), ctypes.c_void_p)
+    assert call(good, sal_=None) == STEPKV_EINVAL                                    # no output
+    assert call(good, n_layers=9) == STEPKV_EUNSUPPORTED                             # the shared checks come first
+
+
 def test_select_rejects_bad_arguments_on_host(lib):
     from paper_2609_22158_gb300 import binding as B
     steps = B.CSteps(0, 256, 256, 256, None, 256, None)
